@@ -1,0 +1,430 @@
+"""Decode-attention throughput over a compressed KV cache on one GB300.
+
+One step = one decode step of the whole hot path over all 32 layers of a
+Llama-3-8B-shaped attention (32 query / 8 KV heads, D = 128) for the batch:
+per layer, append the new token to the compressed cache (KVQuant: quantize it)
+and run decode attention over the cache.  tokens/s = batch / step time.
+
+Default workload: KVQuant NUQ 4-bit, B = 8, context 8192 (the KVQuant decode
+configuration); other workloads via --workload.  Inputs are synthetic and
+seeded (synth), every layer has its own cache buffers, and one step reads
+more than the 129 MB L2 holds, so no flush is needed between steps.
+
+Under torchrun each rank runs an independent replica on its own GPU (the
+units -- batch entries, heads, layers -- are independent; no collective).
+--impl reference times the fp64 CPU oracle on a bounded sample instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+for _v in ("OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "OMP_NUM_THREADS"):
+    os.environ.setdefault(_v, "1")          # the CPU oracle runs on one core
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+WORKLOADS = {
+    "kvquant4": lambda: synth.kvquant_8k(4),
+    "kvquant3": lambda: synth.kvquant_8k(3),
+    "kvquant2": lambda: synth.kvquant_8k(2),
+    "fp16": lambda: synth.Workload(name="fp16_b8_t8192", B=8, L=32, Hq=32, Hkv=8, D=128, T=8192, steps=128),
+    "h2o20": lambda: synth.h2o_16k(20),
+    "rocket1024": lambda: synth.rocket_32k(1024),
+}
+METHOD_OF = {"kvquant4": "kvquant", "kvquant3": "kvquant", "kvquant2": "kvquant", "fp16": "fp16",
+             "h2o20": "h2o", "rocket1024": "rocket"}
+METRIC = "compressed-KV decode attn tokens/s and HBM GB/s (fraction of ~8 TB/s) per config"
+
+
+# --------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples (200 ms) during the timed region."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) == 7:
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait()
+        self.thread.join(timeout=2)
+        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[3 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.rows)}
+
+
+# --------------------------------------------------------------------------- GPU arm
+
+class Runner:
+    """All layers of one workload resident on the device, plus the step."""
+
+    def __init__(self, name: str, w, dev, seed: int, extra_steps: int):
+        import torch
+        import paper_2609_07966_gb300 as mkv
+        from paper_2609_07966_gb300 import caches
+        self.torch, self.mkv, self.name, self.w, self.dev = torch, mkv, name, w, dev
+        self.method = METHOD_OF[name]
+        B, Hq, Hkv, D = w.B, w.Hq, w.Hkv, w.D
+        self.T_cap = w.T + extra_steps + 64
+        mk = {"fp16": mkv.MKV_FP16, "kvquant": mkv.MKV_KVQUANT, "h2o": mkv.MKV_H2O, "rocket": mkv.MKV_ROCKET}
+        kw = {}
+        if self.method == "kvquant":
+            kw = dict(bits=w.bits, quant_mode=mkv.MKV_QUANT_NUQ if w.quant_mode == "nuq" else mkv.MKV_QUANT_UNIFORM,
+                      outlier_frac=w.outlier_frac, rope_theta=w.theta)
+        self.cfg = mkv.config(mk[self.method], B, Hq, Hkv, D, **kw)
+        self.layers = []
+        self.q, self.kn, self.vn, self.out = [], [], [], []
+        ws_cap = self.T_cap
+        self.ws, self.nws = caches.workspace(self.cfg, ws_cap, device=dev)
+        if self.method == "kvquant":
+            self.rope = torch.empty((self.T_cap, D // 2, 2), dtype=torch.float32, device=dev)
+            mkv.mkv_rope_table(D, w.theta, self.T_cap, self.rope.data_ptr())
+        for l in range(w.L):
+            x = synth.device_layer_inputs(w, seed, l, device=dev, n_tokens=w.T + 1)
+            cache = caches.alloc_cache(self.cfg, self.T_cap, device=dev)
+            qp = None
+            if self.method == "fp16":
+                cache.t["k"][:, :, :w.T] = x["k"][:, :, :w.T]
+                cache.t["v"][:, :, :w.T] = x["v"][:, :, :w.T]
+                cache.t["T_len"].fill_(w.T)
+            elif self.method == "kvquant":
+                qp = caches.alloc_quant_params(self.cfg, 1, device=dev)
+                qp.t["rope"] = self.rope
+                qp.c.rope = self.rope.data_ptr()
+                qp.c.rope_len = self.T_cap
+                ncal = min(w.T, 4096)
+                k0, v0 = x["k"][0].contiguous(), x["v"][0].contiguous()     # batch entry 0 calibrates
+                mkv.mkv_kvquant_calibrate(self.cfg, k0.data_ptr(), v0.data_ptr(), ncal, w.T + 1, qp.c,
+                                          self.ws.data_ptr(), self.nws)
+                kp = x["k"][:, :, :w.T].contiguous()
+                vp = x["v"][:, :, :w.T].contiguous()
+                mkv.mkv_quantize_kv(self.cfg, qp.c, kp.data_ptr(), vp.data_ptr(), w.T, cache.c)
+                del kp, vp
+            self.layers.append((cache, qp))
+            self.q.append(x["q"][0].contiguous())
+            self.kn.append(x["k"][:, :, w.T].contiguous())
+            self.vn.append(x["v"][:, :, w.T].contiguous())
+            self.out.append(torch.empty((B, Hq, D), dtype=torch.float16, device=dev))
+            del x
+        torch.cuda.synchronize()
+        flags = mkv.mkv_get_status()
+        assert flags == 0, f"device status flags {flags:#x} after setup"
+        self.graph = None
+
+    def layer_step(self, l, q=None, kn=None, vn=None, out=None):
+        mkv = self.mkv
+        cache, qp = self.layers[l]
+        q = self.q[l] if q is None else q
+        kn = self.kn[l] if kn is None else kn
+        vn = self.vn[l] if vn is None else vn
+        out = self.out[l] if out is None else out
+        if self.method == "kvquant":
+            mkv.mkv_quantize_kv(self.cfg, qp.c, kn.data_ptr(), vn.data_ptr(), 1, cache.c)
+            mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, qp.c, 0, out.data_ptr(), self.ws.data_ptr(),
+                                     self.nws)
+        else:
+            mkv.mkv_append_kv(self.cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
+            mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, None, 0, out.data_ptr(), self.ws.data_ptr(),
+                                     self.nws)
+
+    def step(self):
+        for l in range(self.w.L):
+            self.layer_step(l)
+
+    def capture(self):
+        torch = self.torch
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            self.step()                          # warm the launch paths outside capture
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            self.step()
+        torch.cuda.synchronize()
+
+    def run_step(self):
+        if self.graph is not None:
+            self.graph.replay()
+        else:
+            self.step()
+
+    def launches_per_step(self):
+        # per layer: append (1 kernel) + decode (1) + combine (1)
+        return 3 * self.w.L
+
+    def decode_bytes(self):
+        """Algorithmic bytes one decode launch reads for one layer at the current lengths."""
+        w = self.w
+        cache, _ = self.layers[0]
+        T = int(cache.t["T_len"][0])
+        units = w.B * w.Hkv
+        if self.method == "fp16":
+            return units * T * w.D * 2 * 2, T
+        if self.method == "kvquant":
+            nv = self.mkv.n_value_outliers(w.D, w.outlier_frac)
+            per_tok = 2 * (w.D * w.bits // 8) + 8 + 4 * nv + 4
+            n_kout = int(cache.t["k_out_off"][:, :, T].sum())
+            return units * T * per_tok + 4 * n_kout, T
+        raise NotImplementedError(self.method)
+
+
+def time_steps(runner, steps, warmup):
+    torch = runner.torch
+    for _ in range(warmup):
+        runner.run_step()
+    torch.cuda.synchronize()
+    st = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    for _ in range(steps):
+        runner.run_step()
+    e1.record(st)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def time_decode_launches(runner, steps):
+    """Average duration of one mkv_decode_attention call (decode + combine kernels),
+    CUDA events on the launching stream around each call, eager."""
+    torch, mkv = runner.torch, runner.mkv
+    st = torch.cuda.current_stream()
+    evs = []
+    for _ in range(steps):
+        for l in range(runner.w.L):
+            cache, qp = runner.layers[l]
+            if runner.method == "kvquant":
+                mkv.mkv_quantize_kv(runner.cfg, qp.c, runner.kn[l].data_ptr(), runner.vn[l].data_ptr(), 1, cache.c)
+            else:
+                mkv.mkv_append_kv(runner.cfg, runner.kn[l].data_ptr(), runner.vn[l].data_ptr(), cache.c)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(st)
+            mkv.mkv_decode_attention(runner.cfg, runner.q[l].data_ptr(), cache.c, qp.c if qp else None, 0,
+                                     runner.out[l].data_ptr(), runner.ws.data_ptr(), runner.nws)
+            b.record(st)
+            evs.append((a, b))
+    torch.cuda.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in evs)
+
+
+def time_e2e(runner, steps, warmup):
+    """Through the public API with host buffers: per step, H2D of every layer's q and
+    new k/v from pinned memory, the step, and D2H of every layer's output."""
+    torch = runner.torch
+    w = runner.w
+    hq = [t.cpu().pin_memory() for t in runner.q]
+    hk = [t.cpu().pin_memory() for t in runner.kn]
+    hv = [t.cpu().pin_memory() for t in runner.vn]
+    ho = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in runner.out]
+    dq = [torch.empty_like(t) for t in runner.q]
+    dk = [torch.empty_like(t) for t in runner.kn]
+    dv = [torch.empty_like(t) for t in runner.vn]
+
+    def one():
+        for l in range(w.L):
+            dq[l].copy_(hq[l], non_blocking=True)
+            dk[l].copy_(hk[l], non_blocking=True)
+            dv[l].copy_(hv[l], non_blocking=True)
+            runner.layer_step(l, dq[l], dk[l], dv[l], runner.out[l])
+            ho[l].copy_(runner.out[l], non_blocking=True)
+
+    for _ in range(warmup):
+        one()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one()
+    torch.cuda.synchronize()
+    dt = (time.perf_counter() - t0) / steps
+    h2d = sum(t.numel() * t.element_size() for t in hq + hk + hv)
+    d2h = sum(t.numel() * t.element_size() for t in ho)
+    return dt, h2d, d2h
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d.get("hbm_gbs", 6800.0), "measured"
+    return 6800.0, "fallback"
+
+
+# --------------------------------------------------------------------------- CPU oracle arm
+
+def oracle_tokens_per_s(name: str, w, budget_s: float, seed: int = 0):
+    """The fp64 oracle's decode step, timed on one (layer, batch, kv-head) unit of the
+    workload repeated until ``budget_s`` seconds of oracle work; scaled to the step.
+
+    Returns (tokens/s for the whole workload, sample description)."""
+    from oracle import attention, kvquant
+    method = METHOD_OF[name]
+    rng = np.random.default_rng(seed)
+    T = w.T
+    scale = np.exp(rng.uniform(np.log(0.1), np.log(10), w.D)) if method == "kvquant" else 1.0
+    k = (rng.standard_normal((T + 1, w.D)) * scale).astype(np.float16)
+    v = rng.standard_normal((T + 1, w.D)).astype(np.float16)
+    q = rng.standard_normal((w.G, w.D)).astype(np.float16)
+    if method == "kvquant":
+        p = kvquant.calibrate(k[:min(T, 4096)], v[:min(T, 4096)], w.bits, w.quant_mode, w.outlier_frac)
+        qh = kvquant.quantize_head(k[:T], v[:T], p)
+
+        def unit():
+            new = kvquant.quantize_head(k[T:T + 1], v[T:T + 1], p)     # the step's append
+            full = kvquant.QuantizedHead(*[np.concatenate([a, b]) for a, b in zip(
+                (qh.k_codes, qh.k_mask, qh.k_raw, qh.v_codes, qh.v_mask, qh.v_lo, qh.v_scale, qh.v_raw),
+                (new.k_codes, new.k_mask, new.k_raw, new.v_codes, new.v_mask, new.v_lo, new.v_scale, new.v_raw))])
+            kvquant.decode_head(q, full, p, w.theta)
+    else:
+        def unit():
+            attention.attend(q, k, v)
+    t_units, n_units = 0.0, 0
+    while t_units < budget_s and n_units < 1000:
+        t0 = time.perf_counter()
+        unit()
+        t_units += time.perf_counter() - t0
+        n_units += 1
+    per_unit = t_units / n_units
+    step_s = per_unit * w.B * w.Hkv * w.L
+    sample = (f"{n_units} decodes of one (layer, batch, kv-head) unit of {name} at T={T} "
+              f"({per_unit * 1e3:.1f} ms each), scaled to the step's B*Hkv*L={w.B * w.Hkv * w.L} units")
+    return w.B / step_s, sample
+
+
+# --------------------------------------------------------------------------- main
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="mkv", choices=["mkv", "reference"])
+    ap.add_argument("--workload", default="kvquant4", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--seed", type=int, default=0)
+    args = ap.parse_args()
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    w = WORKLOADS[args.workload]()
+    config = {"workload": w.name, "method": METHOD_OF[args.workload], "batch": w.B, "context": w.T, "layers": w.L,
+              "heads_q": w.Hq, "heads_kv": w.Hkv, "head_dim": w.D, "l2": "inputs larger than L2 (no flush)"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        steps = max(1, args.steps)
+        vals, sample = [], ""
+        budget = min(args.cpu_budget, 120.0 / (steps + args.warmup))
+        for i in range(args.warmup + steps):
+            v, sample = oracle_tokens_per_s(args.workload, w, budget, seed=args.seed + i)
+            if i >= args.warmup:
+                vals.append(v)
+        value = statistics.mean(vals)
+        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+                "steps": steps, "warmup": args.warmup, "ms_per_step": 1e3 * w.B / value,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic", "config": config,
+                "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample},
+                "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    import torch
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+
+    total = args.warmup + args.steps
+    runner = Runner(args.workload, w, dev, args.seed + rank, extra_steps=4 * total + 8)
+    if not args.no_graph:
+        runner.capture()
+
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+    ms = time_steps(runner, args.steps, args.warmup)
+    clk = clocks.stop()
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+        torch.distributed.barrier()
+
+    alg_bytes, T_now = runner.decode_bytes()
+    dec_ms = time_decode_launches(runner, max(1, min(args.steps, 5)))
+    e2e_s, h2d, d2h = time_e2e(runner, max(1, min(args.steps, 5)), 1)
+    peak, peak_kind = peaks()
+    achieved = alg_bytes / (dec_ms * 1e-3) / 1e9
+    value = w.B * world / (ms * 1e-3)
+    line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f16" if runner.method != "kvquant" else f"u{w.bits}+f16",
+            "data": "synthetic (seeded, device-generated)", "config": config,
+            "gpu_launches": runner.launches_per_step() * args.steps,
+            "e2e": {"value": w.B * world / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "kernel": "mkv_decode_attention (decode + combine), one layer",
+                         "peak_kind": peak_kind, "frac_of_8000": achieved / 8000.0,
+                         "alg_bytes_per_launch": alg_bytes, "context_at_measure": T_now,
+                         "avg_launch_ms": dec_ms},
+            "clocks": clk}
+    if rank == 0:
+        if world == 1:
+            v, sample = oracle_tokens_per_s(args.workload, w, args.cpu_budget, seed=args.seed)
+            line["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample}
+        print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

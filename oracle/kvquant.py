@@ -109,29 +109,27 @@ def midpoints(cb16) -> np.ndarray:
 
 
 def value_outlier_mask(x16, n_v: int):
-    """[n, D] bool: the n_v entries of largest |x| per row (ties: lower channel)."""
+    """[n, D] bool: the n_v entries of largest |x| per row (ties: lower channel).
+
+    A stable sort on -|x| keeps equal magnitudes in channel order.
+    """
     x = np.asarray(x16, dtype=np.float16).astype(np.float64)
     n, D = x.shape
     mask = np.zeros((n, D), dtype=bool)
     if n_v <= 0:
         return mask
-    ch = np.arange(D)
-    for t in range(n):
-        order = np.lexsort((ch, -np.abs(x[t])))
-        mask[t, order[:n_v]] = True
+    order = np.argsort(-np.abs(x), axis=1, kind="stable")
+    np.put_along_axis(mask, order[:, :n_v], True, axis=1)
     return mask
 
 
 def value_range(x16, mask):
     """Per-row fp32 (lo, hi) over inliers (0, 0 when a row has no inlier)."""
     x = np.asarray(x16, dtype=np.float16).astype(F32)
-    lo = np.zeros(x.shape[0], F32)
-    hi = np.zeros(x.shape[0], F32)
-    for t in range(x.shape[0]):
-        inl = x[t][~mask[t]]
-        if inl.size:
-            lo[t], hi[t] = inl.min(), inl.max()
-    return lo, hi
+    has = (~mask).any(axis=1)
+    lo = np.where(mask, F32(np.inf), x).min(axis=1).astype(F32)
+    hi = np.where(mask, F32(-np.inf), x).max(axis=1).astype(F32)
+    return np.where(has, lo, F32(0)).astype(F32), np.where(has, hi, F32(0)).astype(F32)
 
 
 def normalized(x16, lo, s):

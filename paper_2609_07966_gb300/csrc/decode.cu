@@ -1,0 +1,356 @@
+// Decode attention over an fp16 cache: FP16 (all slots), H2O (kept slots,
+// with per-slot logits for the score update) and the RocketKV sparse stage
+// (selected pages + tail page).  Section 2.1 of the paper; the operation is
+//   out_h = sum_t softmax_t(scale q_h . k_t) v_t  over the attended set.
+//
+// Design (GB300, HBM-bound): one CTA per (batch, kv-head, split) holds all G
+// query heads of the group, so every K/V byte is read once.  K and V rows are
+// staged by cp.async into XOR-swizzled shared tiles (3-stage pipeline of 64
+// tokens), and each warp multiplies its 16 tokens with one m16n8k16 tensor-
+// core product per 16 dims (G query rows padded to 16): the contraction costs
+// ~5 warp instructions per token, leaving the issue slots to the copies.
+// Online softmax runs in the log2 domain on the accumulator fragments; splits
+// are merged by combine_kernel.
+#include <math.h>
+
+#include "mkv_common.cuh"
+#include "mkv_internal.h"
+
+namespace mkv {
+
+namespace {
+
+constexpr int kStages = 3;
+constexpr int kThreads = 128;   // 4 warps x 16 tokens = one 64-token chunk
+
+struct Fp16Args {
+  const __half* q;        // [B][Hq][D]
+  const __half* k;        // [B][Hkv][T_cap][D]
+  const __half* v;
+  const int32_t* T_len;   // [B]
+  const int32_t* pos;     // H2O [B][Hkv][T_cap]
+  const int32_t* page_idx;// ROCKET [B][Hkv][kp]
+  int64_t T_cap;
+  int Hq, Hkv, G;
+  int chunks_per_split;
+  int kp;
+  float scale_log2;
+  float* part_m;
+  float* part_l;
+  float* part_o;
+  float* logits;          // H2O [B][Hkv][T_cap][G]
+  int n_split;
+};
+
+// Virtual token v of (b, kv-head) -> cache slot, or -1 when v attends nothing.
+template <int MODE>
+__device__ __forceinline__ int64_t slot_of(const Fp16Args& a, int64_t v, int64_t bh, int n_len, int ns) {
+  if (MODE == 0) {                       // FP16: slots 0..T_len-1
+    return v < n_len ? v : -1;
+  } else if (MODE == 1) {                // H2O: slots holding a position
+    if (v >= a.T_cap) return -1;
+    return a.pos[bh * a.T_cap + v] >= 0 ? v : -1;
+  } else {                               // ROCKET: selected pages, then the tail page
+    const int unit = (int)(v / kPage), within = (int)(v % kPage);
+    if (unit < a.kp) {
+      const int p = a.page_idx[bh * a.kp + unit];
+      return p >= 0 ? (int64_t)p * kPage + within : -1;
+    }
+    if (unit == a.kp) {
+      const int64_t s = (int64_t)ns * kPage + within;
+      return s < n_len ? s : -1;
+    }
+    return -1;
+  }
+}
+
+template <int D, int MODE>
+__global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args a) {
+  constexpr int ROWB = D * 2;           // bytes per token row
+  constexpr int NC = D / 8;             // 16-byte chunks per row
+  constexpr int TILE = kChunk * ROWB;   // one K (or V) tile
+  constexpr int KC = D / 16;            // k16 steps of the QK product
+  constexpr int ROWS_PER_PASS = kThreads / NC;
+  extern __shared__ __align__(128) uint8_t smem[];
+  int32_t* slotmap = reinterpret_cast<int32_t*>(smem + kStages * 2 * TILE);   // [kStages][kChunk]
+
+  const int split = blockIdx.x;
+  const int64_t bh = blockIdx.y;
+  const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, r = lane & 3;
+
+  int n_len = 0, ns = 0;
+  int64_t v_total;
+  if (MODE == 0) {
+    n_len = a.T_len[b];
+    v_total = n_len;
+  } else if (MODE == 1) {
+    v_total = a.T_cap;
+  } else {
+    n_len = a.T_len[b];
+    ns = n_len > 0 ? (n_len - 1) / kPage : 0;
+    v_total = (int64_t)(a.kp + 1) * kPage;
+  }
+  const int64_t v_begin = (int64_t)split * a.chunks_per_split * kChunk;
+  int64_t v_end = v_begin + (int64_t)a.chunks_per_split * kChunk;
+  if (v_end > v_total) v_end = v_total;
+  const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
+
+  const __half* kbase = a.k + bh * a.T_cap * D;
+  const __half* vbase = a.v + bh * a.T_cap * D;
+
+  auto load_chunk = [&](int c, int stage) {
+    uint8_t* Ks = smem + stage * 2 * TILE;
+    uint8_t* Vs = Ks + TILE;
+    const int col = tid % NC;
+    for (int rr = tid / NC; rr < kChunk; rr += ROWS_PER_PASS) {
+      const int64_t v = v_begin + (int64_t)c * kChunk + rr;
+      const int64_t s = v < v_end ? slot_of<MODE>(a, v, bh, n_len, ns) : -1;
+      const int64_t ss = s >= 0 ? s : 0;
+      const int off = rr * ROWB + ((col ^ (rr & 7)) << 4);
+      cp_async16(Ks + off, kbase + ss * D + col * 8, s >= 0 ? 16 : 0);
+      cp_async16(Vs + off, vbase + ss * D + col * 8, s >= 0 ? 16 : 0);
+      if (col == 0) slotmap[stage * kChunk + rr] = (int32_t)s;
+    }
+  };
+
+  // query fragments: row g of the 16-row A operand is query head kvh*G + g
+  uint32_t qa0[KC], qa2[KC];
+  {
+    const bool real = g < a.G;
+    const __half* qrow = a.q + ((int64_t)b * a.Hq + (int64_t)kvh * a.G + (real ? g : 0)) * D;
+#pragma unroll
+    for (int kc = 0; kc < KC; ++kc) {
+      qa0[kc] = real ? *reinterpret_cast<const uint32_t*>(qrow + kc * 16 + 2 * r) : 0u;
+      qa2[kc] = real ? *reinterpret_cast<const uint32_t*>(qrow + kc * 16 + 2 * r + 8) : 0u;
+    }
+  }
+
+  float o[D / 8][2];
+#pragma unroll
+  for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = 0.f;
+  float m_run = -INFINITY, l_part = 0.f;
+
+#pragma unroll
+  for (int s = 0; s < kStages - 1; ++s) {
+    if (s < nchunks) load_chunk(s, s);
+    cp_async_commit();
+  }
+
+  for (int c = 0; c < nchunks; ++c) {
+    cp_async_wait<kStages - 2>();
+    __syncthreads();
+    {
+      const int nc = c + kStages - 1;
+      if (nc < nchunks) load_chunk(nc, nc % kStages);
+      cp_async_commit();
+    }
+    const int stage = c % kStages;
+    const uint8_t* Ks = smem + stage * 2 * TILE;
+    const uint8_t* Vs = Ks + TILE;
+    const int32_t* smap = slotmap + stage * kChunk;
+    const int t0 = warp * 16;
+
+    float sc[2][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) sc[0][i] = sc[1][i] = 0.f;
+    {
+      const int mi = lane >> 3, row = lane & 7;
+      const int tok = t0 + (mi >> 1) * 8 + row;
+      const uint8_t* rowp = Ks + tok * ROWB;
+#pragma unroll
+      for (int kc = 0; kc < KC; ++kc) {
+        uint32_t bk[4];
+        const int ch = kc * 2 + (mi & 1);
+        ldsm_x4(bk, rowp + ((ch ^ (tok & 7)) << 4));
+        mma16816(sc[0], qa0[kc], 0u, qa2[kc], 0u, bk[0], bk[1]);
+        mma16816(sc[1], qa0[kc], 0u, qa2[kc], 0u, bk[2], bk[3]);
+      }
+    }
+    // tokens of this lane's four scores
+    const int tk[4] = {t0 + 2 * r, t0 + 2 * r + 1, t0 + 8 + 2 * r, t0 + 9 + 2 * r};
+    float x[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
+    float mx = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int32_t s = smap[tk[i]];
+      x[i] = s >= 0 ? x[i] * a.scale_log2 : -INFINITY;
+      if (MODE == 1 && g < a.G && s >= 0) a.logits[(bh * a.T_cap + s) * a.G + g] = x[i];
+      mx = fmaxf(mx, x[i]);
+    }
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+    const float m_new = fmaxf(m_run, mx);
+    float p[4];
+    float alpha = 1.f;
+    if (m_new == -INFINITY) {
+      p[0] = p[1] = p[2] = p[3] = 0.f;
+    } else {
+      alpha = exp2f(m_run - m_new);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) p[i] = exp2f(x[i] - m_new);
+    }
+    l_part = l_part * alpha + (p[0] + p[1]) + (p[2] + p[3]);
+    m_run = m_new;
+    if (__any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+      for (int i = 0; i < D / 8; ++i) {
+        o[i][0] *= alpha;
+        o[i][1] *= alpha;
+      }
+    }
+    const uint32_t pa0 = pack_half2(p[0], p[1]);
+    const uint32_t pa2 = pack_half2(p[2], p[3]);
+    {
+      const int mi = lane >> 3, row = lane & 7;
+      const int tok = t0 + (mi & 1) * 8 + row;
+      const uint8_t* rowp = Vs + tok * ROWB;
+#pragma unroll
+      for (int j = 0; j < D / 16; ++j) {
+        uint32_t bv[4];
+        const int ch = 2 * j + (mi >> 1);
+        ldsm_x4_t(bv, rowp + ((ch ^ (tok & 7)) << 4));
+        float d0[4] = {o[2 * j][0], o[2 * j][1], 0.f, 0.f};
+        float d1[4] = {o[2 * j + 1][0], o[2 * j + 1][1], 0.f, 0.f};
+        mma16816(d0, pa0, 0u, pa2, 0u, bv[0], bv[1]);
+        mma16816(d1, pa0, 0u, pa2, 0u, bv[2], bv[3]);
+        o[2 * j][0] = d0[0];
+        o[2 * j][1] = d0[1];
+        o[2 * j + 1][0] = d1[0];
+        o[2 * j + 1][1] = d1[1];
+      }
+    }
+  }
+  cp_async_wait<0>();
+  __syncthreads();
+
+  // merge the four warps' (m, l, o) of each query row, then write the split partial
+  l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
+  l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
+  float* wm = reinterpret_cast<float*>(smem);          // [4][8]
+  float* wl = wm + 32;                                 // [4][8]
+  float* wo = wl + 32;                                 // [4][8][D]
+  if (g < a.G) {
+    if (r == 0) {
+      wm[warp * 8 + g] = m_run;
+      wl[warp * 8 + g] = l_part;
+    }
+#pragma unroll
+    for (int i = 0; i < D / 8; ++i) {
+      wo[(warp * 8 + g) * D + i * 8 + 2 * r] = o[i][0];
+      wo[(warp * 8 + g) * D + i * 8 + 2 * r + 1] = o[i][1];
+    }
+  }
+  __syncthreads();
+  for (int e = tid; e < a.G * D; e += kThreads) {
+    const int row = e / D, d = e % D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w * 8 + row]);
+    float L = 0.f, O = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const float f = exp2f(wm[w * 8 + row] - M);
+        L += wl[w * 8 + row] * f;
+        O += wo[(w * 8 + row) * D + d] * f;
+      }
+    }
+    const int64_t hq = (int64_t)b * a.Hq + (int64_t)kvh * a.G + row;
+    const int64_t pi = hq * a.n_split + split;
+    a.part_o[pi * D + d] = O;
+    if (d == 0) {
+      a.part_m[pi] = M;
+      a.part_l[pi] = L;
+    }
+  }
+}
+
+// out[b][h] = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s   (grid B*Hq, D threads)
+__global__ void combine_kernel(const float* __restrict__ part_m, const float* __restrict__ part_l,
+                               const float* __restrict__ part_o, int n_split, int D,
+                               __half* __restrict__ out, float* __restrict__ m_tot,
+                               float* __restrict__ l_tot) {
+  const int64_t hq = blockIdx.x;
+  const int d = threadIdx.x;
+  const float* pm = part_m + hq * n_split;
+  const float* pl = part_l + hq * n_split;
+  float M = -INFINITY;
+  for (int s = 0; s < n_split; ++s) M = fmaxf(M, pm[s]);
+  float L = 0.f, O = 0.f;
+  if (M != -INFINITY) {
+    for (int s = 0; s < n_split; ++s) {
+      const float ms = pm[s];
+      if (ms == -INFINITY) continue;
+      const float f = exp2f(ms - M);
+      L += pl[s] * f;
+      O += part_o[(hq * n_split + s) * D + d] * f;
+    }
+  }
+  out[hq * D + d] = __float2half_rn(L > 0.f ? O / L : 0.f);
+  if (m_tot != nullptr && d == 0) {
+    m_tot[hq] = M;
+    l_tot[hq] = L;
+  }
+}
+
+template <int D, int MODE>
+cudaError_t launch_fp16_t(const Fp16Args& a, int n_units, int n_split, cudaStream_t st) {
+  constexpr int TILE = kChunk * D * 2;
+  const size_t smem = (size_t)kStages * 2 * TILE + kStages * kChunk * sizeof(int32_t);
+  cudaError_t e = cudaFuncSetAttribute(decode_fp16_kernel<D, MODE>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid(n_split, n_units);
+  decode_fp16_kernel<D, MODE><<<grid, kThreads, smem, st>>>(a);
+  return cudaPeekAtLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const mkv_cache& cache,
+                                      const int32_t* page_idx, void* out, const DecodeWs& ws,
+                                      const Split& sp, cudaStream_t st) {
+  (void)out;
+  Fp16Args a{};
+  a.q = static_cast<const __half*>(q);
+  a.k = static_cast<const __half*>(cache.k);
+  a.v = static_cast<const __half*>(cache.v);
+  a.T_len = cache.T_len;
+  a.pos = cache.pos;
+  a.page_idx = page_idx;
+  a.T_cap = cache.T_cap;
+  a.Hq = c.Hq;
+  a.Hkv = c.Hkv;
+  a.G = c.Hq / c.Hkv;
+  a.chunks_per_split = sp.chunks_per_split;
+  a.kp = c.topk_pages;
+  const float scale = c.softmax_scale > 0.f ? c.softmax_scale : 1.0f / sqrtf((float)c.D);
+  a.scale_log2 = scale * kLog2e;
+  a.part_m = ws.part_m;
+  a.part_l = ws.part_l;
+  a.part_o = ws.part_o;
+  a.logits = ws.logits;
+  a.n_split = sp.n_split;
+  const int units = c.B * c.Hkv;
+  const int mode = c.method == MKV_H2O ? 1 : (c.method == MKV_ROCKET ? 2 : 0);
+  if (c.D == 128) {
+    if (mode == 0) return launch_fp16_t<128, 0>(a, units, sp.n_split, st);
+    if (mode == 1) return launch_fp16_t<128, 1>(a, units, sp.n_split, st);
+    return launch_fp16_t<128, 2>(a, units, sp.n_split, st);
+  }
+  if (mode == 0) return launch_fp16_t<64, 0>(a, units, sp.n_split, st);
+  if (mode == 1) return launch_fp16_t<64, 1>(a, units, sp.n_split, st);
+  return launch_fp16_t<64, 2>(a, units, sp.n_split, st);
+}
+
+cudaError_t launch_combine(const mkv_config& c, const DecodeWs& ws, const Split& sp, void* out,
+                           bool h2o_stats, cudaStream_t st) {
+  combine_kernel<<<c.B * c.Hq, c.D, 0, st>>>(ws.part_m, ws.part_l, ws.part_o, sp.n_split, c.D,
+                                             static_cast<__half*>(out), h2o_stats ? ws.m_tot : nullptr,
+                                             h2o_stats ? ws.l_tot : nullptr);
+  return cudaPeekAtLastError();
+}
+
+}  // namespace mkv

@@ -1,0 +1,97 @@
+// Host-side interfaces between the C ABI layer (mkv_api.cu) and the kernel
+// translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "mkv.h"
+
+namespace mkv {
+
+constexpr int kChunk = 64;       // tokens per decode pipeline chunk
+constexpr int kPage = 16;        // ROCKET page size (the only one built)
+
+void set_error(const char* fmt, ...);
+
+inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Work split of a decode call: `n_split` CTAs per (batch, kv-head), each over
+// `chunks_per_split` chunks of kChunk virtual tokens.
+struct Split {
+  int n_split;
+  int chunks_per_split;
+  int64_t v_tokens;  // virtual tokens per (batch, kv-head)
+};
+Split decode_split(const mkv_config& c, int64_t T_cap);
+
+// Workspace carve-up (all float32).  Offsets are 256-byte aligned.
+struct DecodeWs {
+  float* part_m;   // [B][Hq][n_split]   running max (log2 domain)
+  float* part_l;   // [B][Hq][n_split]   sum of 2^(x - m)
+  float* part_o;   // [B][Hq][n_split][D] unnormalized output
+  float* logits;   // H2O: [B][Hkv][T_cap][G] scaled logits (log2 domain)
+  float* m_tot;    // H2O: [B][Hq]
+  float* l_tot;    // H2O: [B][Hq]
+  size_t bytes;
+};
+DecodeWs decode_ws(const mkv_config& c, int64_t T_cap, void* base);
+
+// Prefill workspace (H2O prefill, SnapKV compression): scores and selection.
+struct PrefillWs {
+  float* row_m;    // [B][Hq][T]  per-query-row max (log2 domain)
+  float* row_l;    // [B][Hq][T]  per-query-row sum
+  float* score;    // [B][Hkv][T] accumulated column sums
+  int32_t* keep;   // [B][Hkv][T] kept positions (ascending)
+  size_t bytes;
+};
+PrefillWs prefill_ws(const mkv_config& c, int64_t T, void* base);
+
+// Calibration workspace (KVQuant).
+struct CalibWs {
+  float* sorted;   // [Hkv][D][N] sorted calibration values (keys or u)
+  float* u;        // [Hkv][N][D] normalized values
+  uint8_t* vmask;  // [Hkv][N][D] value-outlier flags
+  size_t bytes;
+};
+CalibWs calib_ws(const mkv_config& c, int64_t N, void* base);
+
+// ---- launchers (return the launch status; arguments already validated) ----
+cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const mkv_cache& cache,
+                                      const int32_t* page_idx, void* out, const DecodeWs& ws,
+                                      const Split& sp, cudaStream_t st);
+cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_cache& cache,
+                                  const mkv_quant_params& qp, void* out,
+                                  const DecodeWs& ws, const Split& sp, cudaStream_t st);
+cudaError_t launch_combine(const mkv_config& c, const DecodeWs& ws, const Split& sp, void* out,
+                           bool h2o_stats, cudaStream_t st);
+cudaError_t launch_append(const mkv_config& c, const void* k_new, const void* v_new,
+                          const mkv_cache& cache, cudaStream_t st);
+cudaError_t launch_rope_table(int D, float theta, int64_t T_max, float* table, cudaStream_t st);
+
+cudaError_t launch_quant_prepare(const mkv_config& c, const mkv_quant_params& qp, cudaStream_t st);
+cudaError_t launch_calibrate(const mkv_config& c, const void* k_cal, const void* v_cal, int64_t N,
+                             int64_t row_stride, const mkv_quant_params& qp, const CalibWs& ws,
+                             cudaStream_t st);
+cudaError_t launch_quantize(const mkv_config& c, const mkv_quant_params& qp, const void* k_pre,
+                            const void* v, int64_t n_tokens, const mkv_cache& cache, cudaStream_t st);
+
+cudaError_t launch_h2o_update(const mkv_config& c, const mkv_cache& cache, const DecodeWs& ws,
+                              cudaStream_t st);
+cudaError_t launch_prefill_scores(const mkv_config& c, const void* q, int64_t q_rows, int64_t T,
+                                  const void* full_k, const PrefillWs& ws, cudaStream_t st);
+cudaError_t launch_h2o_keep(const mkv_config& c, const void* full_k, const void* full_v, int64_t T,
+                            const mkv_cache& cache, const PrefillWs& ws, cudaStream_t st);
+cudaError_t launch_snap_keep(const mkv_config& c, const void* full_k, const void* full_v, int64_t T,
+                             const mkv_cache& cache, int32_t* kept_pos, const PrefillWs& ws,
+                             cudaStream_t st);
+cudaError_t launch_rocket_select(const mkv_config& c, const void* q, const mkv_cache& cache,
+                                 int32_t* page_idx, cudaStream_t st);
+
+// Status word accessors (one per translation unit that can set a flag).
+cudaError_t take_status_kvquant(uint32_t* flags, cudaStream_t st);
+cudaError_t take_status_append(uint32_t* flags, cudaStream_t st);
+
+}  // namespace mkv

@@ -1,0 +1,103 @@
+"""Host-side checks of the C ABI (no GPU needed).
+
+The library must load, export every entry point include/mkv.h declares, and
+reject bad arguments on the host with the documented status codes before
+launching anything.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2609_07966_gb300 as mkv
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    if not os.path.exists(mkv.LIB_PATH):
+        import __graft_entry__
+        __graft_entry__.build()
+    return mkv.lib()
+
+
+def declared_symbols():
+    text = open(os.path.join(ROOT, "include", "mkv.h")).read()
+    return sorted(set(re.findall(r"^(?:mkv_status|const char\*)\s+(mkv_\w+)\(", text, re.M)))
+
+
+def test_exports_every_declared_symbol(L):
+    decl = declared_symbols()
+    assert len(decl) >= 14
+    for name in decl:
+        assert hasattr(L, name), name
+    assert decl == mkv.exported_symbols()
+
+
+def _cfg(**kw):
+    base = dict(method=mkv.MKV_FP16, B=2, Hq=8, Hkv=2, D=64)
+    base.update(kw)
+    m = base.pop("method")
+    return mkv.config(m, base.pop("B"), base.pop("Hq"), base.pop("Hkv"), base.pop("D"), **base)
+
+
+def _status(L, cfg, T=128):
+    n = ctypes.c_size_t(0)
+    return L.mkv_workspace_size(ctypes.byref(cfg) if cfg is not None else None, T, ctypes.byref(n)), n.value
+
+
+def test_config_validation(L):
+    assert _status(L, _cfg())[0] == mkv.MKV_OK
+    assert _status(L, None)[0] == mkv.MKV_ERR_INVALID_ARG
+    c = _cfg()
+    c.abi_version = 99
+    assert _status(L, c)[0] == mkv.MKV_ERR_INVALID_ARG
+    assert _status(L, _cfg(D=96))[0] == mkv.MKV_ERR_UNSUPPORTED
+    assert _status(L, _cfg(Hq=12, Hkv=4))[0] == mkv.MKV_ERR_UNSUPPORTED      # G = 3
+    assert _status(L, _cfg(Hq=9, Hkv=2))[0] == mkv.MKV_ERR_INVALID_ARG       # Hq % Hkv
+    assert _status(L, _cfg(method=mkv.MKV_KVQUANT, bits=5, outlier_frac=0.01))[0] == mkv.MKV_ERR_UNSUPPORTED
+    assert _status(L, _cfg(method=mkv.MKV_KVQUANT, bits=4, outlier_frac=1.5))[0] == mkv.MKV_ERR_INVALID_ARG
+    assert _status(L, _cfg(method=mkv.MKV_H2O))[0] == mkv.MKV_ERR_INVALID_ARG  # zero budget
+    assert _status(L, _cfg(method=mkv.MKV_ROCKET, topk_pages=8, topq_dims=16, snap_window=16,
+                           snap_keep=256, page_size=32))[0] == mkv.MKV_ERR_UNSUPPORTED
+    assert "page_size" in mkv.mkv_last_error()
+
+
+def test_workspace_grows_with_context(L):
+    small = _status(L, _cfg(), 256)[1]
+    big = _status(L, _cfg(), 65536)[1]
+    assert 0 < small <= big
+
+
+def test_cache_bytes_model():
+    cfg = mkv.config(mkv.MKV_FP16, 1, 32, 8, 128)
+    res, peak = mkv.mkv_cache_bytes(cfg, 1000)
+    assert res == peak == 8 * 1000 * 128 * 2 * 2          # 128 KiB per token over 32 layers
+    q4 = mkv.config(mkv.MKV_KVQUANT, 1, 32, 8, 128, bits=4, outlier_frac=0.01)
+    r4, p4 = mkv.mkv_cache_bytes(q4, 1000)
+    assert 0.25 < r4 / res < 0.35 and p4 == r4 + res
+    h = mkv.config(mkv.MKV_H2O, 1, 32, 8, 128, h2o_heavy=100, h2o_recent=100)
+    rh, ph = mkv.mkv_cache_bytes(h, 1000)
+    assert rh == 8 * 200 * (512 + 8) and ph == rh + res
+
+
+def test_pointer_checks_reject_before_launch(L):
+    cfg = _cfg()
+    cache = mkv.mkv_cache()
+    cache.T_cap = 128
+    st = L.mkv_append_kv(ctypes.byref(cfg), None, None, ctypes.byref(cache), None)
+    assert st == mkv.MKV_ERR_INVALID_ARG
+    st = L.mkv_decode_attention(ctypes.byref(cfg), None, ctypes.byref(cache), None, None, None, None, 0, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG
+    cache.T_len = 8
+    cache.k = 16
+    cache.v = 32
+    st = L.mkv_decode_attention(ctypes.byref(cfg), 64, ctypes.byref(cache), None, None, 128, None, 0, None)
+    assert st == mkv.MKV_ERR_WORKSPACE
+    qcfg = _cfg(method=mkv.MKV_KVQUANT, bits=4, outlier_frac=0.01)
+    st = L.mkv_append_kv(ctypes.byref(qcfg), 8, 8, ctypes.byref(cache), None)
+    assert st == mkv.MKV_ERR_INVALID_ARG
+    st = L.mkv_rope_table(96, 10000.0, 10, 8, None)
+    assert st == mkv.MKV_ERR_UNSUPPORTED

@@ -1,0 +1,112 @@
+"""GPU parity: FP16 decode attention (append + split-KV decode + combine) vs the oracle."""
+import numpy as np
+import pytest
+
+import paper_2609_07966_gb300 as mkv
+import synth
+from oracle import attention
+from paper_2609_07966_gb300 import caches
+
+from gpu_util import assert_close, to_dev, torch_cuda
+
+pytestmark = pytest.mark.gpu
+
+
+def _run_fp16(B, Hq, Hkv, D, T_lens, T_cap, steps, seed, dev):
+    """Prefill T_lens[b] tokens, then `steps` append+decode steps; returns outs and the inputs."""
+    torch = torch_cuda()
+    rng = np.random.default_rng(seed)
+    n = max(T_lens) + steps
+    K = rng.standard_normal((B, Hkv, n, D)).astype(np.float16)
+    V = rng.standard_normal((B, Hkv, n, D)).astype(np.float16)
+    Q = rng.standard_normal((steps, B, Hq, D)).astype(np.float16)
+    cfg = mkv.config(mkv.MKV_FP16, B, Hq, Hkv, D)
+    cache = caches.alloc_cache(cfg, T_cap, device=dev)
+    for b in range(B):
+        cache.t["k"][b, :, :T_lens[b]] = to_dev(K[b, :, :T_lens[b]], dev)
+        cache.t["v"][b, :, :T_lens[b]] = to_dev(V[b, :, :T_lens[b]], dev)
+    cache.t["T_len"].copy_(torch.tensor(T_lens, dtype=torch.int32))
+    ws, nws = caches.workspace(cfg, T_cap, device=dev)
+    outs = []
+    for s in range(steps):
+        kn = np.stack([K[b, :, T_lens[b] + s] for b in range(B)])
+        vn = np.stack([V[b, :, T_lens[b] + s] for b in range(B)])
+        kt, vt, qt = to_dev(kn, dev), to_dev(vn, dev), to_dev(Q[s], dev)
+        out = torch.empty_like(qt)
+        mkv.mkv_append_kv(cfg, kt.data_ptr(), vt.data_ptr(), cache.c)
+        mkv.mkv_decode_attention(cfg, qt.data_ptr(), cache.c, None, 0, out.data_ptr(), ws.data_ptr(), nws)
+        outs.append(out.float().cpu().numpy())
+    assert mkv.mkv_get_status() == 0
+    return outs, K, V, Q
+
+
+def _ref(K, V, q, b, n):
+    return attention.decode_gqa(q[b], K[b, :, :n], V[b, :, :n])
+
+
+def test_tiny_all_steps():
+    torch = torch_cuda()
+    w = synth.tiny()
+    x = synth.host_inputs(w, seed=1)
+    dev = torch.device("cuda")
+    cfg = mkv.config(mkv.MKV_FP16, w.B, w.Hq, w.Hkv, w.D)
+    T_cap = w.T + w.steps
+    cache = caches.alloc_cache(cfg, T_cap, device=dev)
+    cache.t["k"][:, :, :w.T] = to_dev(x["k"][0, :, :, :w.T], dev)
+    cache.t["v"][:, :, :w.T] = to_dev(x["v"][0, :, :, :w.T], dev)
+    cache.t["T_len"].fill_(w.T)
+    ws, nws = caches.workspace(cfg, T_cap, device=dev)
+    for s in range(w.steps):
+        kt = to_dev(x["k"][0, :, :, w.T + s], dev)
+        vt = to_dev(x["v"][0, :, :, w.T + s], dev)
+        qt = to_dev(x["q"][s, 0], dev)
+        out = torch.empty_like(qt)
+        mkv.mkv_append_kv(cfg, kt.data_ptr(), vt.data_ptr(), cache.c)
+        mkv.mkv_decode_attention(cfg, qt.data_ptr(), cache.c, None, 0, out.data_ptr(), ws.data_ptr(), nws)
+        got = out.float().cpu().numpy()
+        for b in range(w.B):
+            ref = attention.decode_gqa(x["q"][s, 0, b], x["k"][0, b, :, :w.T + s + 1], x["v"][0, b, :, :w.T + s + 1])
+            assert_close(got[b], ref, f"step {s} b {b}")
+    assert int(cache.t["T_len"][0]) == w.T + w.steps
+
+
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("G", [1, 2, 4, 8])
+def test_shapes_ragged(D, G):
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    Hkv = 2
+    T_lens = [0, 1, 63, 65, 777]
+    outs, K, V, Q = _run_fp16(len(T_lens), G * Hkv, Hkv, D, T_lens, 1024, 2, seed=D * 10 + G, dev=dev)
+    for s in range(2):
+        for b, T in enumerate(T_lens):
+            assert_close(outs[s][b], _ref(K, V, Q[s], b, T + s + 1), f"G{G} D{D} T{T} s{s}")
+
+
+def test_long_context_single_entry():
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    outs, K, V, Q = _run_fp16(1, 32, 8, 128, [40000], 40064, 1, seed=5, dev=dev)
+    assert_close(outs[0][0], _ref(K, V, Q[0], 0, 40001), "T=40001")
+
+
+def test_kvquant_shape_sampled():
+    """Llama-shaped 32/8/128 at B=8, T=8192 (the KVQuant workload's shape), every head checked."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    outs, K, V, Q = _run_fp16(8, 32, 8, 128, [8192] * 8, 8320, 1, seed=6, dev=dev)
+    for b in (0, 3, 7):
+        assert_close(outs[0][b], _ref(K, V, Q[0], b, 8193), f"b{b}")
+
+
+def test_capacity_flag():
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    cfg = mkv.config(mkv.MKV_FP16, 1, 4, 1, 64)
+    cache = caches.alloc_cache(cfg, 4, device=dev)
+    cache.t["T_len"].fill_(4)
+    kn = torch.zeros((1, 1, 64), dtype=torch.float16, device=dev)
+    mkv.mkv_append_kv(cfg, kn.data_ptr(), kn.data_ptr(), cache.c)
+    assert mkv.mkv_get_status() == mkv.MKV_FLAG_CACHE_FULL
+    assert int(cache.t["T_len"][0]) == 4
+    assert mkv.mkv_get_status() == 0      # reading clears the word
