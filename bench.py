@@ -191,8 +191,8 @@ class Runner:
             self.step()
 
     def launches_per_step(self):
-        # per layer: append (1 kernel) + decode (1) + combine (1)
-        return 3 * self.w.L
+        # per layer: append (KVQuant: quantize + length advance) + decode + combine
+        return (4 if self.method == "kvquant" else 3) * self.w.L
 
     def decode_bytes(self):
         """Algorithmic bytes one decode launch reads for one layer at the current lengths."""

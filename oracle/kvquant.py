@@ -8,7 +8,7 @@ remaining choices are readings (each listed in the design doc):
 * keys are quantized before the rotary embedding, per (layer, kv-head,
   channel); values per (token, kv-head);
 * key outliers: per channel, with N_cal calibration tokens and
-  n_t = ceil(frac/2 * N_cal) per tail, t_lo = sorted[n_t] and
+  n_t = ceil(frac/2 * N_cal) per tail (frac taken as an fp32 parameter), t_lo = sorted[n_t] and
   t_hi = sorted[N_cal-1-n_t]; an entry is an outlier iff x < t_lo or x > t_hi;
 * value outliers: the n_v = ceil(frac * D) entries of largest |x| per token
   (ties: lower channel first);
@@ -45,12 +45,17 @@ def n_cal(T_prompt: int) -> int:
     return min(int(T_prompt), 4096)
 
 
+def frac32(frac: float) -> float:
+    """The outlier fraction is an fp32 parameter; counts use its fp32 value."""
+    return float(np.float32(frac))
+
+
 def n_tail(N: int, frac: float) -> int:
-    return int(math.ceil(frac / 2.0 * N))
+    return int(math.ceil(frac32(frac) / 2.0 * N))
 
 
 def n_value_outliers(D: int, frac: float) -> int:
-    return min(D, int(math.ceil(frac * D)))
+    return min(D, int(math.ceil(frac32(frac) * D)))
 
 
 # ----------------------------------------------------------------------------

@@ -208,4 +208,6 @@ def mkv_rocket_select(cfg, q: int, cache: mkv_cache, page_idx_out: int, stream=N
 
 
 def n_value_outliers(D: int, frac: float) -> int:
-    return min(D, int(math.ceil(frac * D - 1e-9)))
+    import ctypes as _ct
+    f32 = _ct.c_float(frac).value
+    return min(D, int(math.ceil(f32 * D)))

@@ -1,0 +1,479 @@
+// KVQuant decode attention with dequantization fused into QK^T / softmax / PV
+// (Section 2.1, KVQuant paragraph: keys quantized per channel before the
+// rotary embedding, values per token, outliers kept in fp16).
+//
+// For each token t of the cache and each query head h of the group:
+//   k_t = rope_t(dq_K(t)) with outliers restored before the rotation,
+//   v_t = lo_t + scale_t * tbl[code] with outliers restored,
+//   out_h = softmax_t(scale q_h . k_t) v_t.
+//
+// GB300 design: one CTA (8 warps) per (batch, kv-head, split); packed codes are
+// staged by cp.async (double buffer, 64 tokens per chunk).  Phase 1: each
+// thread dequantizes half of one token's key or value row from shared tables
+// (all lanes of a warp read the same channel's table -> conflict-free), rotates
+// key pairs (i, i + D/2) by the token's offset delta from its 32-token base,
+// and writes fp16 tiles (keys as hi + lo halves so the tensor-core product
+// keeps fp32 accuracy).  The base rotation R(tb) is applied to the query
+// instead (q . R(tb+d) k = (R(tb)^T q) . (R(d) k)), so only the 32-entry delta
+// table is needed.  Phase 2: tensor-core QK^T (hi*hi + hi*lo + lo*hi), online
+// softmax and PV as in the fp16 kernel.  Tile columns hold pair i at columns
+// (2i, 2i+1) = channels (i, i + D/2); the output is un-permuted at the end.
+#include <math.h>
+
+#include "mkv_common.cuh"
+#include "mkv_internal.h"
+
+namespace mkv {
+
+namespace {
+
+constexpr int kThr = 256;
+
+struct KvqArgs {
+  const __half* q;        // [B][Hq][D]
+  const uint8_t* k_codes; // [B][Hkv][T_cap][row]
+  const uint8_t* v_codes;
+  const float2* v_params; // [B][Hkv][T_cap]
+  const uint32_t* v_out;  // [B][Hkv][T_cap][n_v]
+  const int32_t* k_out_off;
+  const uint32_t* k_out;
+  const float* k_dq;      // [Hkv][D][K]
+  const uint16_t* v_tbl;  // [Hkv][D][K]
+  const float2* rope;     // [rope_len][D/2]
+  int64_t rope_len;
+  const int32_t* T_len;
+  int64_t T_cap, k_out_cap;
+  int Hq, Hkv, G, n_v;
+  int chunks_per_split, n_split;
+  float scale_log2;
+  float* part_m;
+  float* part_l;
+  float* part_o;
+};
+
+template <int D, int BITS>
+struct KvqLayout {
+  static constexpr int NP = D / 2;
+  static constexpr int K = 1 << BITS;
+  static constexpr int ROWB = D * BITS / 8;                  // packed bytes per token row
+  static constexpr int CP = (ROWB % 16 == 0) ? 16 : 8;       // cp.async granularity
+  static constexpr int SROW0 = (ROWB + 15) / 16 * 16;
+  static constexpr int SROW = ((SROW0 / 16) % 2 == 0) ? SROW0 + 16 : SROW0;   // odd # of 16B
+  static constexpr int TILE = kChunk * D * 2;                // fp16 tile bytes
+  // byte offsets
+  static constexpr int DTAB = 0;                             // [NP][32] float2
+  static constexpr int KDQ = DTAB + NP * 32 * 8;             // [D][K] float
+  static constexpr int VTB = KDQ + D * K * 4;                // [D][K] half
+  static constexpr int QHI = VTB + D * K * 2;                // [2 bases][8][NP] half2 (rotated query, hi)
+  static constexpr int QLO = QHI + 2 * 8 * NP * 4;           // [2][8][NP] half2 (lo)
+  static constexpr int STG = QLO + 2 * 8 * NP * 4;           // [2 stages][2 (K,V)][64][SROW]
+  static constexpr int KHI = STG + 2 * 2 * kChunk * SROW;
+  static constexpr int KLO = KHI + TILE;
+  static constexpr int VT = KLO + TILE;
+  static constexpr int BYTES = VT + TILE;
+};
+
+// the `bits`-wide code of channel-in-pair `which` for pair j of a thread's word array
+template <int BITS, int NW>
+__device__ __forceinline__ void pair_codes(const uint32_t (&w)[NW], int j, int& lo, int& hi) {
+  const int bit = 2 * BITS * j;
+  const int wi = bit >> 5, sh = bit & 31;
+  uint32_t x = w[wi] >> sh;
+  if (sh + 2 * BITS > 32 && wi + 1 < NW) x |= w[wi + 1] << (32 - sh);
+  lo = (int)(x & ((1u << BITS) - 1u));
+  hi = (int)((x >> BITS) & ((1u << BITS) - 1u));
+}
+
+__device__ __forceinline__ void split_hi_lo(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __half2 h = __floats2half2_rn(a, b);
+  const float2 hf = __half22float2(h);
+  const __half2 l = __floats2half2_rn(a - hf.x, b - hf.y);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = *reinterpret_cast<const uint32_t*>(&l);
+}
+
+// byte offset of (row, 16B chunk) in a swizzled fp16 tile of D columns
+template <int D>
+__device__ __forceinline__ int tile_off(int row, int ch) {
+  return row * D * 2 + ((ch ^ (row & 7)) << 4);
+}
+
+template <int D, int BITS>
+__global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
+  using Lay = KvqLayout<D, BITS>;
+  constexpr int NP = Lay::NP, K = Lay::K, ROWB = Lay::ROWB, SROW = Lay::SROW;
+  constexpr int KC = D / 16;
+  constexpr int HALF_PAIRS = NP / 2;                  // pairs per thread (half a row)
+  constexpr int HALF_WORDS = HALF_PAIRS * 2 * BITS / 32;
+  extern __shared__ __align__(128) uint8_t smem[];
+  float2* dtab = reinterpret_cast<float2*>(smem + Lay::DTAB);
+  float* kdq = reinterpret_cast<float*>(smem + Lay::KDQ);
+  __half* vtb = reinterpret_cast<__half*>(smem + Lay::VTB);
+  uint32_t* qhi = reinterpret_cast<uint32_t*>(smem + Lay::QHI);
+  uint32_t* qlo = reinterpret_cast<uint32_t*>(smem + Lay::QLO);
+  uint8_t* stg = smem + Lay::STG;
+  uint8_t* khi_t = smem + Lay::KHI;
+  uint8_t* klo_t = smem + Lay::KLO;
+  uint8_t* v_t = smem + Lay::VT;
+
+  const int split = blockIdx.x;
+  const int64_t bh = blockIdx.y;
+  const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, r = lane & 3;
+  const int n_len = a.T_len[b];
+  const int64_t v_begin = (int64_t)split * a.chunks_per_split * kChunk;
+  int64_t v_end = v_begin + (int64_t)a.chunks_per_split * kChunk;
+  if (v_end > n_len) v_end = n_len;
+  const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
+
+  const uint8_t* kc_base = a.k_codes + bh * a.T_cap * ROWB;
+  const uint8_t* vc_base = a.v_codes + bh * a.T_cap * ROWB;
+
+  auto load_chunk = [&](int c, int stage) {
+    uint8_t* dst = stg + stage * 2 * kChunk * SROW;
+    constexpr int PER_ROW = ROWB / Lay::CP;
+    for (int e = tid; e < 2 * kChunk * PER_ROW; e += kThr) {
+      const int kv = e / (kChunk * PER_ROW);
+      const int rem = e % (kChunk * PER_ROW);
+      const int row = rem / PER_ROW, piece = rem % PER_ROW;
+      const int64_t s = v_begin + (int64_t)c * kChunk + row;
+      const bool ok = s < n_len;
+      const uint8_t* src = (kv ? vc_base : kc_base) + (ok ? s : 0) * ROWB + piece * Lay::CP;
+      uint8_t* d = dst + (kv * kChunk + row) * SROW + piece * Lay::CP;
+      if (Lay::CP == 16) {
+        cp_async16(d, src, ok ? 16 : 0);
+      } else {
+        cp_async8(d, src, ok ? 8 : 0);
+      }
+    }
+  };
+
+  if (nchunks > 0) {
+    load_chunk(0, 0);
+    cp_async_commit();
+  }
+  // CTA-resident tables: rotations by delta in [0, 32), dequant tables of this kv-head
+  for (int e = tid; e < NP * 32; e += kThr) {
+    const int i = e / 32, d = e % 32;
+    dtab[e] = a.rope[(int64_t)d * NP + i];
+  }
+  for (int e = tid; e < D * K; e += kThr) {
+    kdq[e] = a.k_dq[(int64_t)kvh * D * K + e];
+    vtb[e] = __ushort_as_half(a.v_tbl[(int64_t)kvh * D * K + e]);
+  }
+
+  float o[D / 16][2];
+#pragma unroll
+  for (int i = 0; i < D / 16; ++i) o[i][0] = o[i][1] = 0.f;
+  float m_run = -INFINITY, l_part = 0.f;
+  const int slab = warp & 3, dhalf = warp >> 2;
+
+  for (int c = 0; c < nchunks; ++c) {
+    cp_async_wait<0>();
+    __syncthreads();
+    if (c + 1 < nchunks) load_chunk(c + 1, (c + 1) & 1);
+    cp_async_commit();
+    const int64_t t0 = v_begin + (int64_t)c * kChunk;      // position of the chunk's first token
+    const uint8_t* st = stg + (c & 1) * 2 * kChunk * SROW;
+
+    // ---- query rotated back by each 32-token base tb: R(tb)^T q as hi/lo fp16 pairs,
+    //      qhi[base][g][i] = (q'_i, q'_{i+NP}), base 0 -> t0, base 1 -> t0 + 32
+    for (int e = tid; e < 2 * a.G * NP; e += kThr) {
+      const int base = e / (a.G * NP), gg = (e / NP) % a.G, i = e % NP;
+      const __half* qr = a.q + ((int64_t)b * a.Hq + (int64_t)kvh * a.G + gg) * D;
+      const float x = __half2float(qr[i]), y = __half2float(qr[i + NP]);
+      const int64_t tb = min(t0 + 32 * base, a.rope_len - 1);
+      const float2 cs = a.rope[tb * NP + i];
+      split_hi_lo(x * cs.x + y * cs.y, y * cs.x - x * cs.y, qhi[(base * 8 + gg) * NP + i],
+                  qlo[(base * 8 + gg) * NP + i]);
+    }
+
+    // ---- phase 1: dequantize the chunk into fp16 tiles
+    {
+      const bool is_v = warp >= 4;
+      const int wl = warp & 3;
+      const int tok = (wl & 1) * 32 + lane;           // row of the chunk
+      const int hp = wl >> 1;                         // which half of the pairs
+      const int64_t slot = t0 + tok;
+      const bool valid = slot < n_len;
+      const uint8_t* row = st + ((is_v ? kChunk : 0) + tok) * SROW + hp * (HALF_WORDS * 4);
+      uint32_t w[HALF_WORDS];
+      if constexpr (HALF_WORDS % 4 == 0) {
+#pragma unroll
+        for (int k = 0; k < HALF_WORDS; k += 4) {
+          const uint4 u = *reinterpret_cast<const uint4*>(row + 4 * k);
+          w[k] = u.x;
+          w[k + 1] = u.y;
+          w[k + 2] = u.z;
+          w[k + 3] = u.w;
+        }
+      } else if constexpr (HALF_WORDS % 2 == 0) {
+#pragma unroll
+        for (int k = 0; k < HALF_WORDS; k += 2) {
+          const uint2 u = *reinterpret_cast<const uint2*>(row + 4 * k);
+          w[k] = u.x;
+          w[k + 1] = u.y;
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < HALF_WORDS; ++k) w[k] = *reinterpret_cast<const uint32_t*>(row + 4 * k);
+      }
+      const int dl = tok & 31;                        // offset from the token's 32-token base
+      uint8_t* tile = is_v ? v_t : khi_t;
+      if (!is_v) {
+#pragma unroll
+        for (int jj = 0; jj < HALF_PAIRS; jj += 4) {
+          uint32_t ph[4], pl[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int j = jj + u, i = hp * HALF_PAIRS + j;
+            int clo, chi;
+            pair_codes<BITS, HALF_WORDS>(w, j, clo, chi);
+            const float x = valid ? kdq[i * K + clo] : 0.f;
+            const float y = valid ? kdq[(i + NP) * K + chi] : 0.f;
+            const float2 cs = dtab[i * 32 + dl];
+            split_hi_lo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph[u], pl[u]);
+          }
+          const int ch = (hp * HALF_PAIRS + jj) / 4;
+          *reinterpret_cast<uint4*>(khi_t + tile_off<D>(tok, ch)) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
+          *reinterpret_cast<uint4*>(klo_t + tile_off<D>(tok, ch)) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
+        }
+        // key outliers of this token in this half: recompute their pair exactly
+        if (valid) {
+          const int32_t* off = a.k_out_off + bh * (a.T_cap + 1) + slot;
+          const int e0 = off[0], e1 = min(off[1], (int32_t)a.k_out_cap);
+          const uint32_t* ents = a.k_out + bh * a.k_out_cap;
+          for (int e = e0; e < e1; ++e) {
+            const int ch = (int)(ents[e] >> 16);
+            const int i = ch % NP;
+            if (i / HALF_PAIRS != hp) continue;
+            int clo, chi;
+            pair_codes<BITS, HALF_WORDS>(w, i - hp * HALF_PAIRS, clo, chi);
+            float x = kdq[i * K + clo], y = kdq[(i + NP) * K + chi];
+            for (int f = e0; f < e1; ++f) {
+              const uint32_t ef = ents[f];
+              const int cf = (int)(ef >> 16);
+              if (cf == i) x = h2f((uint16_t)(ef & 0xffffu));
+              if (cf == i + NP) y = h2f((uint16_t)(ef & 0xffffu));
+            }
+            const float2 cs = dtab[i * 32 + dl];
+            uint32_t ph, pl;
+            split_hi_lo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph, pl);
+            const int byte = tile_off<D>(tok, i / 4) + (i % 4) * 4;
+            *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
+            *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
+          }
+        }
+      } else {
+        const float2 lp = valid ? a.v_params[bh * a.T_cap + slot] : make_float2(0.f, 0.f);
+#pragma unroll
+        for (int jj = 0; jj < HALF_PAIRS; jj += 4) {
+          uint32_t pv[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int j = jj + u, i = hp * HALF_PAIRS + j;
+            int clo, chi;
+            pair_codes<BITS, HALF_WORDS>(w, j, clo, chi);
+            const float x = lp.x + lp.y * __half2float(vtb[i * K + clo]);
+            const float y = lp.x + lp.y * __half2float(vtb[(i + NP) * K + chi]);
+            pv[u] = valid ? pack_half2(x, y) : 0u;
+          }
+          const int ch = (hp * HALF_PAIRS + jj) / 4;
+          *reinterpret_cast<uint4*>(tile + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
+        }
+        if (valid) {
+          const uint32_t* ents = a.v_out + (bh * a.T_cap + slot) * a.n_v;
+          for (int e = 0; e < a.n_v; ++e) {
+            const uint32_t ev = ents[e];
+            const int ch = (int)(ev >> 16);
+            const int i = ch % NP;
+            if (i / HALF_PAIRS != hp) continue;
+            const int col = ch < NP ? 2 * ch : 2 * (ch - NP) + 1;
+            *reinterpret_cast<uint16_t*>(tile + tile_off<D>(tok, col / 8) + (col % 8) * 2) =
+                (uint16_t)(ev & 0xffffu);
+          }
+        }
+      }
+    }
+    __syncthreads();
+
+    // ---- phase 2: warp (slab, dhalf) -> tokens 16*slab.., output dims half dhalf
+    {
+      const bool real = g < a.G;
+      const int t0w = slab * 16;
+      const uint32_t* qh = qhi + (slab >> 1) * 8 * NP;      // slabs 0-1: base t0, 2-3: t0 + 32
+      const uint32_t* ql = qlo + (slab >> 1) * 8 * NP;
+      float sc[2][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) sc[0][i] = sc[1][i] = 0.f;
+      const int mi = lane >> 3, rowi = lane & 7;
+      const int tokk = t0w + (mi >> 1) * 8 + rowi;
+#pragma unroll
+      for (int kc = 0; kc < KC; ++kc) {
+        const uint32_t ah0 = real ? qh[g * NP + kc * 8 + r] : 0u;
+        const uint32_t ah2 = real ? qh[g * NP + kc * 8 + r + 4] : 0u;
+        const uint32_t al0 = real ? ql[g * NP + kc * 8 + r] : 0u;
+        const uint32_t al2 = real ? ql[g * NP + kc * 8 + r + 4] : 0u;
+        uint32_t bh4[4], bl4[4];
+        const int ch = kc * 2 + (mi & 1);
+        ldsm_x4(bh4, khi_t + tile_off<D>(tokk, ch));
+        ldsm_x4(bl4, klo_t + tile_off<D>(tokk, ch));
+        mma16816(sc[0], ah0, 0u, ah2, 0u, bh4[0], bh4[1]);
+        mma16816(sc[1], ah0, 0u, ah2, 0u, bh4[2], bh4[3]);
+        mma16816(sc[0], ah0, 0u, ah2, 0u, bl4[0], bl4[1]);
+        mma16816(sc[1], ah0, 0u, ah2, 0u, bl4[2], bl4[3]);
+        mma16816(sc[0], al0, 0u, al2, 0u, bh4[0], bh4[1]);
+        mma16816(sc[1], al0, 0u, al2, 0u, bh4[2], bh4[3]);
+      }
+      const int tk[4] = {t0w + 2 * r, t0w + 2 * r + 1, t0w + 8 + 2 * r, t0w + 9 + 2 * r};
+      float x[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
+      float mx = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        x[i] = (t0 + tk[i] < n_len) ? x[i] * a.scale_log2 : -INFINITY;
+        mx = fmaxf(mx, x[i]);
+      }
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float m_new = fmaxf(m_run, mx);
+      float p[4];
+      float alpha = 1.f;
+      if (m_new == -INFINITY) {
+        p[0] = p[1] = p[2] = p[3] = 0.f;
+      } else {
+        alpha = exp2f(m_run - m_new);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) p[i] = exp2f(x[i] - m_new);
+      }
+      l_part = l_part * alpha + (p[0] + p[1]) + (p[2] + p[3]);
+      m_run = m_new;
+      if (__any_sync(0xffffffffu, alpha != 1.f)) {
+#pragma unroll
+        for (int i = 0; i < D / 16; ++i) {
+          o[i][0] *= alpha;
+          o[i][1] *= alpha;
+        }
+      }
+      const uint32_t pa0 = pack_half2(p[0], p[1]);
+      const uint32_t pa2 = pack_half2(p[2], p[3]);
+      const int tokv = t0w + (mi & 1) * 8 + rowi;
+#pragma unroll
+      for (int j = 0; j < D / 32; ++j) {
+        uint32_t bv[4];
+        const int jj = dhalf * (D / 32) + j;
+        const int ch = 2 * jj + (mi >> 1);
+        ldsm_x4_t(bv, v_t + tile_off<D>(tokv, ch));
+        float d0[4] = {o[2 * j][0], o[2 * j][1], 0.f, 0.f};
+        float d1[4] = {o[2 * j + 1][0], o[2 * j + 1][1], 0.f, 0.f};
+        mma16816(d0, pa0, 0u, pa2, 0u, bv[0], bv[1]);
+        mma16816(d1, pa0, 0u, pa2, 0u, bv[2], bv[3]);
+        o[2 * j][0] = d0[0];
+        o[2 * j][1] = d0[1];
+        o[2 * j + 1][0] = d1[0];
+        o[2 * j + 1][1] = d1[1];
+      }
+    }
+  }
+  cp_async_wait<0>();
+  __syncthreads();
+
+  // ---- merge the four slabs; warps of dhalf 0 and 1 hold the two halves of the dims
+  l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
+  l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
+  float* wm = reinterpret_cast<float*>(smem + Lay::STG);   // [4][8]
+  float* wl = wm + 32;                                      // [4][8]
+  float* wo = wl + 32;                                      // [4][8][D]  (natural channel order)
+  if (g < a.G) {
+    if (r == 0 && dhalf == 0) {
+      wm[slab * 8 + g] = m_run;
+      wl[slab * 8 + g] = l_part;
+    }
+#pragma unroll
+    for (int j = 0; j < D / 16; ++j) {
+      const int dt = dhalf * (D / 16) + j;                  // 8-column tile of the permuted order
+      const int ch = dt * 4 + r;                            // column dt*8 + 2r -> channel dt*4 + r
+      wo[(slab * 8 + g) * D + ch] = o[j][0];
+      wo[(slab * 8 + g) * D + ch + NP] = o[j][1];
+    }
+  }
+  __syncthreads();
+  for (int e = tid; e < a.G * D; e += kThr) {
+    const int row = e / D, d = e % D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w * 8 + row]);
+    float L = 0.f, O = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const float f = exp2f(wm[w * 8 + row] - M);
+        L += wl[w * 8 + row] * f;
+        O += wo[(w * 8 + row) * D + d] * f;
+      }
+    }
+    const int64_t hq = (int64_t)b * a.Hq + (int64_t)kvh * a.G + row;
+    const int64_t pi = hq * a.n_split + split;
+    a.part_o[pi * D + d] = O;
+    if (d == 0) {
+      a.part_m[pi] = M;
+      a.part_l[pi] = L;
+    }
+  }
+}
+
+template <int D, int BITS>
+cudaError_t launch_kvq_t(const KvqArgs& a, int units, int n_split, cudaStream_t st) {
+  using Lay = KvqLayout<D, BITS>;
+  static_assert(Lay::BYTES <= 113 * 1024, "two CTAs per SM");
+  cudaError_t e = cudaFuncSetAttribute(decode_kvq_kernel<D, BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Lay::BYTES);
+  if (e != cudaSuccess) return e;
+  decode_kvq_kernel<D, BITS><<<dim3(n_split, units), kThr, Lay::BYTES, st>>>(a);
+  return cudaPeekAtLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_cache& cache,
+                                  const mkv_quant_params& qp, void* out, const DecodeWs& ws, const Split& sp,
+                                  cudaStream_t st) {
+  (void)out;
+  KvqArgs a{};
+  a.q = static_cast<const __half*>(q);
+  a.k_codes = cache.k_codes;
+  a.v_codes = cache.v_codes;
+  a.v_params = reinterpret_cast<const float2*>(cache.v_params);
+  a.v_out = cache.v_out;
+  a.k_out_off = cache.k_out_off;
+  a.k_out = cache.k_out;
+  a.k_dq = qp.k_dq;
+  a.v_tbl = qp.v_tbl;
+  a.rope = reinterpret_cast<const float2*>(qp.rope);
+  a.rope_len = qp.rope_len;
+  a.T_len = cache.T_len;
+  a.T_cap = cache.T_cap;
+  a.k_out_cap = cache.k_out_cap;
+  a.Hq = c.Hq;
+  a.Hkv = c.Hkv;
+  a.G = c.Hq / c.Hkv;
+  a.n_v = std::min(c.D, (int)ceil((double)c.outlier_frac * c.D));
+  a.chunks_per_split = sp.chunks_per_split;
+  a.n_split = sp.n_split;
+  const float scale = c.softmax_scale > 0.f ? c.softmax_scale : 1.0f / sqrtf((float)c.D);
+  a.scale_log2 = scale * kLog2e;
+  a.part_m = ws.part_m;
+  a.part_l = ws.part_l;
+  a.part_o = ws.part_o;
+  const int units = c.B * c.Hkv;
+  if (c.D == 128) {
+    if (c.bits == 4) return launch_kvq_t<128, 4>(a, units, sp.n_split, st);
+    if (c.bits == 3) return launch_kvq_t<128, 3>(a, units, sp.n_split, st);
+    return launch_kvq_t<128, 2>(a, units, sp.n_split, st);
+  }
+  if (c.bits == 4) return launch_kvq_t<64, 4>(a, units, sp.n_split, st);
+  if (c.bits == 3) return launch_kvq_t<64, 3>(a, units, sp.n_split, st);
+  return launch_kvq_t<64, 2>(a, units, sp.n_split, st);
+}
+
+}  // namespace mkv

@@ -159,7 +159,7 @@ mkv_status check_config(const mkv_config* c) {
 }
 
 int n_value_outliers(const mkv_config* c) {
-  return std::min(c->D, (int)ceil((double)c->outlier_frac * c->D - 1e-9));
+  return std::min(c->D, (int)ceil((double)c->outlier_frac * c->D));
 }
 
 mkv_status check_cache(const mkv_config* c, const mkv_cache* k) {
@@ -302,8 +302,8 @@ mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_
   if (cfg->method == MKV_ROCKET) MKV_REQUIRE(page_idx != nullptr, MKV_ERR_INVALID_ARG, "ROCKET needs page_idx");
   if (cfg->method == MKV_KVQUANT) {
     MKV_TRY(check_qparams(cfg, qparams, true));
-    MKV_REQUIRE(qparams->rope && qparams->rope_len >= cache->T_cap, MKV_ERR_INVALID_ARG,
-                "KVQUANT decode needs a rope table with rope_len >= T_cap");
+    MKV_REQUIRE(qparams->rope && qparams->rope_len >= std::max<int64_t>(cache->T_cap, 32), MKV_ERR_INVALID_ARG,
+                "KVQUANT decode needs a rope table with rope_len >= max(T_cap, 32)");
   }
   const DecodeWs need = decode_ws(*cfg, cache->T_cap, nullptr);
   MKV_REQUIRE(ws != nullptr && ws_bytes >= need.bytes, MKV_ERR_WORKSPACE,

@@ -4,13 +4,6 @@
 #include "mkv_internal.h"
 
 namespace mkv {
-cudaError_t launch_decode_kvquant(const mkv_config&, const void*, const mkv_cache&, const mkv_quant_params&,
-                                  void*, const DecodeWs&, const Split&, cudaStream_t) { return cudaErrorNotSupported; }
-cudaError_t launch_quant_prepare(const mkv_config&, const mkv_quant_params&, cudaStream_t) { return cudaErrorNotSupported; }
-cudaError_t launch_calibrate(const mkv_config&, const void*, const void*, int64_t, int64_t, const mkv_quant_params&,
-                             const CalibWs&, cudaStream_t) { return cudaErrorNotSupported; }
-cudaError_t launch_quantize(const mkv_config&, const mkv_quant_params&, const void*, const void*, int64_t,
-                            const mkv_cache&, cudaStream_t) { return cudaErrorNotSupported; }
 cudaError_t launch_h2o_update(const mkv_config&, const mkv_cache&, const DecodeWs&, cudaStream_t) { return cudaErrorNotSupported; }
 cudaError_t launch_prefill_scores(const mkv_config&, const void*, int64_t, int64_t, const void*, const PrefillWs&,
                                   cudaStream_t) { return cudaErrorNotSupported; }
@@ -21,5 +14,4 @@ cudaError_t launch_snap_keep(const mkv_config&, const void*, const void*, int64_
 cudaError_t launch_rocket_select(const mkv_config&, const void*, const mkv_cache&, int32_t*, cudaStream_t) {
   return cudaErrorNotSupported;
 }
-cudaError_t take_status_kvquant(uint32_t* flags, cudaStream_t) { (void)flags; return cudaSuccess; }
 }  // namespace mkv
