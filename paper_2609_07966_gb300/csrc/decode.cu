@@ -83,12 +83,12 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
   int n_len = 0, ns = 0;
   int64_t v_total;
   if (MODE == 0) {
-    n_len = a.T_len[b];
+    n_len = min((int64_t)a.T_len[b], a.T_cap);
     v_total = n_len;
   } else if (MODE == 1) {
     v_total = a.T_cap;
   } else {
-    n_len = a.T_len[b];
+    n_len = (int)min((int64_t)a.T_len[b], a.T_cap);
     ns = n_len > 0 ? (n_len - 1) / kPage : 0;
     v_total = (int64_t)(a.kp + 1) * kPage;
   }

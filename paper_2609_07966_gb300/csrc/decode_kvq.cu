@@ -60,14 +60,24 @@ struct KvqLayout {
   static constexpr int SROW0 = (ROWB + 15) / 16 * 16;
   static constexpr int SROW = ((SROW0 / 16) % 2 == 0) ? SROW0 + 16 : SROW0;   // odd # of 16B
   static constexpr int TILE = kChunk * D * 2;                // fp16 tile bytes
+  static constexpr int NVS = 4;                              // value outliers staged per token (<=)
+  // one pipeline stage: codes, then the chunk's per-token side data
+  static constexpr int S_KC = 0;                             // [64][SROW] key codes
+  static constexpr int S_VC = S_KC + kChunk * SROW;          // [64][SROW] value codes
+  static constexpr int S_VP = S_VC + kChunk * SROW;          // [64] float2 (lo, scale)
+  static constexpr int S_KO = S_VP + kChunk * 8;             // [68] int32 key-outlier CSR offsets
+  static constexpr int S_VO = S_KO + 68 * 4;                 // [64][NVS] uint32 value outliers
+  static constexpr int S_RP = S_VO + kChunk * NVS * 4;       // [2][NP] float2 rotations of the bases
+  static constexpr int STAGE = S_RP + 2 * NP * 8;
   // byte offsets
   static constexpr int DTAB = 0;                             // [NP][32] float2
   static constexpr int KDQ = DTAB + NP * 32 * 8;             // [D][K] float
   static constexpr int VTB = KDQ + D * K * 4;                // [D][K] half
-  static constexpr int QHI = VTB + D * K * 2;                // [2 bases][8][NP] half2 (rotated query, hi)
+  static constexpr int QRAW = VTB + D * K * 2;               // [8][D] half (the group's queries)
+  static constexpr int QHI = QRAW + 8 * D * 2;               // [2 bases][8][NP] half2 (rotated query, hi)
   static constexpr int QLO = QHI + 2 * 8 * NP * 4;           // [2][8][NP] half2 (lo)
-  static constexpr int STG = QLO + 2 * 8 * NP * 4;           // [2 stages][2 (K,V)][64][SROW]
-  static constexpr int KHI = STG + 2 * 2 * kChunk * SROW;
+  static constexpr int STG = QLO + 2 * 8 * NP * 4;           // [2 stages][STAGE]
+  static constexpr int KHI = STG + 2 * STAGE;
   static constexpr int KLO = KHI + TILE;
   static constexpr int VT = KLO + TILE;
   static constexpr int BYTES = VT + TILE;
@@ -80,6 +90,18 @@ __device__ __forceinline__ void pair_codes(const uint32_t (&w)[NW], int j, int& 
   const int wi = bit >> 5, sh = bit & 31;
   uint32_t x = w[wi] >> sh;
   if (sh + 2 * BITS > 32 && wi + 1 < NW) x |= w[wi + 1] << (32 - sh);
+  lo = (int)(x & ((1u << BITS) - 1u));
+  hi = (int)((x >> BITS) & ((1u << BITS) - 1u));
+}
+
+// pair j's codes read from a packed row in shared memory (any j)
+template <int BITS>
+__device__ __forceinline__ void pair_codes_row(const uint8_t* row, int j, int& lo, int& hi) {
+  const int bit = 2 * BITS * j;
+  const int wi = bit >> 5, sh = bit & 31;
+  const uint32_t w0 = reinterpret_cast<const uint32_t*>(row)[wi];
+  const uint32_t w1 = reinterpret_cast<const uint32_t*>(row)[wi + 1];
+  const uint32_t x = __funnelshift_r(w0, w1, sh);
   lo = (int)(x & ((1u << BITS) - 1u));
   hi = (int)((x >> BITS) & ((1u << BITS) - 1u));
 }
@@ -112,6 +134,7 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
   uint32_t* qhi = reinterpret_cast<uint32_t*>(smem + Lay::QHI);
   uint32_t* qlo = reinterpret_cast<uint32_t*>(smem + Lay::QLO);
   uint8_t* stg = smem + Lay::STG;
+  __half* qraw = reinterpret_cast<__half*>(smem + Lay::QRAW);
   uint8_t* khi_t = smem + Lay::KHI;
   uint8_t* klo_t = smem + Lay::KLO;
   uint8_t* v_t = smem + Lay::VT;
@@ -121,7 +144,7 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
   const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, r = lane & 3;
-  const int n_len = a.T_len[b];
+  const int n_len = (int)min((int64_t)a.T_len[b], a.T_cap);
   const int64_t v_begin = (int64_t)split * a.chunks_per_split * kChunk;
   int64_t v_end = v_begin + (int64_t)a.chunks_per_split * kChunk;
   if (v_end > n_len) v_end = n_len;
@@ -130,21 +153,46 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
   const uint8_t* kc_base = a.k_codes + bh * a.T_cap * ROWB;
   const uint8_t* vc_base = a.v_codes + bh * a.T_cap * ROWB;
 
+  const bool stage_vout = a.n_v <= Lay::NVS;
   auto load_chunk = [&](int c, int stage) {
-    uint8_t* dst = stg + stage * 2 * kChunk * SROW;
+    uint8_t* dst = stg + stage * Lay::STAGE;
+    const int64_t c0 = v_begin + (int64_t)c * kChunk;
     constexpr int PER_ROW = ROWB / Lay::CP;
     for (int e = tid; e < 2 * kChunk * PER_ROW; e += kThr) {
       const int kv = e / (kChunk * PER_ROW);
       const int rem = e % (kChunk * PER_ROW);
       const int row = rem / PER_ROW, piece = rem % PER_ROW;
-      const int64_t s = v_begin + (int64_t)c * kChunk + row;
+      const int64_t s = c0 + row;
       const bool ok = s < n_len;
       const uint8_t* src = (kv ? vc_base : kc_base) + (ok ? s : 0) * ROWB + piece * Lay::CP;
-      uint8_t* d = dst + (kv * kChunk + row) * SROW + piece * Lay::CP;
+      uint8_t* d = dst + (kv ? Lay::S_VC : Lay::S_KC) + row * SROW + piece * Lay::CP;
       if (Lay::CP == 16) {
         cp_async16(d, src, ok ? 16 : 0);
       } else {
         cp_async8(d, src, ok ? 8 : 0);
+      }
+    }
+    if (tid < kChunk) {                          // value (lo, scale)
+      const int64_t s = c0 + tid;
+      const bool ok = s < n_len;
+      cp_async8(dst + Lay::S_VP + tid * 8, a.v_params + bh * a.T_cap + (ok ? s : 0), ok ? 8 : 0);
+    } else if (tid < kChunk + kChunk + 1) {      // CSR offsets c0 .. c0+64 (clamped to the cache)
+      const int i = tid - kChunk;
+      const int64_t s = min(c0 + i, (int64_t)n_len);
+      cp_async4(dst + Lay::S_KO + i * 4, a.k_out_off + bh * (a.T_cap + 1) + s, 4);
+    } else if (tid < 2 * kChunk + 1 + 2 * NP / 2) {   // rotations of the two 32-token bases
+      const int e = tid - (2 * kChunk + 1);           // 16-byte pieces: 2 float2 each
+      const int base = e / (NP / 2), piece = e % (NP / 2);
+      const int64_t tb = min(c0 + 32 * base, a.rope_len - 1);
+      cp_async16(dst + Lay::S_RP + (base * NP + 2 * piece) * 8, a.rope + tb * NP + 2 * piece, 16);
+    }
+    if (stage_vout && a.n_v > 0) {
+      for (int e = tid; e < kChunk * a.n_v; e += kThr) {
+        const int row = e / a.n_v, k = e % a.n_v;
+        const int64_t s = c0 + row;
+        const bool ok = s < n_len;
+        cp_async4(dst + Lay::S_VO + (row * Lay::NVS + k) * 4, a.v_out + (bh * a.T_cap + (ok ? s : 0)) * a.n_v + k,
+                  ok ? 4 : 0);
       }
     }
   };
@@ -162,6 +210,9 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     kdq[e] = a.k_dq[(int64_t)kvh * D * K + e];
     vtb[e] = __ushort_as_half(a.v_tbl[(int64_t)kvh * D * K + e]);
   }
+  for (int e = tid; e < a.G * D; e += kThr) {
+    qraw[e] = a.q[((int64_t)b * a.Hq + (int64_t)kvh * a.G) * D + e];
+  }
 
   float o[D / 16][2];
 #pragma unroll
@@ -175,16 +226,18 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     if (c + 1 < nchunks) load_chunk(c + 1, (c + 1) & 1);
     cp_async_commit();
     const int64_t t0 = v_begin + (int64_t)c * kChunk;      // position of the chunk's first token
-    const uint8_t* st = stg + (c & 1) * 2 * kChunk * SROW;
+    const uint8_t* st = stg + (c & 1) * Lay::STAGE;
+    const float2* vpar = reinterpret_cast<const float2*>(st + Lay::S_VP);
+    const int32_t* koff = reinterpret_cast<const int32_t*>(st + Lay::S_KO);
+    const uint32_t* vouts = reinterpret_cast<const uint32_t*>(st + Lay::S_VO);
+    const float2* rbase = reinterpret_cast<const float2*>(st + Lay::S_RP);
 
     // ---- query rotated back by each 32-token base tb: R(tb)^T q as hi/lo fp16 pairs,
     //      qhi[base][g][i] = (q'_i, q'_{i+NP}), base 0 -> t0, base 1 -> t0 + 32
     for (int e = tid; e < 2 * a.G * NP; e += kThr) {
       const int base = e / (a.G * NP), gg = (e / NP) % a.G, i = e % NP;
-      const __half* qr = a.q + ((int64_t)b * a.Hq + (int64_t)kvh * a.G + gg) * D;
-      const float x = __half2float(qr[i]), y = __half2float(qr[i + NP]);
-      const int64_t tb = min(t0 + 32 * base, a.rope_len - 1);
-      const float2 cs = a.rope[tb * NP + i];
+      const float x = __half2float(qraw[gg * D + i]), y = __half2float(qraw[gg * D + i + NP]);
+      const float2 cs = rbase[base * NP + i];
       split_hi_lo(x * cs.x + y * cs.y, y * cs.x - x * cs.y, qhi[(base * 8 + gg) * NP + i],
                   qlo[(base * 8 + gg) * NP + i]);
     }
@@ -197,7 +250,8 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
       const int hp = wl >> 1;                         // which half of the pairs
       const int64_t slot = t0 + tok;
       const bool valid = slot < n_len;
-      const uint8_t* row = st + ((is_v ? kChunk : 0) + tok) * SROW + hp * (HALF_WORDS * 4);
+      const uint8_t* rowfull = st + (is_v ? Lay::S_VC : Lay::S_KC) + tok * SROW;
+      const uint8_t* row = rowfull + hp * (HALF_WORDS * 4);
       uint32_t w[HALF_WORDS];
       if constexpr (HALF_WORDS % 4 == 0) {
 #pragma unroll
@@ -241,15 +295,14 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
         }
         // key outliers of this token in this half: recompute their pair exactly
         if (valid) {
-          const int32_t* off = a.k_out_off + bh * (a.T_cap + 1) + slot;
-          const int e0 = off[0], e1 = min(off[1], (int32_t)a.k_out_cap);
+          const int e0 = koff[tok], e1 = (int)min((int64_t)koff[tok + 1], a.k_out_cap);
           const uint32_t* ents = a.k_out + bh * a.k_out_cap;
           for (int e = e0; e < e1; ++e) {
             const int ch = (int)(ents[e] >> 16);
             const int i = ch % NP;
             if (i / HALF_PAIRS != hp) continue;
             int clo, chi;
-            pair_codes<BITS, HALF_WORDS>(w, i - hp * HALF_PAIRS, clo, chi);
+            pair_codes_row<BITS>(rowfull, i, clo, chi);
             float x = kdq[i * K + clo], y = kdq[(i + NP) * K + chi];
             for (int f = e0; f < e1; ++f) {
               const uint32_t ef = ents[f];
@@ -266,7 +319,7 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
           }
         }
       } else {
-        const float2 lp = valid ? a.v_params[bh * a.T_cap + slot] : make_float2(0.f, 0.f);
+        const float2 lp = vpar[tok];
 #pragma unroll
         for (int jj = 0; jj < HALF_PAIRS; jj += 4) {
           uint32_t pv[4];
@@ -283,7 +336,7 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
           *reinterpret_cast<uint4*>(tile + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
         }
         if (valid) {
-          const uint32_t* ents = a.v_out + (bh * a.T_cap + slot) * a.n_v;
+          const uint32_t* ents = stage_vout ? vouts + tok * Lay::NVS : a.v_out + (bh * a.T_cap + slot) * a.n_v;
           for (int e = 0; e < a.n_v; ++e) {
             const uint32_t ev = ents[e];
             const int ch = (int)(ev >> 16);

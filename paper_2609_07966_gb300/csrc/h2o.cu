@@ -1,0 +1,187 @@
+// H2O heavy-hitter eviction (Section 2.1, H2O paragraph): initial keep after
+// the prompt's accumulated scores, and the per-step score update + eviction.
+//
+// Keep: the `recent` newest positions, plus the `heavy` best of the rest under
+// (score desc, position asc) -- an exact radix top-k on unique 64-bit keys --
+// gathered in ascending position into slots 0.. of the cache.
+// Step: acc[slot] += sum_h 2^(x_h(slot) - m_h) / l_h for every held slot (the
+// softmax probability from the decode call), then, if more than heavy+recent
+// tokens are held, evict among all but the `recent` newest positions the one
+// that ranks last under (acc desc, position asc): lowest acc, on a tie the
+// higher position.  Its slot becomes the next append slot.
+#include <math.h>
+
+#include "mkv_common.cuh"
+#include "mkv_internal.h"
+#include "mkv_select.cuh"
+
+namespace mkv {
+
+namespace {
+
+constexpr int kSelThreads = 1024;
+
+// One CTA per (batch, kv-head): flags of kept positions -> ascending keep list.
+__global__ void __launch_bounds__(kSelThreads) h2o_keep_kernel(const float* __restrict__ score, int64_t T, int H,
+                                                               int R, int32_t* __restrict__ keep_out,
+                                                               int32_t* __restrict__ n_keep_out) {
+  __shared__ int hist[256];
+  __shared__ int warp_sums[32];
+  const int64_t bh = blockIdx.x;
+  const float* s = score + bh * T;
+  int32_t* keep = keep_out + bh * T;
+  const int64_t n_cand = T > R ? T - R : 0;           // positions 0 .. T-R-1 compete
+  const int heavy = (int)(n_cand < (int64_t)H ? n_cand : (int64_t)H);
+  uint64_t thr = ~0ull;
+  if (heavy > 0) {
+    thr = block_kth_largest((int)n_cand, heavy, [&](int i) { return rank_key(s[i], (uint32_t)i); }, hist);
+  }
+  // stream compaction in ascending position
+  int64_t base = 0;
+  for (int64_t i0 = 0; i0 < T; i0 += blockDim.x) {
+    const int64_t i = i0 + threadIdx.x;
+    int flag = 0;
+    if (i < T) flag = (i >= n_cand) || (heavy > 0 && rank_key(s[i], (uint32_t)i) >= thr);
+    int total;
+    const int before = block_exclusive_scan(flag, warp_sums, &total);
+    if (flag) keep[base + before] = (int32_t)i;
+    base += total;
+  }
+  if (threadIdx.x == 0) n_keep_out[bh] = (int32_t)base;
+}
+
+// Copy the kept rows into the cache and set pos/acc/slot, T_len.
+__global__ void h2o_gather_kernel(const __half* __restrict__ full_k, const __half* __restrict__ full_v,
+                                  const float* __restrict__ score, const int32_t* __restrict__ keep,
+                                  const int32_t* __restrict__ n_keep, int64_t T, int Hkv, int D, int64_t T_cap,
+                                  __half* k, __half* v, int32_t* pos, float* acc, int32_t* slot, int32_t* T_len) {
+  const int64_t bh = blockIdx.y;
+  const int n = n_keep[bh];
+  const int nc = D / 8;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < T_cap * nc; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t sl = e / nc;
+    const int col = (int)(e % nc);
+    if (sl < n) {
+      const int64_t p = keep[bh * T + sl];
+      reinterpret_cast<uint4*>(k + (bh * T_cap + sl) * D)[col] = reinterpret_cast<const uint4*>(full_k + (bh * T + p) * D)[col];
+      reinterpret_cast<uint4*>(v + (bh * T_cap + sl) * D)[col] = reinterpret_cast<const uint4*>(full_v + (bh * T + p) * D)[col];
+      if (col == 0) {
+        pos[bh * T_cap + sl] = (int32_t)p;
+        acc[bh * T_cap + sl] = score[bh * T + p];
+      }
+    } else if (col == 0) {
+      pos[bh * T_cap + sl] = -1;
+      acc[bh * T_cap + sl] = 0.f;
+    }
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    slot[bh] = n;            // first free slot
+    if (bh % Hkv == 0) T_len[bh / Hkv] = (int32_t)T;
+  }
+}
+
+// One CTA per (batch, kv-head): score update and eviction.
+__global__ void __launch_bounds__(256) h2o_update_kernel(const float* __restrict__ logits, const float* __restrict__ m_tot,
+                                                         const float* __restrict__ l_tot, int Hkv, int G, int64_t T_cap,
+                                                         int H, int R, const int32_t* __restrict__ T_len,
+                                                         int32_t* __restrict__ pos, float* __restrict__ acc,
+                                                         int32_t* __restrict__ slot_out) {
+  const int64_t bh = blockIdx.x;
+  const int b = (int)(bh / Hkv), kvh = (int)(bh % Hkv);
+  const int64_t newest = (int64_t)T_len[b] - 1;
+  float m[8], il[8];
+  for (int h = 0; h < G; ++h) {
+    const int64_t hq = (int64_t)b * Hkv * G + (int64_t)kvh * G + h;
+    m[h] = m_tot[hq];
+    il[h] = l_tot[hq] > 0.f ? 1.f / l_tot[hq] : 0.f;
+  }
+  int held = 0;
+  uint64_t best = ~0ull;          // minimum key among candidates -> evicted
+  int best_slot = -1, first_free = INT32_MAX;
+  for (int64_t s = threadIdx.x; s < T_cap; s += blockDim.x) {
+    const int32_t p = pos[bh * T_cap + s];
+    if (p < 0) {
+      first_free = min(first_free, (int)s);
+      continue;
+    }
+    ++held;
+    float add = 0.f;
+    for (int h = 0; h < G; ++h) add += exp2f(logits[(bh * T_cap + s) * G + h] - m[h]) * il[h];
+    const float a2 = acc[bh * T_cap + s] + add;
+    acc[bh * T_cap + s] = a2;
+    if ((int64_t)p <= newest - R) {
+      const uint64_t key = rank_key(a2, (uint32_t)p);
+      if (key < best) {
+        best = key;
+        best_slot = (int)s;
+      }
+    }
+  }
+  // block reductions: held count, first free slot, min key (with its slot)
+  __shared__ int s_held[8], s_free[8];
+  __shared__ uint64_t s_key[8];
+  __shared__ int s_slot[8];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int o = 16; o > 0; o >>= 1) {
+    held += __shfl_xor_sync(0xffffffffu, held, o);
+    first_free = min(first_free, __shfl_xor_sync(0xffffffffu, first_free, o));
+    const uint64_t ok = __shfl_xor_sync(0xffffffffu, best, o);
+    const int os = __shfl_xor_sync(0xffffffffu, best_slot, o);
+    if (ok < best) {
+      best = ok;
+      best_slot = os;
+    }
+  }
+  if (lane == 0) {
+    s_held[warp] = held;
+    s_free[warp] = first_free;
+    s_key[warp] = best;
+    s_slot[warp] = best_slot;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int hsum = 0, ff = INT32_MAX, bs = -1;
+    uint64_t bk = ~0ull;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+      hsum += s_held[w];
+      ff = min(ff, s_free[w]);
+      if (s_key[w] < bk) {
+        bk = s_key[w];
+        bs = s_slot[w];
+      }
+    }
+    if (hsum > H + R && bs >= 0) {
+      pos[bh * T_cap + bs] = -1;
+      slot_out[bh] = bs;
+    } else {
+      slot_out[bh] = ff == INT32_MAX ? -1 : ff;
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_h2o_keep(const mkv_config& c, const void* full_k, const void* full_v, int64_t T,
+                            const mkv_cache& cache, const PrefillWs& ws, cudaStream_t st) {
+  const int units = c.B * c.Hkv;
+  int32_t* n_keep = reinterpret_cast<int32_t*>(ws.row_l);   // row stats are dead after scoring
+  h2o_keep_kernel<<<units, kSelThreads, 0, st>>>(ws.score, T, c.h2o_heavy, c.h2o_recent, ws.keep, n_keep);
+  cudaError_t e = cudaPeekAtLastError();
+  if (e != cudaSuccess) return e;
+  const int64_t work = cache.T_cap * (c.D / 8);
+  const int bx = (int)std::min<int64_t>(ceil_div(work, 256), 64);
+  h2o_gather_kernel<<<dim3(bx, units), 256, 0, st>>>(
+      static_cast<const __half*>(full_k), static_cast<const __half*>(full_v), ws.score, ws.keep, n_keep, T, c.Hkv,
+      c.D, cache.T_cap, static_cast<__half*>(cache.k), static_cast<__half*>(cache.v), cache.pos, cache.acc,
+      cache.slot, cache.T_len);
+  return cudaPeekAtLastError();
+}
+
+cudaError_t launch_h2o_update(const mkv_config& c, const mkv_cache& cache, const DecodeWs& ws, cudaStream_t st) {
+  h2o_update_kernel<<<c.B * c.Hkv, 256, 0, st>>>(ws.logits, ws.m_tot, ws.l_tot, c.Hkv, c.Hq / c.Hkv, cache.T_cap,
+                                                 c.h2o_heavy, c.h2o_recent, cache.T_len, cache.pos, cache.acc,
+                                                 cache.slot);
+  return cudaPeekAtLastError();
+}
+
+}  // namespace mkv

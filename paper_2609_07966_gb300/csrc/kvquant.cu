@@ -87,6 +87,10 @@ __global__ void quantize_kernel(const QuantArgs a) {
   __shared__ float s_lo[32], s_hi[32];
 
   const int64_t t_base = a.T_len[b];
+  if (t_base < 0 || t_base + a.n_tokens > a.T_cap) {   // no room: drop, flag, keep T_len
+    if (c == 0 && h == 0) atomicOr(&g_status_kvquant, MKV_FLAG_CACHE_FULL);
+    return;
+  }
   const int rowb = D * a.bits / 8;
   const int nwords = (rowb + 3) / 4;
   // per-channel parameters
@@ -206,10 +210,11 @@ __global__ void quantize_kernel(const QuantArgs a) {
   }
 }
 
-// T_len[b] += n after every (b, h) CTA of quantize_kernel finished (stream order).
-__global__ void advance_kernel(int32_t* T_len, int B, int64_t n) {
+// T_len[b] += n after every (b, h) CTA of quantize_kernel finished (stream order);
+// a batch entry without room was left unwritten and keeps its length.
+__global__ void advance_kernel(int32_t* T_len, int B, int64_t n, int64_t T_cap) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b < B) T_len[b] += (int32_t)n;
+  if (b < B && T_len[b] >= 0 && T_len[b] + n <= T_cap) T_len[b] += (int32_t)n;
 }
 
 // ----------------------------------------------------------------- calibrate
@@ -461,7 +466,7 @@ cudaError_t launch_quantize(const mkv_config& c, const mkv_quant_params& qp, con
   quantize_kernel<<<c.B * c.Hkv, c.D, smem, st>>>(a);
   cudaError_t e = cudaPeekAtLastError();
   if (e != cudaSuccess) return e;
-  advance_kernel<<<(c.B + 127) / 128, 128, 0, st>>>(cache.T_len, c.B, n_tokens);
+  advance_kernel<<<(c.B + 127) / 128, 128, 0, st>>>(cache.T_len, c.B, n_tokens, cache.T_cap);
   return cudaPeekAtLastError();
 }
 

@@ -1,0 +1,196 @@
+// RocketKV (Section 2.1, RocketKV paragraph).
+// Stage 1, SnapKV prefill compression: the observation window's aggregated
+// scores of the prefix (prefill.cu), max-pooled over |j' - j| <= pool/2,
+// the keep - W best prefix positions under (pooled desc, position asc) plus
+// the window, gathered in ascending position; per-page key min/max of the
+// compact cache.
+// Stage 2, page choice at decode: dims = the topq_dims largest sum_h |q_h,i|
+// (dim asc on ties), page score = sum_h sum_{i in dims}
+// max(q_h,i kmin_i, q_h,i kmax_i) over full pages before the newest token's,
+// best topk_pages under (score desc, page asc), listed ascending.
+#include <math.h>
+
+#include "mkv_common.cuh"
+#include "mkv_internal.h"
+#include "mkv_select.cuh"
+
+namespace mkv {
+
+namespace {
+
+constexpr int kSelThreads = 1024;
+
+__device__ __forceinline__ float pooled_at(const float* s, int64_t n, int64_t j, int r) {
+  float m = -INFINITY;
+  const int64_t lo = j - r < 0 ? 0 : j - r, hi = j + r >= n ? n - 1 : j + r;
+  for (int64_t i = lo; i <= hi; ++i) m = fmaxf(m, s[i]);
+  return m;
+}
+
+// One CTA per (batch, kv-head): keep list (ascending) of the compressed cache.
+__global__ void __launch_bounds__(kSelThreads) snap_keep_kernel(const float* __restrict__ score, int64_t T, int W,
+                                                                int pool, int keep, float* __restrict__ pooled_ws,
+                                                                int32_t* __restrict__ keep_out) {
+  __shared__ int hist[256];
+  __shared__ int warp_sums[32];
+  const int64_t bh = blockIdx.x;
+  const int64_t n = T - W;                        // prefix positions compete
+  const float* s = score + bh * T;
+  float* pooled = pooled_ws + bh * T;
+  int32_t* out = keep_out + bh * T;
+  const int r = pool / 2;
+  for (int64_t j = threadIdx.x; j < n; j += blockDim.x) pooled[j] = pooled_at(s, n, j, r);
+  __syncthreads();
+  const int k = keep - W;
+  uint64_t thr = ~0ull;
+  if (k > 0) thr = block_kth_largest((int)n, k, [&](int i) { return rank_key(pooled[i], (uint32_t)i); }, hist);
+  int64_t base = 0;
+  for (int64_t i0 = 0; i0 < T; i0 += blockDim.x) {
+    const int64_t i = i0 + threadIdx.x;
+    int flag = 0;
+    if (i < T) flag = (i >= n) || (k > 0 && rank_key(pooled[i], (uint32_t)i) >= thr);
+    int total;
+    const int before = block_exclusive_scan(flag, warp_sums, &total);
+    if (flag) out[base + before] = (int32_t)i;
+    base += total;
+  }
+}
+
+// Gather kept rows (keep list, or the identity when keep >= T) into slots 0..n-1.
+__global__ void snap_gather_kernel(const __half* __restrict__ full_k, const __half* __restrict__ full_v,
+                                   const int32_t* __restrict__ keep, int identity, int64_t T, int64_t n, int Hkv,
+                                   int D, int64_t T_cap, __half* k, __half* v, int32_t* kept_pos, int32_t* T_len) {
+  const int64_t bh = blockIdx.y;
+  const int nc = D / 8;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n * nc; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t sl = e / nc;
+    const int col = (int)(e % nc);
+    const int64_t p = identity ? sl : keep[bh * T + sl];
+    reinterpret_cast<uint4*>(k + (bh * T_cap + sl) * D)[col] = reinterpret_cast<const uint4*>(full_k + (bh * T + p) * D)[col];
+    reinterpret_cast<uint4*>(v + (bh * T_cap + sl) * D)[col] = reinterpret_cast<const uint4*>(full_v + (bh * T + p) * D)[col];
+    if (col == 0 && kept_pos) kept_pos[bh * n + sl] = (int32_t)p;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0 && bh % Hkv == 0) T_len[bh / Hkv] = (int32_t)n;
+}
+
+// kmin/kmax [bh][D][T_cap/16] of every full page among slots 0..n-1.
+__global__ void page_meta_kernel(const __half* __restrict__ k, int64_t T_cap, int D, int64_t n, __half* kmin,
+                                 __half* kmax) {
+  const int64_t bh = blockIdx.y;
+  const int64_t npc = T_cap / kPage, np = n / kPage;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < np * D; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t p = e / D;
+    const int d = (int)(e % D);
+    const __half* base = k + (bh * T_cap + p * kPage) * D + d;
+    __half lo = base[0], hi = base[0];
+    for (int j = 1; j < kPage; ++j) {
+      const __half x = base[(int64_t)j * D];
+      lo = __hlt(x, lo) ? x : lo;
+      hi = __hgt(x, hi) ? x : hi;
+    }
+    kmin[(bh * D + d) * npc + p] = lo;
+    kmax[(bh * D + d) * npc + p] = hi;
+  }
+}
+
+// One CTA per (batch, kv-head): dims, page scores, top-k pages.
+__global__ void __launch_bounds__(kSelThreads) rocket_select_kernel(const __half* __restrict__ q, const __half* __restrict__ kmin,
+                                                                    const __half* __restrict__ kmax,
+                                                                    const int32_t* __restrict__ T_len, int Hkv, int G, int D,
+                                                                    int64_t T_cap, int kp, int rd, int32_t* __restrict__ out) {
+  extern __shared__ float sm[];
+  float* qs = sm;                       // [G][D]
+  float* ssc = qs + G * D;              // [npc] page scores
+  __shared__ int hist[256];
+  __shared__ int warp_sums[32];
+  __shared__ int dims[128];
+  __shared__ float a_dim[128];
+  const int64_t bh = blockIdx.x;
+  const int b = (int)(bh / Hkv), kvh = (int)(bh % Hkv);
+  const int64_t npc = T_cap / kPage;
+  const int n = (int)min((int64_t)T_len[b], T_cap);
+  const int ns = n > 0 ? (n - 1) / kPage : 0;
+  for (int e = threadIdx.x; e < G * D; e += blockDim.x) qs[e] = __half2float(q[((int64_t)b * Hkv * G + (int64_t)kvh * G) * D + e]);
+  __syncthreads();
+  if (threadIdx.x < D) {
+    float a = 0.f;
+    for (int h = 0; h < G; ++h) a += fabsf(qs[h * D + threadIdx.x]);
+    a_dim[threadIdx.x] = a;
+  }
+  __syncthreads();
+  if (threadIdx.x < D) {
+    const uint64_t mine = rank_key(a_dim[threadIdx.x], (uint32_t)threadIdx.x);
+    int rank = 0;
+    for (int j = 0; j < D; ++j) rank += rank_key(a_dim[j], (uint32_t)j) > mine ? 1 : 0;
+    if (rank < rd) dims[rank] = threadIdx.x;
+  }
+  __syncthreads();
+  for (int p = threadIdx.x; p < ns; p += blockDim.x) {
+    float sc = 0.f;
+    for (int h = 0; h < G; ++h) {
+      for (int t = 0; t < rd; ++t) {
+        const int i = dims[t];
+        const float qv = qs[h * D + i];
+        const float lo = __half2float(kmin[(bh * D + i) * npc + p]) * qv;
+        const float hi = __half2float(kmax[(bh * D + i) * npc + p]) * qv;
+        sc += fmaxf(lo, hi);
+      }
+    }
+    ssc[p] = sc;
+  }
+  __syncthreads();
+  const int k = min(kp, ns);
+  uint64_t thr = ~0ull;
+  if (k > 0) thr = block_kth_largest(ns, k, [&](int i) { return rank_key(ssc[i], (uint32_t)i); }, hist);
+  int base = 0;
+  for (int i0 = 0; i0 < ns; i0 += blockDim.x) {
+    const int i = i0 + threadIdx.x;
+    const int flag = (i < ns && k > 0 && rank_key(ssc[i], (uint32_t)i) >= thr) ? 1 : 0;
+    int total;
+    const int before = block_exclusive_scan(flag, warp_sums, &total);
+    if (flag) out[bh * kp + base + before] = i;
+    base += total;
+  }
+  for (int i = base + threadIdx.x; i < kp; i += blockDim.x) out[bh * kp + i] = -1;
+}
+
+}  // namespace
+
+cudaError_t launch_snap_keep(const mkv_config& c, const void* full_k, const void* full_v, int64_t T,
+                             const mkv_cache& cache, int32_t* kept_pos, const PrefillWs& ws, cudaStream_t st) {
+  const int units = c.B * c.Hkv;
+  const bool identity = T <= c.snap_keep;
+  const int64_t n = identity ? T : c.snap_keep;
+  if (!identity) {
+    snap_keep_kernel<<<units, kSelThreads, 0, st>>>(ws.score, T, c.snap_window, c.snap_pool, c.snap_keep, ws.row_m,
+                                                    ws.keep);
+    cudaError_t e = cudaPeekAtLastError();
+    if (e != cudaSuccess) return e;
+  }
+  const int bx = (int)std::min<int64_t>(ceil_div(n * (c.D / 8), 256), 128);
+  snap_gather_kernel<<<dim3(bx, units), 256, 0, st>>>(
+      static_cast<const __half*>(full_k), static_cast<const __half*>(full_v), ws.keep, identity ? 1 : 0, T, n, c.Hkv,
+      c.D, cache.T_cap, static_cast<__half*>(cache.k), static_cast<__half*>(cache.v), kept_pos, cache.T_len);
+  cudaError_t e = cudaPeekAtLastError();
+  if (e != cudaSuccess) return e;
+  const int bm = (int)std::min<int64_t>(ceil_div((n / kPage) * c.D, 256), 128);
+  if (n >= kPage) {
+    page_meta_kernel<<<dim3(bm, units), 256, 0, st>>>(static_cast<const __half*>(cache.k), cache.T_cap, c.D, n,
+                                                      static_cast<__half*>(cache.kmin), static_cast<__half*>(cache.kmax));
+  }
+  return cudaPeekAtLastError();
+}
+
+cudaError_t launch_rocket_select(const mkv_config& c, const void* q, const mkv_cache& cache, int32_t* page_idx,
+                                 cudaStream_t st) {
+  const int G = c.Hq / c.Hkv;
+  const size_t smem = ((size_t)G * c.D + cache.T_cap / kPage) * sizeof(float);
+  cudaError_t e = cudaFuncSetAttribute(rocket_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  rocket_select_kernel<<<c.B * c.Hkv, kSelThreads, smem, st>>>(
+      static_cast<const __half*>(q), static_cast<const __half*>(cache.kmin), static_cast<const __half*>(cache.kmax),
+      cache.T_len, c.Hkv, G, c.D, cache.T_cap, c.topk_pages, c.topq_dims, page_idx);
+  return cudaPeekAtLastError();
+}
+
+}  // namespace mkv

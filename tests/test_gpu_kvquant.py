@@ -186,7 +186,7 @@ def test_decode_tiny_workload():
     k, v = x["k"][0], x["v"][0]
     plist = _oracle_params(k, v, w.T, w.bits, w.quant_mode, w.outlier_frac)
     cfg = make_cfg(w.B, w.Hq, w.Hkv, w.D, w.bits, w.quant_mode, w.outlier_frac, w.theta)
-    cache, qp = _quantized_cache(cfg, k, v, plist, w.T, 0, dev)
+    cache, qp = _quantized_cache(cfg, k, v, plist, w.T, 0, dev, T_cap=w.T + w.steps)
     ws, nws = caches.workspace(cfg, cache.T_cap, device=dev)
     for s in range(w.steps):
         kn, vn = to_dev(k[:, :, w.T + s:w.T + s + 1], dev), to_dev(v[:, :, w.T + s:w.T + s + 1], dev)
@@ -215,6 +215,22 @@ def test_decode_shapes_ragged(D, G):
 def test_decode_all_outliers_equals_fp16_path():
     """outlier_frac = 1: every entry is stored exactly, so the fused path is plain attention."""
     _decode_vs_oracle(B=1, Hq=8, Hkv=2, D=64, bits=2, mode="uniform", T=130, steps=1, seed=77, frac=1.0)
+
+
+def test_quantize_capacity_flag():
+    """An append past T_cap writes nothing, keeps T_len and raises MKV_FLAG_CACHE_FULL."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    k, v = _data(1, 2, 40, 64, seed=3)
+    plist = _oracle_params(k, v, 32, 4, "uniform", 0.01)
+    cfg = make_cfg(1, 4, 2, 64, 4, "uniform")
+    cache, qp = _quantized_cache(cfg, k, v, plist, 32, 0, dev, T_cap=32)
+    before = cache.t["k_codes"].clone()
+    kn, vn = to_dev(k[:, :, 32:33], dev), to_dev(v[:, :, 32:33], dev)
+    mkv.mkv_quantize_kv(cfg, qp.c, kn.data_ptr(), vn.data_ptr(), 1, cache.c)
+    assert mkv.mkv_get_status() == mkv.MKV_FLAG_CACHE_FULL
+    assert int(cache.t["T_len"][0]) == 32
+    assert torch.equal(before, cache.t["k_codes"])
 
 
 def test_decode_full_size_sampled():

@@ -1,0 +1,138 @@
+"""GPU parity: SnapKV prefill compression, page metadata, page selection and sparse decode."""
+import numpy as np
+import pytest
+
+import paper_2609_07966_gb300 as mkv
+import synth
+from oracle import attention, rocket, snapkv
+from paper_2609_07966_gb300 import caches
+
+from gpu_util import assert_close, to_dev, torch_cuda
+from lockstep import check_topk, tiny_seed
+
+pytestmark = pytest.mark.gpu
+
+
+def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev, exact, units, tag):
+    """K, V [B,Hkv,T+steps,D]; QW [B,Hq,W,D] window queries; Q [steps,B,Hq,D] (device tensors)."""
+    torch = torch_cuda()
+    G = Hq // Hkv
+    cfg = mkv.config(mkv.MKV_ROCKET, B, Hq, Hkv, D, snap_window=W, snap_pool=pool, snap_keep=keep,
+                     page_size=16, topk_pages=kp, topq_dims=rd)
+    kept_n = min(T, keep)
+    T_cap = (kept_n + steps + 15) // 16 * 16
+    cache = caches.alloc_cache(cfg, T_cap, device=dev)
+    ws, nws = caches.workspace(cfg, max(T, T_cap), device=dev)
+    kept_pos = torch.zeros((B, Hkv, kept_n), dtype=torch.int32, device=dev)
+    Kp, Vp = K[:, :, :T].contiguous(), V[:, :, :T].contiguous()
+    mkv.mkv_snap_compress(cfg, QW.data_ptr(), Kp.data_ptr(), Vp.data_ptr(), T, cache.c, kept_pos.data_ptr(),
+                          ws.data_ptr(), nws)
+    torch.cuda.synchronize()
+    assert int(cache.t["T_len"][0]) == kept_n
+    near = 0
+    host = {}
+    for (b, h) in units:
+        k = K[b, h].cpu().numpy()
+        v = V[b, h].cpu().numpy()
+        qw = QW[b, h * G:(h + 1) * G].cpu().numpy()
+        got = kept_pos[b, h].cpu().numpy()
+        assert np.all(np.diff(got) > 0), "kept positions must ascend"
+        if keep >= T:
+            assert np.array_equal(got, np.arange(T))
+        else:
+            s = snapkv.window_scores(qw, k[:T])
+            pooled = snapkv.max_pool(s, pool)
+            pre = np.arange(T - W)
+            near += check_topk(pooled, pre, keep - W, got[got < T - W], exact, f"{tag} snap b{b} h{h}")
+            assert np.array_equal(got[got >= T - W], np.arange(T - W, T))
+        # the compact cache holds exactly the kept rows, and page min/max match
+        gk = cache.t["k"][b, h, :kept_n].cpu().numpy()
+        assert np.array_equal(gk.view(np.uint16), k[got].view(np.uint16))
+        npg = kept_n // 16
+        kmin, kmax = rocket.page_minmax(k[got], 16, npg)
+        assert np.array_equal(cache.t["kmin"][b, h, :, :npg].cpu().numpy().T.astype(np.float64), kmin)
+        assert np.array_equal(cache.t["kmax"][b, h, :, :npg].cpu().numpy().T.astype(np.float64), kmax)
+        host[(b, h)] = (list(k[got]), list(v[got]), k, v)
+    page_idx = torch.zeros((B, Hkv, kp), dtype=torch.int32, device=dev)
+    for s in range(steps):
+        kn = K[:, :, T + s].contiguous()
+        vn = V[:, :, T + s].contiguous()
+        q = Q[s].contiguous()
+        out = torch.empty_like(q)
+        mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
+        mkv.mkv_rocket_select(cfg, q.data_ptr(), cache.c, page_idx.data_ptr())
+        mkv.mkv_decode_attention(cfg, q.data_ptr(), cache.c, None, page_idx.data_ptr(), out.data_ptr(), ws.data_ptr(),
+                                 nws)
+        got = out.float().cpu().numpy()
+        pidx = page_idx.cpu().numpy()
+        for (b, h) in units:
+            Kc, Vc, k, v = host[(b, h)]
+            Kc.append(k[T + s])
+            Vc.append(v[T + s])
+            n = len(Kc)
+            qh = q[b, h * G:(h + 1) * G].cpu().numpy()
+            sel_ref, scores = rocket.select_pages(qh, np.array(Kc), n, 16, kp, rd)
+            sel_got = pidx[b, h][pidx[b, h] >= 0]
+            assert np.all(np.diff(sel_got) > 0), "pages must ascend"
+            ns = rocket.n_scored_pages(n, 16)
+            nn = check_topk(scores, np.arange(ns), min(kp, ns), sel_got, exact, f"{tag} pages step {s} b{b} h{h}")
+            near += nn
+            ref, _, _ = rocket.decode(qh, np.array(Kc), np.array(Vc), n, 16, kp, rd, forced_pages=sel_got)
+            assert_close(got[b, h * G:(h + 1) * G], ref, f"{tag} step {s} b{b} h{h}")
+    assert mkv.mkv_get_status() == 0
+    return near
+
+
+def test_tiny_exact():
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    w = synth.tiny()
+    x = synth.host_inputs(w, seed=tiny_seed())
+    K, V = to_dev(x["k"][0], dev), to_dev(x["v"][0], dev)
+    QW = to_dev(x["q_prompt"][0, :, :, w.T - w.snap_window:], dev)
+    Q = to_dev(x["q"][:, 0], dev)
+    near = run_rocket(w.B, w.Hq, w.Hkv, w.D, w.T, w.steps, w.snap_window, w.snap_pool, w.snap_keep, w.topk_pages,
+                      w.topq_dims, K, V, QW, Q, dev, True, [(0, 0), (0, 1)], "tiny")
+    assert near == 0
+
+
+def test_keep_everything_is_full_attention():
+    """keep >= T and k_p >= pages: every step attends the whole cache."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(8)
+    B, Hq, Hkv, D, T, steps = 2, 8, 2, 64, 150, 3
+    K = rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16)
+    V = rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16)
+    QW = rng.standard_normal((B, Hq, 8, D)).astype(np.float16)
+    Q = rng.standard_normal((steps, B, Hq, D)).astype(np.float16)
+    run_rocket(B, Hq, Hkv, D, T, steps, 8, 7, 160, 64, 16, to_dev(K, dev), to_dev(V, dev), to_dev(QW, dev),
+               to_dev(Q, dev), dev, False, [(0, 0), (1, 1)], "all")
+
+
+@pytest.mark.parametrize("G,D", [(1, 128), (8, 64)])
+def test_shapes_lockstep(G, D):
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(G + D)
+    B, Hkv, T, steps, W = 2, 2, 700, 5, 16
+    Hq = G * Hkv
+    K = rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16)
+    V = rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16)
+    QW = rng.standard_normal((B, Hq, W, D)).astype(np.float16)
+    Q = rng.standard_normal((steps, B, Hq, D)).astype(np.float16)
+    run_rocket(B, Hq, Hkv, D, T, steps, W, 7, 300, 6, D // 4, to_dev(K, dev), to_dev(V, dev), to_dev(QW, dev),
+               to_dev(Q, dev), dev, False, [(0, 1), (1, 0)], f"G{G}D{D}")
+
+
+def test_full_size_lockstep():
+    """B=4, T=32768 -> keep 4096, W=32, pool 7, top-64 pages over top-32 dims: one layer,
+    16 steps, two (batch, kv-head) units in lockstep with the oracle."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    w = synth.rocket_32k(1024)
+    x = synth.device_layer_inputs(w, seed=12, layer=0, device=dev, n_tokens=w.T + 16, with_prompt_queries=True)
+    QW = x["q_prompt"][:, :, w.T - w.snap_window:].contiguous()
+    near = run_rocket(w.B, w.Hq, w.Hkv, w.D, w.T, 16, w.snap_window, w.snap_pool, w.snap_keep, w.topk_pages,
+                      w.topq_dims, x["k"], x["v"], QW, x["q"][:16], dev, False, [(0, 0), (3, 7)], "rocket32k")
+    print(f"near-ties adopted: {near}")
