@@ -343,12 +343,19 @@ def main():
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--layers", type=int, default=None,
+                    help="profiling only: fewer layers than the workload (the line is then not a bench number)")
+    ap.add_argument("--profile", action="store_true",
+                    help="profiling only: run warmup + steps and exit (for ncu), no JSON line")
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     w = WORKLOADS[args.workload]()
+    if args.layers is not None:
+        import dataclasses
+        w = dataclasses.replace(w, L=args.layers)
     config = {"workload": w.name, "method": METHOD_OF[args.workload], "batch": w.B, "context": w.T, "layers": w.L,
               "heads_q": w.Hq, "heads_kv": w.Hkv, "head_dim": w.D, "l2": "inputs larger than L2 (no flush)"}
 
@@ -383,6 +390,11 @@ def main():
     runner = Runner(args.workload, w, dev, args.seed + rank, extra_steps=4 * total + 8)
     if not args.no_graph:
         runner.capture()
+    if args.profile:
+        for _ in range(total):
+            runner.run_step()
+        torch.cuda.synchronize()
+        return
 
     if world > 1:
         torch.distributed.barrier()

@@ -43,8 +43,8 @@ def alloc_cache(cfg, T_cap: int, device="cuda", k_out_cap: int | None = None) ->
     if cfg.method == MKV_KVQUANT:
         row = D * cfg.bits // 8
         nv = n_value_outliers(D, cfg.outlier_frac)
-        if k_out_cap is None:
-            k_out_cap = max(64, int(T_cap * D * max(cfg.outlier_frac, 1e-6) * 2) + 64)
+        if k_out_cap is None:   # 4x the nominal outlier rate (data beyond the calibration range)
+            k_out_cap = int(T_cap * D * min(1.0, max(cfg.outlier_frac, 1e-6) * 4)) + 1024
         t["k_codes"] = torch.zeros((B, Hkv, T_cap, row), dtype=torch.uint8, device=device)
         t["v_codes"] = torch.zeros((B, Hkv, T_cap, row), dtype=torch.uint8, device=device)
         t["v_params"] = torch.zeros((B, Hkv, T_cap, 2), dtype=torch.float32, device=device)

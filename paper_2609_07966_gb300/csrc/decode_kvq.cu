@@ -61,12 +61,13 @@ struct KvqLayout {
   static constexpr int SROW = ((SROW0 / 16) % 2 == 0) ? SROW0 + 16 : SROW0;   // odd # of 16B
   static constexpr int TILE = kChunk * D * 2;                // fp16 tile bytes
   static constexpr int NVS = 4;                              // value outliers staged per token (<=)
+  static constexpr int KE_CAP = 128;                         // key outliers staged per chunk (<=)
   // one pipeline stage: codes, then the chunk's per-token side data
   static constexpr int S_KC = 0;                             // [64][SROW] key codes
   static constexpr int S_VC = S_KC + kChunk * SROW;          // [64][SROW] value codes
   static constexpr int S_VP = S_VC + kChunk * SROW;          // [64] float2 (lo, scale)
-  static constexpr int S_KO = S_VP + kChunk * 8;             // [68] int32 key-outlier CSR offsets
-  static constexpr int S_VO = S_KO + 68 * 4;                 // [64][NVS] uint32 value outliers
+  static constexpr int S_KE = S_VP + kChunk * 8;             // [KE_CAP] uint32 key outliers of the chunk
+  static constexpr int S_VO = S_KE + KE_CAP * 4;             // [64][NVS] uint32 value outliers
   static constexpr int S_RP = S_VO + kChunk * NVS * 4;       // [2][NP] float2 rotations of the bases
   static constexpr int STAGE = S_RP + 2 * NP * 8;
   // byte offsets
@@ -76,7 +77,8 @@ struct KvqLayout {
   static constexpr int QRAW = VTB + D * K * 2;               // [8][D] half (the group's queries)
   static constexpr int QHI = QRAW + 8 * D * 2;               // [2 bases][8][NP] half2 (rotated query, hi)
   static constexpr int QLO = QHI + 2 * 8 * NP * 4;           // [2][8][NP] half2 (lo)
-  static constexpr int STG = QLO + 2 * 8 * NP * 4;           // [2 stages][STAGE]
+  static constexpr int KOFF = QLO + 2 * 8 * NP * 4;          // [3 chunks][68] int32 key-outlier CSR offsets
+  static constexpr int STG = KOFF + 3 * 68 * 4;              // [2 stages][STAGE]
   static constexpr int KHI = STG + 2 * STAGE;
   static constexpr int KLO = KHI + TILE;
   static constexpr int VT = KLO + TILE;
@@ -135,6 +137,7 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
   uint32_t* qlo = reinterpret_cast<uint32_t*>(smem + Lay::QLO);
   uint8_t* stg = smem + Lay::STG;
   __half* qraw = reinterpret_cast<__half*>(smem + Lay::QRAW);
+  int32_t* kring = reinterpret_cast<int32_t*>(smem + Lay::KOFF);
   uint8_t* khi_t = smem + Lay::KHI;
   uint8_t* klo_t = smem + Lay::KLO;
   uint8_t* v_t = smem + Lay::VT;
@@ -176,12 +179,8 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
       const int64_t s = c0 + tid;
       const bool ok = s < n_len;
       cp_async8(dst + Lay::S_VP + tid * 8, a.v_params + bh * a.T_cap + (ok ? s : 0), ok ? 8 : 0);
-    } else if (tid < kChunk + kChunk + 1) {      // CSR offsets c0 .. c0+64 (clamped to the cache)
-      const int i = tid - kChunk;
-      const int64_t s = min(c0 + i, (int64_t)n_len);
-      cp_async4(dst + Lay::S_KO + i * 4, a.k_out_off + bh * (a.T_cap + 1) + s, 4);
-    } else if (tid < 2 * kChunk + 1 + 2 * NP / 2) {   // rotations of the two 32-token bases
-      const int e = tid - (2 * kChunk + 1);           // 16-byte pieces: 2 float2 each
+    } else if (tid < kChunk + NP) {              // rotations of the two 32-token bases
+      const int e = tid - kChunk;                // 16-byte pieces: 2 float2 each
       const int base = e / (NP / 2), piece = e % (NP / 2);
       const int64_t tb = min(c0 + 32 * base, a.rope_len - 1);
       cp_async16(dst + Lay::S_RP + (base * NP + 2 * piece) * 8, a.rope + tb * NP + 2 * piece, 16);
@@ -197,8 +196,30 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     }
   };
 
+  // key-outlier CSR offsets run one chunk ahead of the codes so that each
+  // chunk's outlier entries can be staged together with its codes
+  auto load_koff = [&](int c) {
+    if (tid <= kChunk) {
+      const int64_t s = min(v_begin + (int64_t)c * kChunk + tid, (int64_t)n_len);
+      cp_async4(kring + (c % 3) * 68 + tid, a.k_out_off + bh * (a.T_cap + 1) + s, 4);
+    }
+  };
+  auto load_kents = [&](int c, int stage) {      // needs chunk c's offsets in kring
+    const int32_t* ko = kring + (c % 3) * 68;
+    const int e0 = ko[0];
+    const int n = min((int)min((int64_t)ko[kChunk], a.k_out_cap) - e0, Lay::KE_CAP);
+    for (int e = tid; e < n; e += kThr)
+      cp_async4(stg + stage * Lay::STAGE + Lay::S_KE + e * 4, a.k_out + bh * a.k_out_cap + e0 + e, 4);
+  };
   if (nchunks > 0) {
+    load_koff(0);
+    if (nchunks > 1) load_koff(1);
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
     load_chunk(0, 0);
+    load_kents(0, 0);
+    if (nchunks > 2) load_koff(2);
     cp_async_commit();
   }
   // CTA-resident tables: rotations by delta in [0, 32), dequant tables of this kv-head
@@ -223,12 +244,19 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
   for (int c = 0; c < nchunks; ++c) {
     cp_async_wait<0>();
     __syncthreads();
-    if (c + 1 < nchunks) load_chunk(c + 1, (c + 1) & 1);
+    if (c + 1 < nchunks) {
+      load_chunk(c + 1, (c + 1) & 1);
+      load_kents(c + 1, (c + 1) & 1);
+    }
+    if (c + 2 < nchunks) load_koff(c + 2);
     cp_async_commit();
     const int64_t t0 = v_begin + (int64_t)c * kChunk;      // position of the chunk's first token
     const uint8_t* st = stg + (c & 1) * Lay::STAGE;
     const float2* vpar = reinterpret_cast<const float2*>(st + Lay::S_VP);
-    const int32_t* koff = reinterpret_cast<const int32_t*>(st + Lay::S_KO);
+    const int32_t* koff = kring + (c % 3) * 68;
+    const uint32_t* kents = reinterpret_cast<const uint32_t*>(st + Lay::S_KE);
+    const int kbase = koff[0];
+    const int kstaged = min((int)min((int64_t)koff[kChunk], a.k_out_cap) - kbase, Lay::KE_CAP);
     const uint32_t* vouts = reinterpret_cast<const uint32_t*>(st + Lay::S_VO);
     const float2* rbase = reinterpret_cast<const float2*>(st + Lay::S_RP);
 
@@ -296,16 +324,17 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
         // key outliers of this token in this half: recompute their pair exactly
         if (valid) {
           const int e0 = koff[tok], e1 = (int)min((int64_t)koff[tok + 1], a.k_out_cap);
-          const uint32_t* ents = a.k_out + bh * a.k_out_cap;
+          const uint32_t* gents = a.k_out + bh * a.k_out_cap;
+          auto ent = [&](int e) { return e - kbase < kstaged ? kents[e - kbase] : gents[e]; };
           for (int e = e0; e < e1; ++e) {
-            const int ch = (int)(ents[e] >> 16);
+            const int ch = (int)(ent(e) >> 16);
             const int i = ch % NP;
             if (i / HALF_PAIRS != hp) continue;
             int clo, chi;
             pair_codes_row<BITS>(rowfull, i, clo, chi);
             float x = kdq[i * K + clo], y = kdq[(i + NP) * K + chi];
             for (int f = e0; f < e1; ++f) {
-              const uint32_t ef = ents[f];
+              const uint32_t ef = ent(f);
               const int cf = (int)(ef >> 16);
               if (cf == i) x = h2f((uint16_t)(ef & 0xffffu));
               if (cf == i + NP) y = h2f((uint16_t)(ef & 0xffffu));

@@ -28,13 +28,22 @@ Split decode_split(const mkv_config& c, int64_t T_cap) {
   s.v_tokens = c.method == MKV_ROCKET ? (int64_t)(c.topk_pages + 1) * kPage : T_cap;
   const int64_t chunks = std::max<int64_t>(1, ceil_div(s.v_tokens, kChunk));
   const int64_t units = (int64_t)c.B * c.Hkv;
-  // about four CTAs per SM in total (two resident per SM, two waves)
-  const int64_t target = 4 * kNumSMs;
-  int64_t n = std::min<int64_t>(chunks, std::max<int64_t>(1, ceil_div(target, units)));
-  const int64_t cps = ceil_div(chunks, n);
-  n = ceil_div(chunks, cps);
-  s.n_split = (int)n;
-  s.chunks_per_split = (int)cps;
+  // The decode kernels keep two CTAs resident per SM.  Pick the split count
+  // that minimises (waves of CTAs) x (chunks per CTA), i.e. the time of the
+  // busiest SM; among equals prefer fewer splits (smaller partials).
+  const int64_t slots = 2 * kNumSMs;
+  int64_t best_n = 1, best_cost = INT64_MAX;
+  for (int64_t n = 1; n <= std::min<int64_t>(chunks, 1024); ++n) {
+    const int64_t cps = ceil_div(chunks, n);
+    if (ceil_div(chunks, cps) != n) continue;      // n is not the split count of any cps
+    const int64_t cost = ceil_div(units * n, slots) * cps;
+    if (cost < best_cost) {
+      best_cost = cost;
+      best_n = n;
+    }
+  }
+  s.chunks_per_split = (int)ceil_div(chunks, best_n);
+  s.n_split = (int)ceil_div(chunks, s.chunks_per_split);
   return s;
 }
 
