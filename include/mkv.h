@@ -216,6 +216,31 @@ mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_
                                 const mkv_quant_params* qparams, const int32_t* page_idx,
                                 void* out, void* ws, size_t ws_bytes, void* stream);
 
+/* FP16 decode attention that allocates nothing and takes no workspace.
+ * No counterpart in the paper: it exists for callers that cannot call
+ * cudaMalloc or hand this library a scratch buffer -- for instance code that
+ * runs inside a host framework owning every device allocation, or an existing
+ * C interface with no place to pass a workspace.  It computes exactly what
+ * mkv_decode_attention computes for an FP16 cache (same kernels, same
+ * result); only the split partials live elsewhere: in one array of 8 MiB
+ * compiled into the library, which every GPU that loads the library keeps
+ * until the process exits.
+ *  - cfg->method must be MKV_FP16 (else MKV_ERR_UNSUPPORTED).
+ *  - The partials of B*Hq*n_split*(D+2) floats (what mkv_workspace_size
+ *    reports for this config and T_cap) must fit in 8 MiB, else
+ *    MKV_ERR_WORKSPACE and nothing is launched.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress) and caches it; make that first call before any
+ *    stream capture.
+ *  - All calls share the one array per device: calls whose kernels overlap on
+ *    the GPU (different streams, or a second call before the first finished
+ *    on another stream) race and corrupt each other's result.  Calls in order
+ *    on one stream are safe; every partial is rewritten before it is read, so
+ *    nothing has to be cleared between calls.
+ * q, out fp16 [B][Hq][D]; cache as for mkv_decode_attention. */
+mkv_status mkv_decode_attention_noalloc(const mkv_config* cfg, const void* q, const mkv_cache* cache,
+                                        void* out, void* stream);
+
 /* ------------------------------------------------------------- KVQuant */
 
 /* Learn one layer's calibration from the first N_cal tokens of the prompt:

@@ -79,6 +79,7 @@ _SIGS = {
     "mkv_h2o_update": [_CFG, _CACHE, _P, ctypes.c_size_t, _P],
     "mkv_snap_compress": [_CFG, _P, _P, _P, ctypes.c_int64, _CACHE, _P, _P, ctypes.c_size_t, _P],
     "mkv_rocket_select": [_CFG, _P, _CACHE, _P, _P],
+    "mkv_decode_attention_noalloc": [_CFG, _P, _CACHE, _P, _P],
 }
 
 
@@ -170,6 +171,10 @@ def mkv_decode_attention(cfg, q: int, cache: mkv_cache, qparams, page_idx: int, 
     _call("mkv_decode_attention", ctypes.byref(cfg), q, ctypes.byref(cache),
           ctypes.byref(qparams) if qparams is not None else None, page_idx, out, ws, ws_bytes,
           _stream(stream))
+
+
+def mkv_decode_attention_noalloc(cfg, q: int, cache: mkv_cache, out: int, stream=None):
+    _call("mkv_decode_attention_noalloc", ctypes.byref(cfg), q, ctypes.byref(cache), out, _stream(stream))
 
 
 def mkv_kvquant_calibrate(cfg, k_cal: int, v_cal: int, N_cal: int, row_stride: int, qparams, ws: int,

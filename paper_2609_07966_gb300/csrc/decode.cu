@@ -13,6 +13,8 @@
 // are merged by combine_kernel.
 #include <math.h>
 
+#include <mutex>
+
 #include "mkv_common.cuh"
 #include "mkv_internal.h"
 
@@ -353,4 +355,67 @@ cudaError_t launch_combine(const mkv_config& c, const DecodeWs& ws, const Split&
   return cudaPeekAtLastError();
 }
 
+// ---------------------------------------------------------------------------
+// FP16 decode without a caller workspace (mkv_decode_attention_noalloc).
+//
+// The split partials normally live in the caller's `ws`.  Here they live in a
+// fixed array compiled into this library, one copy per GPU that loads it, so a
+// caller that cannot allocate device memory can still decode.  Host code must
+// not hand the array's host-side name to a kernel: the device address is
+// looked up once per device with cudaGetSymbolAddress and cached.
+constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;   // 8 MiB per GPU
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace {
+std::mutex g_noalloc_mu;
+constexpr int kMaxDevices = 128;
+void* g_noalloc_addr[kMaxDevices] = {};
+
+// Device address of g_noalloc_scratch on the current device (looked up once).
+cudaError_t noalloc_scratch(void** addr) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (g_noalloc_addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    g_noalloc_addr[dev] = p;
+  }
+  *addr = g_noalloc_addr[dev];
+  return cudaSuccess;
+}
+}  // namespace
+
 }  // namespace mkv
+
+extern "C" mkv_status mkv_decode_attention_noalloc(const mkv_config* cfg, const void* q, const mkv_cache* cache,
+                                                   void* out, void* stream) {
+  using namespace mkv;
+  const mkv_status st0 = check_fp16_decode_args(cfg, cache, q, out);
+  if (st0 != MKV_OK) return st0;
+  const DecodeWs need = decode_ws(*cfg, cache->T_cap, nullptr);
+  if (need.bytes > kNoAllocScratchBytes) {
+    set_error("this call needs %zu bytes of scratch; the built-in array holds %zu (use mkv_decode_attention "
+              "with a workspace)", need.bytes, kNoAllocScratchBytes);
+    return MKV_ERR_WORKSPACE;
+  }
+  void* scratch = nullptr;
+  cudaError_t e = noalloc_scratch(&scratch);
+  if (e != cudaSuccess) {
+    set_error("cudaGetSymbolAddress of the built-in scratch: %s", cudaGetErrorString(e));
+    return MKV_ERR_CUDA;
+  }
+  const DecodeWs w = decode_ws(*cfg, cache->T_cap, scratch);
+  const Split sp = decode_split(*cfg, cache->T_cap);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  e = launch_decode_fp16_family(*cfg, q, *cache, nullptr, out, w, sp, st);
+  if (e == cudaSuccess) e = launch_combine(*cfg, w, sp, out, false, st);
+  if (e != cudaSuccess) {
+    set_error("decode launch: %s", cudaGetErrorString(e));
+    return MKV_ERR_CUDA;
+  }
+  return MKV_OK;
+}

@@ -227,6 +227,15 @@ size_t workspace_bytes(const mkv_config* c, int64_t T_cap) {
 
 }  // namespace
 
+mkv_status mkv::check_fp16_decode_args(const mkv_config* cfg, const mkv_cache* cache, const void* q,
+                                       const void* out) {
+  MKV_TRY(check_config(cfg));
+  MKV_REQUIRE(cfg->method == MKV_FP16, MKV_ERR_UNSUPPORTED, "this entry point serves FP16 caches only");
+  MKV_TRY(check_cache(cfg, cache));
+  MKV_REQUIRE(q && out, MKV_ERR_INVALID_ARG, "q/out NULL");
+  return MKV_OK;
+}
+
 extern "C" {
 
 const char* mkv_last_error(void) { return mkv::g_err; }

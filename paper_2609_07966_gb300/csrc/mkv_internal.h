@@ -90,6 +90,9 @@ cudaError_t launch_snap_keep(const mkv_config& c, const void* full_k, const void
 cudaError_t launch_rocket_select(const mkv_config& c, const void* q, const mkv_cache& cache,
                                  int32_t* page_idx, cudaStream_t st);
 
+// Host-side argument checks of an FP16 decode call (config, cache, q/out pointers).
+mkv_status check_fp16_decode_args(const mkv_config* cfg, const mkv_cache* cache, const void* q, const void* out);
+
 // Status word accessors (one per translation unit that can set a flag).
 cudaError_t take_status_kvquant(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_append(uint32_t* flags, cudaStream_t st);
