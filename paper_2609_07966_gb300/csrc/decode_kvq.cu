@@ -43,7 +43,7 @@ struct KvqArgs {
   int64_t rope_len;
   const int32_t* T_len;
   int64_t T_cap, k_out_cap;
-  int Hq, Hkv, G, n_v;
+  int Hq, Hkv, G, log2G, n_v;
   int chunks_per_split, n_split;
   float scale_log2;
   float* part_m;
@@ -68,14 +68,12 @@ struct KvqLayout {
   static constexpr int S_VP = S_VC + kChunk * SROW;          // [64] float2 (lo, scale)
   static constexpr int S_KE = S_VP + kChunk * 8;             // [KE_CAP] uint32 key outliers of the chunk
   static constexpr int S_VO = S_KE + KE_CAP * 4;             // [64][NVS] uint32 value outliers
-  static constexpr int S_RP = S_VO + kChunk * NVS * 4;       // [2][NP] float2 rotations of the bases
-  static constexpr int STAGE = S_RP + 2 * NP * 8;
+  static constexpr int STAGE = S_VO + kChunk * NVS * 4;
   // byte offsets
   static constexpr int DTAB = 0;                             // [NP][32] float2
   static constexpr int KDQ = DTAB + NP * 32 * 8;             // [D][K] float
-  static constexpr int VTB = KDQ + D * K * 4;                // [D][K] half
-  static constexpr int QRAW = VTB + D * K * 2;               // [8][D] half (the group's queries)
-  static constexpr int QHI = QRAW + 8 * D * 2;               // [2 bases][8][NP] half2 (rotated query, hi)
+  static constexpr int VTB = KDQ + D * K * 4;                // [D][K] float
+  static constexpr int QHI = VTB + D * K * 4;                // [2 bases][8][NP] half2 (rotated query, hi)
   static constexpr int QLO = QHI + 2 * 8 * NP * 4;           // [2][8][NP] half2 (lo)
   static constexpr int KOFF = QLO + 2 * 8 * NP * 4;          // [3 chunks][68] int32 key-outlier CSR offsets
   static constexpr int STG = KOFF + 3 * 68 * 4;              // [2 stages][STAGE]
@@ -116,6 +114,14 @@ __device__ __forceinline__ void split_hi_lo(float a, float b, uint32_t& hi, uint
   lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
+// D(16x8 f32) += A(16x8 f16, row) * B(8x8 f16, col)
+__device__ __forceinline__ void mma1688(float c[4], uint32_t a0, uint32_t a1, uint32_t b0) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5}, {%6}, {%0,%1,%2,%3};\n"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(b0));
+}
+
 // byte offset of (row, 16B chunk) in a swizzled fp16 tile of D columns
 template <int D>
 __device__ __forceinline__ int tile_off(int row, int ch) {
@@ -127,16 +133,18 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
   using Lay = KvqLayout<D, BITS>;
   constexpr int NP = Lay::NP, K = Lay::K, ROWB = Lay::ROWB, SROW = Lay::SROW;
   constexpr int KC = D / 16;
-  constexpr int HALF_PAIRS = NP / 2;                  // pairs per thread (half a row)
-  constexpr int HALF_WORDS = HALF_PAIRS * 2 * BITS / 32;
+  // Phase 1 splits each row's pairs into GROUPS groups of whole 32-bit words.
+  constexpr int GROUPS = ((NP / 4) * 2 * BITS) % 32 == 0 ? 4 : 2;
+  constexpr int QP = NP / GROUPS;                         // pairs per group
+  constexpr int NWQ = QP * 2 * BITS / 32;                 // code words per group
+  constexpr bool SPLIT_KV = GROUPS == 2;                  // then a thread does K or V, not both
   extern __shared__ __align__(128) uint8_t smem[];
   float2* dtab = reinterpret_cast<float2*>(smem + Lay::DTAB);
   float* kdq = reinterpret_cast<float*>(smem + Lay::KDQ);
-  __half* vtb = reinterpret_cast<__half*>(smem + Lay::VTB);
+  float* vtb = reinterpret_cast<float*>(smem + Lay::VTB);
   uint32_t* qhi = reinterpret_cast<uint32_t*>(smem + Lay::QHI);
   uint32_t* qlo = reinterpret_cast<uint32_t*>(smem + Lay::QLO);
   uint8_t* stg = smem + Lay::STG;
-  __half* qraw = reinterpret_cast<__half*>(smem + Lay::QRAW);
   int32_t* kring = reinterpret_cast<int32_t*>(smem + Lay::KOFF);
   uint8_t* khi_t = smem + Lay::KHI;
   uint8_t* klo_t = smem + Lay::KLO;
@@ -179,11 +187,6 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
       const int64_t s = c0 + tid;
       const bool ok = s < n_len;
       cp_async8(dst + Lay::S_VP + tid * 8, a.v_params + bh * a.T_cap + (ok ? s : 0), ok ? 8 : 0);
-    } else if (tid < kChunk + NP) {              // rotations of the two 32-token bases
-      const int e = tid - kChunk;                // 16-byte pieces: 2 float2 each
-      const int base = e / (NP / 2), piece = e % (NP / 2);
-      const int64_t tb = min(c0 + 32 * base, a.rope_len - 1);
-      cp_async16(dst + Lay::S_RP + (base * NP + 2 * piece) * 8, a.rope + tb * NP + 2 * piece, 16);
     }
     if (stage_vout && a.n_v > 0) {
       for (int e = tid; e < kChunk * a.n_v; e += kThr) {
@@ -223,23 +226,43 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     cp_async_commit();
   }
   // CTA-resident tables: rotations by delta in [0, 32), dequant tables of this kv-head
-  for (int e = tid; e < NP * 32; e += kThr) {
-    const int i = e / 32, d = e % 32;
-    dtab[e] = a.rope[(int64_t)d * NP + i];
+  for (int e = tid; e < NP * 32; e += kThr) {      // coalesced read of rows 0..31, transposed
+    const int d = e / NP, i = e % NP;
+    dtab[i * 32 + d] = a.rope[(int64_t)d * NP + i];
   }
   for (int e = tid; e < D * K; e += kThr) {
     kdq[e] = a.k_dq[(int64_t)kvh * D * K + e];
-    vtb[e] = __ushort_as_half(a.v_tbl[(int64_t)kvh * D * K + e]);
+    vtb[e] = __half2float(__ushort_as_half(a.v_tbl[(int64_t)kvh * D * K + e]));
   }
-  for (int e = tid; e < a.G * D; e += kThr) {
-    qraw[e] = a.q[((int64_t)b * a.Hq + (int64_t)kvh * a.G) * D + e];
+  // This thread's fixed share of the rotated-query table: element e = (base, head, pair) for
+  // e = tid + k*kThr.  Its raw query pair is loaded once; the rotation of its base is
+  // prefetched one chunk ahead.
+  constexpr int kQE = 2 * 8 * NP / kThr;                   // at most G = 8
+  float qx[kQE], qy[kQE];
+  float2 qcs[kQE];
+  const int nqe = 2 * a.G * NP;
+#pragma unroll
+  for (int k = 0; k < kQE; ++k) {
+    const int e = tid + k * kThr;
+    qx[k] = qy[k] = 0.f;
+    qcs[k] = make_float2(1.f, 0.f);
+    if (e < nqe) {
+      const int t = e / NP, i = e % NP;
+      const int gg = t & (a.G - 1), base = t >> a.log2G;
+      const __half* qr = a.q + ((int64_t)b * a.Hq + (int64_t)kvh * a.G + gg) * D;
+      qx[k] = __half2float(qr[i]);
+      qy[k] = __half2float(qr[i + NP]);
+      if (nchunks > 0) qcs[k] = a.rope[min(v_begin + 32 * base, a.rope_len - 1) * NP + i];
+    }
   }
 
-  float o[D / 16][2];
+  float o[D / 8][2];
 #pragma unroll
-  for (int i = 0; i < D / 16; ++i) o[i][0] = o[i][1] = 0.f;
+  for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = 0.f;
   float m_run = -INFINITY, l_part = 0.f;
-  const int slab = warp & 3, dhalf = warp >> 2;
+  const int t4 = warp & 3;                 // phase 1: pair group (or K/V role) of this warp
+  const int tok = (warp >> 2) * 32 + lane; // phase 1: this thread's token in the chunk
+  const int dl = tok & 31;                 // its offset from its 32-token base
 
   for (int c = 0; c < nchunks; ++c) {
     cp_async_wait<0>();
@@ -258,78 +281,63 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     const int kbase = koff[0];
     const int kstaged = min((int)min((int64_t)koff[kChunk], a.k_out_cap) - kbase, Lay::KE_CAP);
     const uint32_t* vouts = reinterpret_cast<const uint32_t*>(st + Lay::S_VO);
-    const float2* rbase = reinterpret_cast<const float2*>(st + Lay::S_RP);
 
-    // ---- query rotated back by each 32-token base tb: R(tb)^T q as hi/lo fp16 pairs,
-    //      qhi[base][g][i] = (q'_i, q'_{i+NP}), base 0 -> t0, base 1 -> t0 + 32
-    for (int e = tid; e < 2 * a.G * NP; e += kThr) {
-      const int base = e / (a.G * NP), gg = (e / NP) % a.G, i = e % NP;
-      const float x = __half2float(qraw[gg * D + i]), y = __half2float(qraw[gg * D + i + NP]);
-      const float2 cs = rbase[base * NP + i];
-      split_hi_lo(x * cs.x + y * cs.y, y * cs.x - x * cs.y, qhi[(base * 8 + gg) * NP + i],
-                  qlo[(base * 8 + gg) * NP + i]);
+    // ---- query rotated back by each 32-token base tb: R(tb)^T q as hi/lo fp16 pairs, stored in
+    //      the order the mma fragments read: pair i = kc*8 + 4*hf + r at word kc*8 + 2*r + hf
+#pragma unroll
+    for (int k = 0; k < kQE; ++k) {
+      const int e = tid + k * kThr;
+      if (e < nqe) {
+        const int t = e / NP, i = e % NP;
+        const int gg = t & (a.G - 1), base = t >> a.log2G;
+        const float x = qx[k], y = qy[k];
+        const float2 cs = qcs[k];
+        const int wpos = (i / 8) * 8 + (i % 4) * 2 + ((i % 8) / 4);
+        split_hi_lo(x * cs.x + y * cs.y, y * cs.x - x * cs.y, qhi[(base * 8 + gg) * NP + wpos],
+                    qlo[(base * 8 + gg) * NP + wpos]);
+        if (c + 1 < nchunks) qcs[k] = a.rope[min(t0 + kChunk + 32 * base, a.rope_len - 1) * NP + i];
+      }
     }
 
-    // ---- phase 1: dequantize the chunk into fp16 tiles
+    // ---- phase 1: dequantize one pair group of the thread's token (keys and/or values)
     {
-      const bool is_v = warp >= 4;
-      const int wl = warp & 3;
-      const int tok = (wl & 1) * 32 + lane;           // row of the chunk
-      const int hp = wl >> 1;                         // which half of the pairs
       const int64_t slot = t0 + tok;
       const bool valid = slot < n_len;
-      const uint8_t* rowfull = st + (is_v ? Lay::S_VC : Lay::S_KC) + tok * SROW;
-      const uint8_t* row = rowfull + hp * (HALF_WORDS * 4);
-      uint32_t w[HALF_WORDS];
-      if constexpr (HALF_WORDS % 4 == 0) {
+      const bool do_k = SPLIT_KV ? (t4 < 2) : true;
+      const bool do_v = SPLIT_KV ? (t4 >= 2) : true;
+      const int grp = SPLIT_KV ? (t4 & 1) : t4;
+      if (do_k) {
+        const uint8_t* rowfull = st + Lay::S_KC + tok * SROW;
+        uint32_t w[NWQ];
 #pragma unroll
-        for (int k = 0; k < HALF_WORDS; k += 4) {
-          const uint4 u = *reinterpret_cast<const uint4*>(row + 4 * k);
-          w[k] = u.x;
-          w[k + 1] = u.y;
-          w[k + 2] = u.z;
-          w[k + 3] = u.w;
-        }
-      } else if constexpr (HALF_WORDS % 2 == 0) {
+        for (int k = 0; k < NWQ; ++k) w[k] = reinterpret_cast<const uint32_t*>(rowfull)[grp * NWQ + k];
 #pragma unroll
-        for (int k = 0; k < HALF_WORDS; k += 2) {
-          const uint2 u = *reinterpret_cast<const uint2*>(row + 4 * k);
-          w[k] = u.x;
-          w[k + 1] = u.y;
-        }
-      } else {
-#pragma unroll
-        for (int k = 0; k < HALF_WORDS; ++k) w[k] = *reinterpret_cast<const uint32_t*>(row + 4 * k);
-      }
-      const int dl = tok & 31;                        // offset from the token's 32-token base
-      uint8_t* tile = is_v ? v_t : khi_t;
-      if (!is_v) {
-#pragma unroll
-        for (int jj = 0; jj < HALF_PAIRS; jj += 4) {
+        for (int jj = 0; jj < QP; jj += 4) {
           uint32_t ph[4], pl[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const int j = jj + u, i = hp * HALF_PAIRS + j;
+            const int j = jj + u, i = grp * QP + j;
             int clo, chi;
-            pair_codes<BITS, HALF_WORDS>(w, j, clo, chi);
-            const float x = valid ? kdq[i * K + clo] : 0.f;
-            const float y = valid ? kdq[(i + NP) * K + chi] : 0.f;
+            pair_codes<BITS, NWQ>(w, j, clo, chi);
+            // rows past the cache end were zero-filled: finite keys, masked in phase 2
+            const float x = kdq[i * K + clo];
+            const float y = kdq[(i + NP) * K + chi];
             const float2 cs = dtab[i * 32 + dl];
             split_hi_lo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph[u], pl[u]);
           }
-          const int ch = (hp * HALF_PAIRS + jj) / 4;
+          const int ch = (grp * QP + jj) / 4;
           *reinterpret_cast<uint4*>(khi_t + tile_off<D>(tok, ch)) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
           *reinterpret_cast<uint4*>(klo_t + tile_off<D>(tok, ch)) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
         }
-        // key outliers of this token in this half: recompute their pair exactly
+        // key outliers of this token in this group: recompute their pair exactly
         if (valid) {
           const int e0 = koff[tok], e1 = (int)min((int64_t)koff[tok + 1], a.k_out_cap);
           const uint32_t* gents = a.k_out + bh * a.k_out_cap;
           auto ent = [&](int e) { return e - kbase < kstaged ? kents[e - kbase] : gents[e]; };
           for (int e = e0; e < e1; ++e) {
-            const int ch = (int)(ent(e) >> 16);
-            const int i = ch % NP;
-            if (i / HALF_PAIRS != hp) continue;
+            const int chn = (int)(ent(e) >> 16);
+            const int i = chn % NP;
+            if (i / QP != grp) continue;
             int clo, chi;
             pair_codes_row<BITS>(rowfull, i, clo, chi);
             float x = kdq[i * K + clo], y = kdq[(i + NP) * K + chi];
@@ -347,32 +355,38 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
             *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
           }
         }
-      } else {
+      }
+      if (do_v) {
+        const uint8_t* rowfull = st + Lay::S_VC + tok * SROW;
+        uint32_t w[NWQ];
+#pragma unroll
+        for (int k = 0; k < NWQ; ++k) w[k] = reinterpret_cast<const uint32_t*>(rowfull)[grp * NWQ + k];
         const float2 lp = vpar[tok];
 #pragma unroll
-        for (int jj = 0; jj < HALF_PAIRS; jj += 4) {
+        for (int jj = 0; jj < QP; jj += 4) {
           uint32_t pv[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const int j = jj + u, i = hp * HALF_PAIRS + j;
+            const int j = jj + u, i = grp * QP + j;
             int clo, chi;
-            pair_codes<BITS, HALF_WORDS>(w, j, clo, chi);
-            const float x = lp.x + lp.y * __half2float(vtb[i * K + clo]);
-            const float y = lp.x + lp.y * __half2float(vtb[(i + NP) * K + chi]);
-            pv[u] = valid ? pack_half2(x, y) : 0u;
+            pair_codes<BITS, NWQ>(w, j, clo, chi);
+            // rows past the cache end have lo = scale = 0 (zero-filled): value 0
+            const float x = fmaf(lp.y, vtb[i * K + clo], lp.x);
+            const float y = fmaf(lp.y, vtb[(i + NP) * K + chi], lp.x);
+            pv[u] = pack_half2(x, y);
           }
-          const int ch = (hp * HALF_PAIRS + jj) / 4;
-          *reinterpret_cast<uint4*>(tile + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
+          const int ch = (grp * QP + jj) / 4;
+          *reinterpret_cast<uint4*>(v_t + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
         }
         if (valid) {
           const uint32_t* ents = stage_vout ? vouts + tok * Lay::NVS : a.v_out + (bh * a.T_cap + slot) * a.n_v;
           for (int e = 0; e < a.n_v; ++e) {
             const uint32_t ev = ents[e];
-            const int ch = (int)(ev >> 16);
-            const int i = ch % NP;
-            if (i / HALF_PAIRS != hp) continue;
-            const int col = ch < NP ? 2 * ch : 2 * (ch - NP) + 1;
-            *reinterpret_cast<uint16_t*>(tile + tile_off<D>(tok, col / 8) + (col % 8) * 2) =
+            const int chn = (int)(ev >> 16);
+            const int i = chn % NP;
+            if (i / QP != grp) continue;
+            const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
+            *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(tok, col / 8) + (col % 8) * 2) =
                 (uint16_t)(ev & 0xffffu);
           }
         }
@@ -380,103 +394,84 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     }
     __syncthreads();
 
-    // ---- phase 2: warp (slab, dhalf) -> tokens 16*slab.., output dims half dhalf
+    // ---- phase 2: warp w owns tokens 8w..8w+7 of the chunk and every output dim
     {
       const bool real = g < a.G;
-      const int t0w = slab * 16;
-      const uint32_t* qh = qhi + (slab >> 1) * 8 * NP;      // slabs 0-1: base t0, 2-3: t0 + 32
-      const uint32_t* ql = qlo + (slab >> 1) * 8 * NP;
-      float sc[2][4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) sc[0][i] = sc[1][i] = 0.f;
-      const int mi = lane >> 3, rowi = lane & 7;
-      const int tokk = t0w + (mi >> 1) * 8 + rowi;
+      const int base = warp >> 2;                            // tokens 0-31: base t0, 32-63: t0 + 32
+      const uint2* qh2 = reinterpret_cast<const uint2*>(qhi + (base * 8 + (real ? g : 0)) * NP);
+      const uint2* ql2 = reinterpret_cast<const uint2*>(qlo + (base * 8 + (real ? g : 0)) * NP);
+      float sc[4] = {0.f, 0.f, 0.f, 0.f};
+      // ldmatrix x4: lanes 0-15 address the hi tile, 16-31 the lo tile (dims kc*16 + 0..7 / 8..15)
+      const int mtx = lane >> 3, rowi = lane & 7;
+      const int tokk = warp * 8 + rowi;
+      const uint8_t* kt = (mtx < 2) ? khi_t : klo_t;
 #pragma unroll
       for (int kc = 0; kc < KC; ++kc) {
-        const uint32_t ah0 = real ? qh[g * NP + kc * 8 + r] : 0u;
-        const uint32_t ah2 = real ? qh[g * NP + kc * 8 + r + 4] : 0u;
-        const uint32_t al0 = real ? ql[g * NP + kc * 8 + r] : 0u;
-        const uint32_t al2 = real ? ql[g * NP + kc * 8 + r + 4] : 0u;
-        uint32_t bh4[4], bl4[4];
-        const int ch = kc * 2 + (mi & 1);
-        ldsm_x4(bh4, khi_t + tile_off<D>(tokk, ch));
-        ldsm_x4(bl4, klo_t + tile_off<D>(tokk, ch));
-        mma16816(sc[0], ah0, 0u, ah2, 0u, bh4[0], bh4[1]);
-        mma16816(sc[1], ah0, 0u, ah2, 0u, bh4[2], bh4[3]);
-        mma16816(sc[0], ah0, 0u, ah2, 0u, bl4[0], bl4[1]);
-        mma16816(sc[1], ah0, 0u, ah2, 0u, bl4[2], bl4[3]);
-        mma16816(sc[0], al0, 0u, al2, 0u, bh4[0], bh4[1]);
-        mma16816(sc[1], al0, 0u, al2, 0u, bh4[2], bh4[3]);
+        const uint2 ah = real ? qh2[kc * 4 + r] : make_uint2(0u, 0u);
+        const uint2 al = real ? ql2[kc * 4 + r] : make_uint2(0u, 0u);
+        uint32_t bk[4];
+        ldsm_x4(bk, kt + tile_off<D>(tokk, kc * 2 + (mtx & 1)));
+        mma16816(sc, ah.x, 0u, ah.y, 0u, bk[0], bk[1]);
+        mma16816(sc, ah.x, 0u, ah.y, 0u, bk[2], bk[3]);
+        mma16816(sc, al.x, 0u, al.y, 0u, bk[0], bk[1]);
       }
-      const int tk[4] = {t0w + 2 * r, t0w + 2 * r + 1, t0w + 8 + 2 * r, t0w + 9 + 2 * r};
-      float x[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
-      float mx = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        x[i] = (t0 + tk[i] < n_len) ? x[i] * a.scale_log2 : -INFINITY;
-        mx = fmaxf(mx, x[i]);
-      }
+      const int tk0 = warp * 8 + 2 * r;
+      float x0 = (t0 + tk0 < n_len) ? sc[0] * a.scale_log2 : -INFINITY;
+      float x1 = (t0 + tk0 + 1 < n_len) ? sc[1] * a.scale_log2 : -INFINITY;
+      float mx = fmaxf(x0, x1);
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
       const float m_new = fmaxf(m_run, mx);
-      float p[4];
-      float alpha = 1.f;
-      if (m_new == -INFINITY) {
-        p[0] = p[1] = p[2] = p[3] = 0.f;
-      } else {
+      float p0 = 0.f, p1 = 0.f, alpha = 1.f;
+      if (m_new != -INFINITY) {
         alpha = exp2f(m_run - m_new);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) p[i] = exp2f(x[i] - m_new);
+        p0 = exp2f(x0 - m_new);
+        p1 = exp2f(x1 - m_new);
       }
-      l_part = l_part * alpha + (p[0] + p[1]) + (p[2] + p[3]);
+      l_part = l_part * alpha + p0 + p1;
       m_run = m_new;
       if (__any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll
-        for (int i = 0; i < D / 16; ++i) {
+        for (int i = 0; i < D / 8; ++i) {
           o[i][0] *= alpha;
           o[i][1] *= alpha;
         }
       }
-      const uint32_t pa0 = pack_half2(p[0], p[1]);
-      const uint32_t pa2 = pack_half2(p[2], p[3]);
-      const int tokv = t0w + (mi & 1) * 8 + rowi;
+      const uint32_t pa = pack_half2(p0, p1);
+      const int tokv = warp * 8 + rowi;
 #pragma unroll
-      for (int j = 0; j < D / 32; ++j) {
+      for (int dq = 0; dq < D / 32; ++dq) {                  // four 8-dim tiles per ldmatrix
         uint32_t bv[4];
-        const int jj = dhalf * (D / 32) + j;
-        const int ch = 2 * jj + (mi >> 1);
-        ldsm_x4_t(bv, v_t + tile_off<D>(tokv, ch));
-        float d0[4] = {o[2 * j][0], o[2 * j][1], 0.f, 0.f};
-        float d1[4] = {o[2 * j + 1][0], o[2 * j + 1][1], 0.f, 0.f};
-        mma16816(d0, pa0, 0u, pa2, 0u, bv[0], bv[1]);
-        mma16816(d1, pa0, 0u, pa2, 0u, bv[2], bv[3]);
-        o[2 * j][0] = d0[0];
-        o[2 * j][1] = d0[1];
-        o[2 * j + 1][0] = d1[0];
-        o[2 * j + 1][1] = d1[1];
+        ldsm_x4_t(bv, v_t + tile_off<D>(tokv, dq * 4 + mtx));
+#pragma unroll
+        for (int m = 0; m < 4; ++m) {
+          float d[4] = {o[dq * 4 + m][0], o[dq * 4 + m][1], 0.f, 0.f};
+          mma1688(d, pa, 0u, bv[m]);
+          o[dq * 4 + m][0] = d[0];
+          o[dq * 4 + m][1] = d[1];
+        }
       }
     }
   }
   cp_async_wait<0>();
   __syncthreads();
 
-  // ---- merge the four slabs; warps of dhalf 0 and 1 hold the two halves of the dims
+  // ---- merge the eight warps' (m, l, o) per query row; o is in the permuted column order
   l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
   l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
-  float* wm = reinterpret_cast<float*>(smem + Lay::STG);   // [4][8]
-  float* wl = wm + 32;                                      // [4][8]
-  float* wo = wl + 32;                                      // [4][8][D]  (natural channel order)
+  float* wm = reinterpret_cast<float*>(khi_t);              // [8 warps][8 rows]
+  float* wl = wm + 64;                                       // [8][8]
+  float* wo = wl + 64;                                       // [8][8][D]  natural channel order
   if (g < a.G) {
-    if (r == 0 && dhalf == 0) {
-      wm[slab * 8 + g] = m_run;
-      wl[slab * 8 + g] = l_part;
+    if (r == 0) {
+      wm[warp * 8 + g] = m_run;
+      wl[warp * 8 + g] = l_part;
     }
 #pragma unroll
-    for (int j = 0; j < D / 16; ++j) {
-      const int dt = dhalf * (D / 16) + j;                  // 8-column tile of the permuted order
-      const int ch = dt * 4 + r;                            // column dt*8 + 2r -> channel dt*4 + r
-      wo[(slab * 8 + g) * D + ch] = o[j][0];
-      wo[(slab * 8 + g) * D + ch + NP] = o[j][1];
+    for (int dt = 0; dt < D / 8; ++dt) {
+      const int chn = dt * 4 + r;                            // column dt*8 + 2r -> channel dt*4 + r
+      wo[(warp * 8 + g) * D + chn] = o[dt][0];
+      wo[(warp * 8 + g) * D + chn + NP] = o[dt][1];
     }
   }
   __syncthreads();
@@ -484,11 +479,11 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     const int row = e / D, d = e % D;
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < 4; ++w) M = fmaxf(M, wm[w * 8 + row]);
+    for (int w = 0; w < 8; ++w) M = fmaxf(M, wm[w * 8 + row]);
     float L = 0.f, O = 0.f;
     if (M != -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
+      for (int w = 0; w < 8; ++w) {
         const float f = exp2f(wm[w * 8 + row] - M);
         L += wl[w * 8 + row] * f;
         O += wo[(w * 8 + row) * D + d] * f;
@@ -539,6 +534,7 @@ cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_
   a.Hq = c.Hq;
   a.Hkv = c.Hkv;
   a.G = c.Hq / c.Hkv;
+  a.log2G = a.G == 8 ? 3 : (a.G == 4 ? 2 : (a.G == 2 ? 1 : 0));
   a.n_v = std::min(c.D, (int)ceil((double)c.outlier_frac * c.D));
   a.chunks_per_split = sp.chunks_per_split;
   a.n_split = sp.n_split;
