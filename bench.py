@@ -52,7 +52,7 @@ METRIC = "compressed-KV decode attn tokens/s and HBM GB/s (fraction of ~8 TB/s) 
 # --------------------------------------------------------------------------- clocks
 
 class ClockSampler:
-    """nvidia-smi samples (200 ms) during the timed region."""
+    """nvidia-smi samples (50 ms) around the timed region."""
 
     Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
          "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
@@ -66,7 +66,7 @@ class ClockSampler:
     def start(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
@@ -105,22 +105,34 @@ class Runner:
         self.torch, self.mkv, self.name, self.w, self.dev = torch, mkv, name, w, dev
         self.method = METHOD_OF[name]
         B, Hq, Hkv, D = w.B, w.Hq, w.Hkv, w.D
-        self.T_cap = w.T + extra_steps + 64
         mk = {"fp16": mkv.MKV_FP16, "kvquant": mkv.MKV_KVQUANT, "h2o": mkv.MKV_H2O, "rocket": mkv.MKV_ROCKET}
         kw = {}
         if self.method == "kvquant":
             kw = dict(bits=w.bits, quant_mode=mkv.MKV_QUANT_NUQ if w.quant_mode == "nuq" else mkv.MKV_QUANT_UNIFORM,
                       outlier_frac=w.outlier_frac, rope_theta=w.theta)
+        elif self.method == "h2o":
+            kw = dict(h2o_heavy=w.h2o_heavy, h2o_recent=w.h2o_recent)
+        elif self.method == "rocket":
+            kw = dict(snap_window=w.snap_window, snap_pool=w.snap_pool, snap_keep=w.snap_keep, page_size=w.page,
+                      topk_pages=w.topk_pages, topq_dims=w.topq_dims)
         self.cfg = mkv.config(mk[self.method], B, Hq, Hkv, D, **kw)
+        if self.method == "h2o":
+            self.T_cap = w.h2o_heavy + w.h2o_recent + 1
+        elif self.method == "rocket":
+            self.T_cap = (min(w.T, w.snap_keep) + extra_steps + 15) // 16 * 16
+        else:
+            self.T_cap = w.T + extra_steps + 64
         self.layers = []
-        self.q, self.kn, self.vn, self.out = [], [], [], []
-        ws_cap = self.T_cap
-        self.ws, self.nws = caches.workspace(self.cfg, ws_cap, device=dev)
+        self.q, self.kn, self.vn, self.out, self.pidx = [], [], [], [], []
+        # prefill-side calls need workspace for the whole prompt
+        self.ws, self.nws = caches.workspace(self.cfg, max(self.T_cap, w.T), device=dev)
         if self.method == "kvquant":
             self.rope = torch.empty((self.T_cap, D // 2, 2), dtype=torch.float32, device=dev)
             mkv.mkv_rope_table(D, w.theta, self.T_cap, self.rope.data_ptr())
+        t_setup = time.perf_counter()
         for l in range(w.L):
-            x = synth.device_layer_inputs(w, seed, l, device=dev, n_tokens=w.T + 1)
+            x = synth.device_layer_inputs(w, seed, l, device=dev, n_tokens=w.T + 1,
+                                          with_prompt_queries=self.method in ("h2o", "rocket"))
             cache = caches.alloc_cache(self.cfg, self.T_cap, device=dev)
             qp = None
             if self.method == "fp16":
@@ -140,6 +152,20 @@ class Runner:
                 vp = x["v"][:, :, :w.T].contiguous()
                 mkv.mkv_quantize_kv(self.cfg, qp.c, kp.data_ptr(), vp.data_ptr(), w.T, cache.c)
                 del kp, vp
+            elif self.method == "h2o":
+                kp = x["k"][:, :, :w.T].contiguous()
+                vp = x["v"][:, :, :w.T].contiguous()
+                mkv.mkv_h2o_prefill(self.cfg, x["q_prompt"].data_ptr(), kp.data_ptr(), vp.data_ptr(), w.T, cache.c,
+                                    self.ws.data_ptr(), self.nws)
+                del kp, vp
+            else:
+                kp = x["k"][:, :, :w.T].contiguous()
+                vp = x["v"][:, :, :w.T].contiguous()
+                qw = x["q_prompt"][:, :, w.T - w.snap_window:].contiguous()
+                mkv.mkv_snap_compress(self.cfg, qw.data_ptr(), kp.data_ptr(), vp.data_ptr(), w.T, cache.c, 0,
+                                      self.ws.data_ptr(), self.nws)
+                del kp, vp, qw
+                self.pidx.append(torch.zeros((B, Hkv, w.topk_pages), dtype=torch.int32, device=dev))
             self.layers.append((cache, qp))
             self.q.append(x["q"][0].contiguous())
             self.kn.append(x["k"][:, :, w.T].contiguous())
@@ -147,25 +173,41 @@ class Runner:
             self.out.append(torch.empty((B, Hq, D), dtype=torch.float16, device=dev))
             del x
         torch.cuda.synchronize()
+        self.setup_s = time.perf_counter() - t_setup
         flags = mkv.mkv_get_status()
         assert flags == 0, f"device status flags {flags:#x} after setup"
         self.graph = None
 
-    def layer_step(self, l, q=None, kn=None, vn=None, out=None):
+    def append(self, l, kn=None, vn=None):
+        mkv = self.mkv
+        cache, qp = self.layers[l]
+        kn = self.kn[l] if kn is None else kn
+        vn = self.vn[l] if vn is None else vn
+        if self.method == "kvquant":
+            mkv.mkv_quantize_kv(self.cfg, qp.c, kn.data_ptr(), vn.data_ptr(), 1, cache.c)
+        else:
+            mkv.mkv_append_kv(self.cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
+
+    def decode(self, l, q=None, out=None):
         mkv = self.mkv
         cache, qp = self.layers[l]
         q = self.q[l] if q is None else q
-        kn = self.kn[l] if kn is None else kn
-        vn = self.vn[l] if vn is None else vn
         out = self.out[l] if out is None else out
-        if self.method == "kvquant":
-            mkv.mkv_quantize_kv(self.cfg, qp.c, kn.data_ptr(), vn.data_ptr(), 1, cache.c)
-            mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, qp.c, 0, out.data_ptr(), self.ws.data_ptr(),
-                                     self.nws)
-        else:
-            mkv.mkv_append_kv(self.cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
-            mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, None, 0, out.data_ptr(), self.ws.data_ptr(),
-                                     self.nws)
+        pidx = self.pidx[l].data_ptr() if self.method == "rocket" else 0
+        mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, qp.c if qp else None, pidx, out.data_ptr(),
+                                 self.ws.data_ptr(), self.nws)
+
+    def layer_step(self, l, q=None, kn=None, vn=None, out=None):
+        """One layer of one decode step: append the token, (select pages,) attend, (update scores)."""
+        mkv = self.mkv
+        cache, _ = self.layers[l]
+        self.append(l, kn, vn)
+        if self.method == "rocket":
+            mkv.mkv_rocket_select(self.cfg, (self.q[l] if q is None else q).data_ptr(), cache.c,
+                                  self.pidx[l].data_ptr())
+        self.decode(l, q, out)
+        if self.method == "h2o":
+            mkv.mkv_h2o_update(self.cfg, cache.c, self.ws.data_ptr(), self.nws)
 
     def step(self):
         for l in range(self.w.L):
@@ -191,15 +233,17 @@ class Runner:
             self.step()
 
     def launches_per_step(self):
-        # per layer: append (KVQuant: quantize + length advance) + decode + combine
-        return (4 if self.method == "kvquant" else 3) * self.w.L
+        # per layer: append (KVQuant: quantize + length advance), (page select), decode + combine,
+        # (score update)
+        per = {"fp16": 3, "kvquant": 4, "h2o": 4, "rocket": 4}[self.method]
+        return per * self.w.L
 
     def decode_bytes(self):
-        """Algorithmic bytes one decode launch reads for one layer at the current lengths."""
+        """Algorithmic bytes one decode launch (decode + combine) reads for one layer now."""
         w = self.w
         cache, _ = self.layers[0]
-        T = int(cache.t["T_len"][0])
         units = w.B * w.Hkv
+        T = int(cache.t["T_len"][0])
         if self.method == "fp16":
             return units * T * w.D * 2 * 2, T
         if self.method == "kvquant":
@@ -207,7 +251,13 @@ class Runner:
             per_tok = 2 * (w.D * w.bits // 8) + 8 + 4 * nv + 4
             n_kout = int(cache.t["k_out_off"][:, :, T].sum())
             return units * T * per_tok + 4 * n_kout, T
-        raise NotImplementedError(self.method)
+        if self.method == "h2o":
+            slots = self.T_cap
+            # K and V rows, the slot's position (mask) and the G logits written for the update
+            return units * slots * (w.D * 2 * 2 + 4 + 4 * w.G), int(cache.t["pos"][0, 0].ge(0).sum())
+        n = T
+        tail = n - 16 * ((n - 1) // 16)
+        return units * ((w.topk_pages * 16 + tail) * w.D * 2 * 2 + 4 * w.topk_pages), n
 
 
 def time_steps(runner, steps, warmup):
@@ -233,16 +283,16 @@ def time_decode_launches(runner, steps):
     evs = []
     for _ in range(steps):
         for l in range(runner.w.L):
-            cache, qp = runner.layers[l]
-            if runner.method == "kvquant":
-                mkv.mkv_quantize_kv(runner.cfg, qp.c, runner.kn[l].data_ptr(), runner.vn[l].data_ptr(), 1, cache.c)
-            else:
-                mkv.mkv_append_kv(runner.cfg, runner.kn[l].data_ptr(), runner.vn[l].data_ptr(), cache.c)
+            cache, _ = runner.layers[l]
+            runner.append(l)
+            if runner.method == "rocket":
+                mkv.mkv_rocket_select(runner.cfg, runner.q[l].data_ptr(), cache.c, runner.pidx[l].data_ptr())
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record(st)
-            mkv.mkv_decode_attention(runner.cfg, runner.q[l].data_ptr(), cache.c, qp.c if qp else None, 0,
-                                     runner.out[l].data_ptr(), runner.ws.data_ptr(), runner.nws)
+            runner.decode(l)
             b.record(st)
+            if runner.method == "h2o":
+                mkv.mkv_h2o_update(runner.cfg, cache.c, runner.ws.data_ptr(), runner.nws)
             evs.append((a, b))
     torch.cuda.synchronize()
     return statistics.mean(a.elapsed_time(b) for a, b in evs)
@@ -315,6 +365,19 @@ def oracle_tokens_per_s(name: str, w, budget_s: float, seed: int = 0):
                 (qh.k_codes, qh.k_mask, qh.k_raw, qh.v_codes, qh.v_mask, qh.v_lo, qh.v_scale, qh.v_raw),
                 (new.k_codes, new.k_mask, new.k_raw, new.v_codes, new.v_mask, new.v_lo, new.v_scale, new.v_raw))])
             kvquant.decode_head(q, full, p, w.theta)
+    elif method == "h2o":
+        from oracle import h2o
+        n = w.h2o_heavy + w.h2o_recent
+        st = h2o.H2OHead(np.arange(n), k[:n], v[:n], np.abs(rng.standard_normal(n)))
+
+        def unit():
+            h2o.decode_step(st, q, k[n], v[n], T, w.h2o_heavy, w.h2o_recent)
+    elif method == "rocket":
+        from oracle import rocket
+        n = min(T, w.snap_keep) + 1
+
+        def unit():
+            rocket.decode(q, k[:n], v[:n], n, w.page, w.topk_pages, w.topq_dims)
     else:
         def unit():
             attention.attend(q, k, v)
@@ -345,6 +408,8 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--layers", type=int, default=None,
                     help="profiling only: fewer layers than the workload (the line is then not a bench number)")
+    ap.add_argument("--per-config", default="fp16,kvquant3,kvquant2,h2o20,rocket1024",
+                    help="other workloads measured after the headline one (comma list, '' for none)")
     ap.add_argument("--profile", action="store_true",
                     help="profiling only: run warmup + steps and exit (for ncu), no JSON line")
     args = ap.parse_args()
@@ -401,8 +466,10 @@ def main():
     torch.cuda.synchronize()
     clocks = ClockSampler(torch.cuda.current_device())
     clocks.start()
+    time.sleep(0.3)                              # first samples before the warm-up begins
     ms = time_steps(runner, args.steps, args.warmup)
     clk = clocks.stop()
+    clk["window"] = "sampled every 50 ms from just before the warm-up to the end of the timed steps"
     if world > 1:
         t = torch.tensor([ms], device=dev)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
@@ -415,6 +482,7 @@ def main():
     peak, peak_kind = peaks()
     achieved = alg_bytes / (dec_ms * 1e-3) / 1e9
     value = w.B * world / (ms * 1e-3)
+    res, pk = runner.mkv.mkv_cache_bytes(runner.cfg, w.T)
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f16" if runner.method != "kvquant" else f"u{w.bits}+f16",
@@ -428,7 +496,33 @@ def main():
                          "peak_kind": peak_kind, "frac_of_8000": achieved / 8000.0,
                          "alg_bytes_per_launch": alg_bytes, "context_at_measure": T_now,
                          "avg_launch_ms": dec_ms},
+            "kv_bytes": {"resident": res * w.L, "peak": pk * w.L, "unit": "bytes, all layers"},
             "clocks": clk}
+    del runner
+    torch.cuda.empty_cache()
+    if world == 1 and args.per_config:
+        line["per_config"] = {}
+        for name in [n for n in args.per_config.split(",") if n and n != args.workload]:
+            wx = WORKLOADS[name]()
+            if args.layers is not None:
+                import dataclasses
+                wx = dataclasses.replace(wx, L=args.layers)
+            rx = Runner(name, wx, dev, args.seed, extra_steps=4 * total + 8)
+            if not args.no_graph:
+                rx.capture()
+            msx = time_steps(rx, args.steps, args.warmup)
+            bx, tx = rx.decode_bytes()
+            dx = time_decode_launches(rx, max(1, min(args.steps, 3)))
+            rres, rpk = rx.mkv.mkv_cache_bytes(rx.cfg, wx.T)
+            line["per_config"][wx.name] = {
+                "tokens_per_s": wx.B / (msx * 1e-3), "ms_per_step": msx, "batch": wx.B, "context": wx.T,
+                "decode_launch_ms": dx, "decode_alg_bytes": bx, "attended_tokens": tx,
+                "decode_gbs": bx / (dx * 1e-3) / 1e9, "frac_of_measured_peak": bx / (dx * 1e-3) / 1e9 / peak,
+                "frac_of_8000": bx / (dx * 1e-3) / 1e9 / 8000.0,
+                "kv_bytes_resident": rres * wx.L, "kv_bytes_peak": rpk * wx.L,
+                "setup_s": rx.setup_s, "gpu_launches_per_step": rx.launches_per_step()}
+            del rx
+            torch.cuda.empty_cache()
     if rank == 0:
         if world == 1:
             v, sample = oracle_tokens_per_s(args.workload, w, args.cpu_budget, seed=args.seed)
