@@ -233,13 +233,13 @@ class Runner:
             self.step()
 
     def launches_per_step(self):
-        # per layer: append (KVQuant: quantize + length advance), (page select), decode + combine,
+        # per layer: append (KVQuant: quantize + length advance), (page select), decode,
         # (score update)
-        per = {"fp16": 3, "kvquant": 4, "h2o": 4, "rocket": 4}[self.method]
+        per = {"fp16": 2, "kvquant": 3, "h2o": 3, "rocket": 3}[self.method]
         return per * self.w.L
 
     def decode_bytes(self):
-        """Algorithmic bytes one decode launch (decode + combine) reads for one layer now."""
+        """Algorithmic bytes one decode launch reads for one layer now."""
         w = self.w
         cache, _ = self.layers[0]
         units = w.B * w.Hkv
@@ -275,27 +275,33 @@ def time_steps(runner, steps, warmup):
     return e0.elapsed_time(e1) / steps
 
 
-def time_decode_launches(runner, steps):
-    """Average duration of one mkv_decode_attention call (decode + combine kernels),
-    CUDA events on the launching stream around each call, eager."""
-    torch, mkv = runner.torch, runner.mkv
-    st = torch.cuda.current_stream()
-    evs = []
-    for _ in range(steps):
+def time_decode_launches(runner, reps):
+    """Average duration of one mkv_decode_attention call (one fused decode kernel per layer):
+    a CUDA graph of every layer's decode call, replayed `reps` times between CUDA events on the
+    launching stream (graph replay removes host launch overhead; the cache is not modified)."""
+    torch = runner.torch
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
         for l in range(runner.w.L):
-            cache, _ = runner.layers[l]
-            runner.append(l)
-            if runner.method == "rocket":
-                mkv.mkv_rocket_select(runner.cfg, runner.q[l].data_ptr(), cache.c, runner.pidx[l].data_ptr())
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record(st)
             runner.decode(l)
-            b.record(st)
-            if runner.method == "h2o":
-                mkv.mkv_h2o_update(runner.cfg, cache.c, runner.ws.data_ptr(), runner.nws)
-            evs.append((a, b))
+    torch.cuda.current_stream().wait_stream(side)
     torch.cuda.synchronize()
-    return statistics.mean(a.elapsed_time(b) for a, b in evs)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for l in range(runner.w.L):
+            runner.decode(l)
+    for _ in range(2):
+        g.replay()
+    st = torch.cuda.current_stream()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record(st)
+    for _ in range(reps):
+        g.replay()
+    b.record(st)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / (reps * runner.w.L)
 
 
 def time_e2e(runner, steps, warmup):
@@ -477,7 +483,7 @@ def main():
         torch.distributed.barrier()
 
     alg_bytes, T_now = runner.decode_bytes()
-    dec_ms = time_decode_launches(runner, max(1, min(args.steps, 5)))
+    dec_ms = time_decode_launches(runner, 10)
     e2e_s, h2d, d2h = time_e2e(runner, max(1, min(args.steps, 5)), 1)
     peak, peak_kind = peaks()
     achieved = alg_bytes / (dec_ms * 1e-3) / 1e9
@@ -492,7 +498,7 @@ def main():
                     "d2h_bytes_per_step": d2h},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": None,
-                         "kernel": "mkv_decode_attention (decode + combine), one layer",
+                         "kernel": "mkv_decode_attention (one fused split-KV decode kernel), one layer",
                          "peak_kind": peak_kind, "frac_of_8000": achieved / 8000.0,
                          "alg_bytes_per_launch": alg_bytes, "context_at_measure": T_now,
                          "avg_launch_ms": dec_ms},
@@ -512,7 +518,7 @@ def main():
                 rx.capture()
             msx = time_steps(rx, args.steps, args.warmup)
             bx, tx = rx.decode_bytes()
-            dx = time_decode_launches(rx, max(1, min(args.steps, 3)))
+            dx = time_decode_launches(rx, 10)
             rres, rpk = rx.mkv.mkv_cache_bytes(rx.cfg, wx.T)
             line["per_config"][wx.name] = {
                 "tokens_per_s": wx.B / (msx * 1e-3), "ms_per_step": msx, "batch": wx.B, "context": wx.T,

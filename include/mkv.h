@@ -15,8 +15,12 @@
  *  - All tensor arguments are DEVICE pointers to caller-allocated memory
  *    unless a parameter says "host".  The library never allocates or frees
  *    device memory; scratch space is the caller's `ws` buffer, sized by
- *    mkv_workspace_size().  Nothing is retained between calls except the
- *    library's status word (see mkv_get_status).
+ *    mkv_workspace_size().  The first 16 KiB of a workspace hold counters
+ *    that must be zero before the first call that uses it (allocate it
+ *    zero-filled); every call leaves them zero again.  Calls that share a
+ *    workspace must not overlap on the GPU.  Nothing is retained between
+ *    calls except the library's status word (see mkv_get_status).
+ *  - B * Hkv is at most 4096.
  *  - fp16 means IEEE binary16 stored as uint16 bits; fp32 is IEEE binary32.
  *  - Calls are asynchronous on `stream` (a cudaStream_t passed as void*;
  *    NULL is the legacy default stream).  Arguments are validated on the host

@@ -90,7 +90,8 @@ def alloc_quant_params(cfg, rope_len: int, device="cuda") -> QuantParams:
 
 
 def workspace(cfg, T_cap: int, device="cuda"):
-    """(tensor, nbytes) of the workspace mkv_workspace_size asks for."""
+    """(tensor, nbytes) of the workspace mkv_workspace_size asks for, zero-filled
+    (its leading counters must start at zero; the library keeps them zero)."""
     import torch
     n = mkv_workspace_size(cfg, T_cap)
-    return torch.empty(n, dtype=torch.uint8, device=device), n
+    return torch.zeros(n, dtype=torch.uint8, device=device), n

@@ -10,13 +10,14 @@
 // core product per 16 dims (G query rows padded to 16): the contraction costs
 // ~5 warp instructions per token, leaving the issue slots to the copies.
 // Online softmax runs in the log2 domain on the accumulator fragments; splits
-// are merged by combine_kernel.
+// are merged by the last CTA of each (batch, kv-head) (mkv_merge.cuh).
 #include <math.h>
 
 #include <mutex>
 
 #include "mkv_common.cuh"
 #include "mkv_internal.h"
+#include "mkv_merge.cuh"
 
 namespace mkv {
 
@@ -42,20 +43,24 @@ struct Fp16Args {
   float* part_o;
   float* logits;          // H2O [B][Hkv][T_cap][G]
   int n_split;
+  MergeArgs merge;
 };
 
-// Virtual token v of (b, kv-head) -> cache slot, or -1 when v attends nothing.
+constexpr int kMaxSplitPages = 1024;   // ROCKET: page ids of one split, staged in shared memory
+
+// Virtual token v of (b, kv-head) -> cache slot to load, or -1 when nothing is loaded.
+// H2O loads every slot and masks it later by its staged position.
 template <int MODE>
-__device__ __forceinline__ int64_t slot_of(const Fp16Args& a, int64_t v, int64_t bh, int n_len, int ns) {
+__device__ __forceinline__ int64_t slot_of(const Fp16Args& a, int64_t v, int n_len, int ns, const int32_t* pages,
+                                           int unit0) {
   if (MODE == 0) {                       // FP16: slots 0..T_len-1
     return v < n_len ? v : -1;
-  } else if (MODE == 1) {                // H2O: slots holding a position
-    if (v >= a.T_cap) return -1;
-    return a.pos[bh * a.T_cap + v] >= 0 ? v : -1;
+  } else if (MODE == 1) {                // H2O: every slot (masked by pos afterwards)
+    return v < a.T_cap ? v : -1;
   } else {                               // ROCKET: selected pages, then the tail page
     const int unit = (int)(v / kPage), within = (int)(v % kPage);
     if (unit < a.kp) {
-      const int p = a.page_idx[bh * a.kp + unit];
+      const int p = pages[unit - unit0];
       return p >= 0 ? (int64_t)p * kPage + within : -1;
     }
     if (unit == a.kp) {
@@ -75,6 +80,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
   constexpr int ROWS_PER_PASS = kThreads / NC;
   extern __shared__ __align__(128) uint8_t smem[];
   int32_t* slotmap = reinterpret_cast<int32_t*>(smem + kStages * 2 * TILE);   // [kStages][kChunk]
+  int32_t* pages = slotmap + kStages * kChunk;                                 // ROCKET [kMaxSplitPages]
 
   const int split = blockIdx.x;
   const int64_t bh = blockIdx.y;
@@ -101,19 +107,38 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
 
   const __half* kbase = a.k + bh * a.T_cap * D;
   const __half* vbase = a.v + bh * a.T_cap * D;
+  const int unit0 = (int)(v_begin / kPage);
+  if (MODE == 2) {                       // this split's page ids, read once
+    int64_t nu64 = ceil_div_dev(v_end, kPage) - unit0;
+    if (nu64 > kMaxSplitPages) nu64 = kMaxSplitPages;
+    const int nu = (int)nu64;
+    for (int u = tid; u < nu; u += kThreads) {
+      const int unit = unit0 + u;
+      pages[u] = unit < a.kp ? a.page_idx[bh * a.kp + unit] : -1;
+    }
+    __syncthreads();
+  }
 
+  // slotmap holds, per row of a stage: the loaded slot (-1: none), or for H2O the slot's
+  // position (-1: empty), staged by cp.async so no load waits on it
   auto load_chunk = [&](int c, int stage) {
     uint8_t* Ks = smem + stage * 2 * TILE;
     uint8_t* Vs = Ks + TILE;
     const int col = tid % NC;
     for (int rr = tid / NC; rr < kChunk; rr += ROWS_PER_PASS) {
       const int64_t v = v_begin + (int64_t)c * kChunk + rr;
-      const int64_t s = v < v_end ? slot_of<MODE>(a, v, bh, n_len, ns) : -1;
+      const int64_t s = v < v_end ? slot_of<MODE>(a, v, n_len, ns, pages, unit0) : -1;
       const int64_t ss = s >= 0 ? s : 0;
       const int off = rr * ROWB + ((col ^ (rr & 7)) << 4);
       cp_async16(Ks + off, kbase + ss * D + col * 8, s >= 0 ? 16 : 0);
       cp_async16(Vs + off, vbase + ss * D + col * 8, s >= 0 ? 16 : 0);
-      if (col == 0) slotmap[stage * kChunk + rr] = (int32_t)s;
+      if (col == 0) {
+        if (MODE == 1 && s >= 0) {
+          cp_async4(&slotmap[stage * kChunk + rr], a.pos + bh * a.T_cap + s, 4);
+        } else {
+          slotmap[stage * kChunk + rr] = (int32_t)s;
+        }
+      }
     }
   };
 
@@ -178,7 +203,10 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
     for (int i = 0; i < 4; ++i) {
       const int32_t s = smap[tk[i]];
       x[i] = s >= 0 ? x[i] * a.scale_log2 : -INFINITY;
-      if (MODE == 1 && g < a.G && s >= 0) a.logits[(bh * a.T_cap + s) * a.G + g] = x[i];
+      if (MODE == 1 && g < a.G && s >= 0) {
+        const int64_t slot = v_begin + (int64_t)c * kChunk + tk[i];
+        a.logits[(bh * a.T_cap + slot) * a.G + g] = x[i];
+      }
       mx = fmaxf(mx, x[i]);
     }
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
@@ -267,40 +295,13 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
       a.part_l[pi] = L;
     }
   }
-}
-
-// out[b][h] = sum_s 2^(m_s - M) o_s / sum_s 2^(m_s - M) l_s   (grid B*Hq, D threads)
-__global__ void combine_kernel(const float* __restrict__ part_m, const float* __restrict__ part_l,
-                               const float* __restrict__ part_o, int n_split, int D,
-                               __half* __restrict__ out, float* __restrict__ m_tot,
-                               float* __restrict__ l_tot) {
-  const int64_t hq = blockIdx.x;
-  const int d = threadIdx.x;
-  const float* pm = part_m + hq * n_split;
-  const float* pl = part_l + hq * n_split;
-  float M = -INFINITY;
-  for (int s = 0; s < n_split; ++s) M = fmaxf(M, pm[s]);
-  float L = 0.f, O = 0.f;
-  if (M != -INFINITY) {
-    for (int s = 0; s < n_split; ++s) {
-      const float ms = pm[s];
-      if (ms == -INFINITY) continue;
-      const float f = exp2f(ms - M);
-      L += pl[s] * f;
-      O += part_o[(hq * n_split + s) * D + d] * f;
-    }
-  }
-  out[hq * D + d] = __float2half_rn(L > 0.f ? O / L : 0.f);
-  if (m_tot != nullptr && d == 0) {
-    m_tot[hq] = M;
-    l_tot[hq] = L;
-  }
+  merge_if_last<D, kThreads>(a.merge, bh, b, kvh);
 }
 
 template <int D, int MODE>
 cudaError_t launch_fp16_t(const Fp16Args& a, int n_units, int n_split, cudaStream_t st) {
   constexpr int TILE = kChunk * D * 2;
-  const size_t smem = (size_t)kStages * 2 * TILE + kStages * kChunk * sizeof(int32_t);
+  const size_t smem = (size_t)kStages * 2 * TILE + (kStages * kChunk + kMaxSplitPages) * sizeof(int32_t);
   cudaError_t e = cudaFuncSetAttribute(decode_fp16_kernel<D, MODE>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
@@ -311,10 +312,24 @@ cudaError_t launch_fp16_t(const Fp16Args& a, int n_units, int n_split, cudaStrea
 
 }  // namespace
 
+MergeArgs merge_args(const mkv_config& c, const DecodeWs& ws, const Split& sp, void* out, bool h2o_stats) {
+  MergeArgs m{};
+  m.part_m = ws.part_m;
+  m.part_l = ws.part_l;
+  m.part_o = ws.part_o;
+  m.counters = ws.counters;
+  m.out = static_cast<__half*>(out);
+  m.m_tot = h2o_stats ? ws.m_tot : nullptr;
+  m.l_tot = h2o_stats ? ws.l_tot : nullptr;
+  m.Hq = c.Hq;
+  m.G = c.Hq / c.Hkv;
+  m.n_split = sp.n_split;
+  return m;
+}
+
 cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const mkv_cache& cache,
                                       const int32_t* page_idx, void* out, const DecodeWs& ws,
                                       const Split& sp, cudaStream_t st) {
-  (void)out;
   Fp16Args a{};
   a.q = static_cast<const __half*>(q);
   a.k = static_cast<const __half*>(cache.k);
@@ -335,6 +350,7 @@ cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const 
   a.part_o = ws.part_o;
   a.logits = ws.logits;
   a.n_split = sp.n_split;
+  a.merge = merge_args(c, ws, sp, out, c.method == MKV_H2O);
   const int units = c.B * c.Hkv;
   const int mode = c.method == MKV_H2O ? 1 : (c.method == MKV_ROCKET ? 2 : 0);
   if (c.D == 128) {
@@ -347,13 +363,6 @@ cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const 
   return launch_fp16_t<64, 2>(a, units, sp.n_split, st);
 }
 
-cudaError_t launch_combine(const mkv_config& c, const DecodeWs& ws, const Split& sp, void* out,
-                           bool h2o_stats, cudaStream_t st) {
-  combine_kernel<<<c.B * c.Hq, c.D, 0, st>>>(ws.part_m, ws.part_l, ws.part_o, sp.n_split, c.D,
-                                             static_cast<__half*>(out), h2o_stats ? ws.m_tot : nullptr,
-                                             h2o_stats ? ws.l_tot : nullptr);
-  return cudaPeekAtLastError();
-}
 
 // ---------------------------------------------------------------------------
 // FP16 decode without a caller workspace (mkv_decode_attention_noalloc).
@@ -412,7 +421,6 @@ extern "C" mkv_status mkv_decode_attention_noalloc(const mkv_config* cfg, const 
   const Split sp = decode_split(*cfg, cache->T_cap);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   e = launch_decode_fp16_family(*cfg, q, *cache, nullptr, out, w, sp, st);
-  if (e == cudaSuccess) e = launch_combine(*cfg, w, sp, out, false, st);
   if (e != cudaSuccess) {
     set_error("decode launch: %s", cudaGetErrorString(e));
     return MKV_ERR_CUDA;

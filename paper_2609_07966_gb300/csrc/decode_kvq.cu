@@ -22,6 +22,7 @@
 
 #include "mkv_common.cuh"
 #include "mkv_internal.h"
+#include "mkv_merge.cuh"
 
 namespace mkv {
 
@@ -49,6 +50,7 @@ struct KvqArgs {
   float* part_m;
   float* part_l;
   float* part_o;
+  MergeArgs merge;
 };
 
 template <int D, int BITS>
@@ -497,6 +499,7 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
       a.part_l[pi] = L;
     }
   }
+  merge_if_last<D, kThr>(a.merge, bh, b, kvh);
 }
 
 template <int D, int BITS>
@@ -515,7 +518,6 @@ cudaError_t launch_kvq_t(const KvqArgs& a, int units, int n_split, cudaStream_t 
 cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_cache& cache,
                                   const mkv_quant_params& qp, void* out, const DecodeWs& ws, const Split& sp,
                                   cudaStream_t st) {
-  (void)out;
   KvqArgs a{};
   a.q = static_cast<const __half*>(q);
   a.k_codes = cache.k_codes;
@@ -543,6 +545,7 @@ cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_
   a.part_m = ws.part_m;
   a.part_l = ws.part_l;
   a.part_o = ws.part_o;
+  a.merge = merge_args(c, ws, sp, out, false);
   const int units = c.B * c.Hkv;
   if (c.D == 128) {
     if (c.bits == 4) return launch_kvq_t<128, 4>(a, units, sp.n_split, st);

@@ -51,7 +51,7 @@ DecodeWs decode_ws(const mkv_config& c, int64_t T_cap, void* base) {
   const Split sp = decode_split(c, T_cap);
   const size_t hq = (size_t)c.B * c.Hq;
   uint8_t* p = static_cast<uint8_t*>(base);
-  size_t off = 0;
+  size_t off = kCounterBytes;
   DecodeWs w{};
   auto take = [&](size_t bytes) -> float* {
     float* r = base ? reinterpret_cast<float*>(p + off) : nullptr;
@@ -61,6 +61,7 @@ DecodeWs decode_ws(const mkv_config& c, int64_t T_cap, void* base) {
   w.part_m = take(hq * sp.n_split * 4);
   w.part_l = take(hq * sp.n_split * 4);
   w.part_o = take(hq * sp.n_split * c.D * 4);
+  w.counters = base ? static_cast<int*>(base) : nullptr;
   if (c.method == MKV_H2O) {
     w.logits = take((size_t)c.B * c.Hkv * T_cap * (c.Hq / c.Hkv) * 4);
     w.m_tot = take(hq * 4);
@@ -72,7 +73,7 @@ DecodeWs decode_ws(const mkv_config& c, int64_t T_cap, void* base) {
 
 PrefillWs prefill_ws(const mkv_config& c, int64_t T, void* base) {
   uint8_t* p = static_cast<uint8_t*>(base);
-  size_t off = 0;
+  size_t off = kCounterBytes;
   auto take = [&](size_t bytes) -> void* {
     void* r = base ? p + off : nullptr;
     off += align256(bytes);
@@ -89,7 +90,7 @@ PrefillWs prefill_ws(const mkv_config& c, int64_t T, void* base) {
 
 CalibWs calib_ws(const mkv_config& c, int64_t N, void* base) {
   uint8_t* p = static_cast<uint8_t*>(base);
-  size_t off = 0;
+  size_t off = kCounterBytes;
   auto take = [&](size_t bytes) -> void* {
     void* r = base ? p + off : nullptr;
     off += align256(bytes);
@@ -137,6 +138,8 @@ mkv_status check_config(const mkv_config* c) {
   MKV_REQUIRE(c->B >= 1 && c->Hq >= 1 && c->Hkv >= 1 && c->D >= 1, MKV_ERR_INVALID_ARG,
               "B, Hq, Hkv, D must be positive");
   MKV_REQUIRE(c->Hq % c->Hkv == 0, MKV_ERR_INVALID_ARG, "Hq %% Hkv != 0");
+  MKV_REQUIRE((int64_t)c->B * c->Hkv <= kMaxUnits, MKV_ERR_UNSUPPORTED, "B * Hkv = %lld above %d",
+              (long long)c->B * c->Hkv, kMaxUnits);
   const int G = c->Hq / c->Hkv;
   MKV_REQUIRE(G == 1 || G == 2 || G == 4 || G == 8, MKV_ERR_UNSUPPORTED, "G = %d not built", G);
   MKV_REQUIRE(c->D == 64 || c->D == 128, MKV_ERR_UNSUPPORTED, "D = %d not built", c->D);
@@ -328,13 +331,14 @@ mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_
               "workspace %zu bytes < %zu needed", ws_bytes, need.bytes);
   const DecodeWs w = decode_ws(*cfg, cache->T_cap, ws);
   const Split sp = decode_split(*cfg, cache->T_cap);
+  MKV_REQUIRE(cfg->method != MKV_ROCKET || (int64_t)sp.chunks_per_split * (kChunk / kPage) + 1 <= 1024,
+              MKV_ERR_UNSUPPORTED, "topk_pages too large for one decode split");
   cudaStream_t st = as_stream(stream);
   if (cfg->method == MKV_KVQUANT) {
     MKV_CUDA(launch_decode_kvquant(*cfg, q, *cache, *qparams, out, w, sp, st));
   } else {
     MKV_CUDA(launch_decode_fp16_family(*cfg, q, *cache, page_idx, out, w, sp, st));
   }
-  MKV_CUDA(launch_combine(*cfg, w, sp, out, cfg->method == MKV_H2O, st));
   return MKV_OK;
 }
 

@@ -16,6 +16,12 @@ constexpr int kPage = 16;        // ROCKET page size (the only one built)
 void set_error(const char* fmt, ...);
 
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Every workspace starts with this many bytes of split tickets (one int per
+// (batch, kv-head)); they must be zero before first use and every call leaves
+// them zero.  Nothing else is ever written there, whatever the config.
+constexpr size_t kCounterBytes = 16384;
+constexpr int kMaxUnits = (int)(kCounterBytes / 4);
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Work split of a decode call: `n_split` CTAs per (batch, kv-head), each over
@@ -35,6 +41,7 @@ struct DecodeWs {
   float* logits;   // H2O: [B][Hkv][T_cap][G] scaled logits (log2 domain)
   float* m_tot;    // H2O: [B][Hq]
   float* l_tot;    // H2O: [B][Hq]
+  int* counters;   // [B][Hkv] split tickets; zero between calls
   size_t bytes;
 };
 DecodeWs decode_ws(const mkv_config& c, int64_t T_cap, void* base);
@@ -58,6 +65,9 @@ struct CalibWs {
 };
 CalibWs calib_ws(const mkv_config& c, int64_t N, void* base);
 
+struct MergeArgs;
+MergeArgs merge_args(const mkv_config& c, const DecodeWs& ws, const Split& sp, void* out, bool h2o_stats);
+
 // ---- launchers (return the launch status; arguments already validated) ----
 cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const mkv_cache& cache,
                                       const int32_t* page_idx, void* out, const DecodeWs& ws,
@@ -65,8 +75,6 @@ cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const 
 cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_cache& cache,
                                   const mkv_quant_params& qp, void* out,
                                   const DecodeWs& ws, const Split& sp, cudaStream_t st);
-cudaError_t launch_combine(const mkv_config& c, const DecodeWs& ws, const Split& sp, void* out,
-                           bool h2o_stats, cudaStream_t st);
 cudaError_t launch_append(const mkv_config& c, const void* k_new, const void* v_new,
                           const mkv_cache& cache, cudaStream_t st);
 cudaError_t launch_rope_table(int D, float theta, int64_t T_max, float* table, cudaStream_t st);

@@ -125,20 +125,35 @@ __global__ void __launch_bounds__(kSelThreads) rocket_select_kernel(const __half
     if (rank < rd) dims[rank] = threadIdx.x;
   }
   __syncthreads();
-  for (int p = threadIdx.x; p < ns; p += blockDim.x) {
-    float sc = 0.f;
-    for (int h = 0; h < G; ++h) {
-      for (int t = 0; t < rd; ++t) {
-        const int i = dims[t];
-        const float qv = qs[h * D + i];
-        const float lo = __half2float(kmin[(bh * D + i) * npc + p]) * qv;
-        const float hi = __half2float(kmax[(bh * D + i) * npc + p]) * qv;
-        sc += fmaxf(lo, hi);
+  // page scores, 256 pages at a time: the selected dims' min/max rows are staged with
+  // coalesced loads (dim-major layout), then each thread scores one page from shared memory
+  __half* bmin = reinterpret_cast<__half*>(ssc + npc);          // [rd][256]
+  __half* bmax = bmin + rd * 256;
+  for (int p0 = 0; p0 < ns; p0 += 256) {
+    const int np = min(256, ns - p0);
+    for (int e = threadIdx.x; e < rd * 256; e += blockDim.x) {
+      const int t = e / 256, pp = e % 256;
+      if (pp < np) {
+        const int64_t src = (bh * D + dims[t]) * npc + p0 + pp;
+        bmin[e] = kmin[src];
+        bmax[e] = kmax[src];
       }
     }
-    ssc[p] = sc;
+    __syncthreads();
+    if (threadIdx.x < np) {
+      float sc = 0.f;
+      for (int h = 0; h < G; ++h) {
+        for (int t = 0; t < rd; ++t) {
+          const float qv = qs[h * D + dims[t]];
+          const float lo = __half2float(bmin[t * 256 + threadIdx.x]) * qv;
+          const float hi = __half2float(bmax[t * 256 + threadIdx.x]) * qv;
+          sc += fmaxf(lo, hi);
+        }
+      }
+      ssc[p0 + threadIdx.x] = sc;
+    }
+    __syncthreads();
   }
-  __syncthreads();
   const int k = min(kp, ns);
   uint64_t thr = ~0ull;
   if (k > 0) thr = block_kth_largest(ns, k, [&](int i) { return rank_key(ssc[i], (uint32_t)i); }, hist);
@@ -184,7 +199,7 @@ cudaError_t launch_snap_keep(const mkv_config& c, const void* full_k, const void
 cudaError_t launch_rocket_select(const mkv_config& c, const void* q, const mkv_cache& cache, int32_t* page_idx,
                                  cudaStream_t st) {
   const int G = c.Hq / c.Hkv;
-  const size_t smem = ((size_t)G * c.D + cache.T_cap / kPage) * sizeof(float);
+  const size_t smem = ((size_t)G * c.D + cache.T_cap / kPage) * sizeof(float) + 2 * (size_t)c.topq_dims * 256 * 2;
   cudaError_t e = cudaFuncSetAttribute(rocket_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   rocket_select_kernel<<<c.B * c.Hkv, kSelThreads, smem, st>>>(
