@@ -295,7 +295,8 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
       a.part_l[pi] = L;
     }
   }
-  merge_if_last<D, kThreads>(a.merge, bh, b, kvh);
+  __syncthreads();                     // the stage buffers now serve as the merge's scratch
+  merge_if_last<D, kThreads>(a.merge, bh, b, kvh, reinterpret_cast<float*>(smem), kStages * 2 * TILE / 4);
 }
 
 template <int D, int MODE>

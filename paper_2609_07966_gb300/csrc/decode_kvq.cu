@@ -499,7 +499,8 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
       a.part_l[pi] = L;
     }
   }
-  merge_if_last<D, kThr>(a.merge, bh, b, kvh);
+  __syncthreads();                     // the stage buffers now serve as the merge's scratch
+  merge_if_last<D, kThr>(a.merge, bh, b, kvh, reinterpret_cast<float*>(stg), 2 * Lay::STAGE / 4);
 }
 
 template <int D, int BITS>

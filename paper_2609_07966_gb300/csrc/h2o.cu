@@ -81,7 +81,7 @@ __global__ void h2o_gather_kernel(const __half* __restrict__ full_k, const __hal
 }
 
 // One CTA per (batch, kv-head): score update and eviction.
-__global__ void __launch_bounds__(256) h2o_update_kernel(const float* __restrict__ logits, const float* __restrict__ m_tot,
+__global__ void __launch_bounds__(1024) h2o_update_kernel(const float* __restrict__ logits, const float* __restrict__ m_tot,
                                                          const float* __restrict__ l_tot, int Hkv, int G, int64_t T_cap,
                                                          int H, int R, const int32_t* __restrict__ T_len,
                                                          int32_t* __restrict__ pos, float* __restrict__ acc,
@@ -106,7 +106,14 @@ __global__ void __launch_bounds__(256) h2o_update_kernel(const float* __restrict
     }
     ++held;
     float add = 0.f;
-    for (int h = 0; h < G; ++h) add += exp2f(logits[(bh * T_cap + s) * G + h] - m[h]) * il[h];
+    const float* lg = logits + (bh * T_cap + s) * G;
+    if (G == 4) {
+      const float4 x = *reinterpret_cast<const float4*>(lg);
+      add = exp2f(x.x - m[0]) * il[0] + exp2f(x.y - m[1]) * il[1] + exp2f(x.z - m[2]) * il[2] +
+            exp2f(x.w - m[3]) * il[3];
+    } else {
+      for (int h = 0; h < G; ++h) add += exp2f(lg[h] - m[h]) * il[h];
+    }
     const float a2 = acc[bh * T_cap + s] + add;
     acc[bh * T_cap + s] = a2;
     if ((int64_t)p <= newest - R) {
@@ -118,9 +125,9 @@ __global__ void __launch_bounds__(256) h2o_update_kernel(const float* __restrict
     }
   }
   // block reductions: held count, first free slot, min key (with its slot)
-  __shared__ int s_held[8], s_free[8];
-  __shared__ uint64_t s_key[8];
-  __shared__ int s_slot[8];
+  __shared__ int s_held[32], s_free[32];
+  __shared__ uint64_t s_key[32];
+  __shared__ int s_slot[32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int o = 16; o > 0; o >>= 1) {
     held += __shfl_xor_sync(0xffffffffu, held, o);
@@ -178,7 +185,7 @@ cudaError_t launch_h2o_keep(const mkv_config& c, const void* full_k, const void*
 }
 
 cudaError_t launch_h2o_update(const mkv_config& c, const mkv_cache& cache, const DecodeWs& ws, cudaStream_t st) {
-  h2o_update_kernel<<<c.B * c.Hkv, 256, 0, st>>>(ws.logits, ws.m_tot, ws.l_tot, c.Hkv, c.Hq / c.Hkv, cache.T_cap,
+  h2o_update_kernel<<<c.B * c.Hkv, 1024, 0, st>>>(ws.logits, ws.m_tot, ws.l_tot, c.Hkv, c.Hq / c.Hkv, cache.T_cap,
                                                  c.h2o_heavy, c.h2o_recent, cache.T_len, cache.pos, cache.acc,
                                                  cache.slot);
   return cudaPeekAtLastError();

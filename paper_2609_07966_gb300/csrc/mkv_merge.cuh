@@ -20,8 +20,10 @@ struct MergeArgs {
   int Hq, G, n_split;
 };
 
+// `scratch`: shared memory the caller no longer needs, `cap` floats of it.
 template <int D, int NT>
-__device__ __forceinline__ void merge_if_last(const MergeArgs& a, int64_t bh, int b, int kvh) {
+__device__ __forceinline__ void merge_if_last(const MergeArgs& a, int64_t bh, int b, int kvh, float* scratch,
+                                              int cap) {
   __shared__ int s_last;
   __threadfence();
   __syncthreads();
@@ -33,21 +35,67 @@ __device__ __forceinline__ void merge_if_last(const MergeArgs& a, int64_t bh, in
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  for (int e = threadIdx.x; e < a.G * D; e += NT) {
+  const int ns = a.n_split, G = a.G;
+  const int64_t hq0 = (int64_t)b * a.Hq + (int64_t)kvh * G;
+  if (2 * G * ns + 2 * G <= cap) {
+    // weights f[row][s] = 2^(m_s - M) and totals, then independent loads of the o partials
+    float* f = scratch;                 // [G][ns]
+    float* tot = scratch + G * ns;      // [G] M, [G] L
+    for (int e = threadIdx.x; e < G * ns; e += NT) f[e] = __ldcg(a.part_m + hq0 * ns + e);
+    __syncthreads();
+    if (threadIdx.x < G) {
+      const int row = threadIdx.x;
+      float M = -INFINITY;
+      for (int s = 0; s < ns; ++s) M = fmaxf(M, f[row * ns + s]);
+      float L = 0.f;
+      for (int s = 0; s < ns; ++s) {
+        const float ms = f[row * ns + s];
+        const float w = (M == -INFINITY || ms == -INFINITY) ? 0.f : exp2f(ms - M);
+        f[row * ns + s] = w;
+        L += __ldcg(a.part_l + (hq0 + row) * ns + s) * w;
+      }
+      tot[row] = M;
+      tot[G + row] = L;
+    }
+    __syncthreads();
+    for (int e = threadIdx.x; e < G * D; e += NT) {
+      const int row = e / D, d = e % D;
+      const float* po = a.part_o + ((hq0 + row) * ns) * D + d;
+      const float* fw = f + row * ns;
+      float O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
+      int s = 0;
+      for (; s + 4 <= ns; s += 4) {
+        O0 += __ldcg(po + (int64_t)(s + 0) * D) * fw[s + 0];
+        O1 += __ldcg(po + (int64_t)(s + 1) * D) * fw[s + 1];
+        O2 += __ldcg(po + (int64_t)(s + 2) * D) * fw[s + 2];
+        O3 += __ldcg(po + (int64_t)(s + 3) * D) * fw[s + 3];
+      }
+      for (; s < ns; ++s) O0 += __ldcg(po + (int64_t)s * D) * fw[s];
+      const float O = (O0 + O1) + (O2 + O3);
+      const float L = tot[G + row];
+      a.out[(hq0 + row) * D + d] = __float2half_rn(L > 0.f ? O / L : 0.f);
+      if (a.m_tot != nullptr && d == 0) {
+        a.m_tot[hq0 + row] = tot[row];
+        a.l_tot[hq0 + row] = L;
+      }
+    }
+    return;
+  }
+  for (int e = threadIdx.x; e < G * D; e += NT) {      // many splits: direct loop
     const int row = e / D, d = e % D;
-    const int64_t hq = (int64_t)b * a.Hq + (int64_t)kvh * a.G + row;
-    const float* pm = a.part_m + hq * a.n_split;
-    const float* pl = a.part_l + hq * a.n_split;
+    const int64_t hq = hq0 + row;
+    const float* pm = a.part_m + hq * ns;
+    const float* pl = a.part_l + hq * ns;
     float M = -INFINITY;
-    for (int s = 0; s < a.n_split; ++s) M = fmaxf(M, __ldcg(pm + s));
+    for (int s = 0; s < ns; ++s) M = fmaxf(M, __ldcg(pm + s));
     float L = 0.f, O = 0.f;
     if (M != -INFINITY) {
-      for (int s = 0; s < a.n_split; ++s) {
+      for (int s = 0; s < ns; ++s) {
         const float ms = __ldcg(pm + s);
         if (ms == -INFINITY) continue;
-        const float f = exp2f(ms - M);
-        L += __ldcg(pl + s) * f;
-        O += __ldcg(a.part_o + (hq * a.n_split + s) * D + d) * f;
+        const float w = exp2f(ms - M);
+        L += __ldcg(pl + s) * w;
+        O += __ldcg(a.part_o + (hq * ns + s) * D + d) * w;
       }
     }
     a.out[hq * D + d] = __float2half_rn(L > 0.f ? O / L : 0.f);

@@ -35,14 +35,27 @@ __device__ uint64_t block_kth_largest(int n, int k, KeyOf key_of, int* hist) {
       if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255], 1);
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      int kr = s_k, bin = 255;
-      for (; bin > 0; --bin) {
-        if (hist[bin] >= kr) break;
-        kr -= hist[bin];
+    if (threadIdx.x < 32) {
+      // lane l owns bins 255-8l .. 248-8l (descending); find the bin holding the kr-th key
+      const int lane = threadIdx.x, kr = s_k;
+      int cnt = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) cnt += hist[255 - 8 * lane - j];
+      int incl = cnt;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
       }
-      s_k = kr;
-      s_prefix = prefix | ((uint64_t)bin << shift);
+      const int excl = incl - cnt;
+      if (excl < kr && incl >= kr) {       // exactly one lane
+        int rem = kr - excl, bin = 255 - 8 * lane;
+        for (int j = 0; j < 8; ++j, --bin) {
+          if (hist[bin] >= rem) break;
+          rem -= hist[bin];
+        }
+        s_k = rem;
+        s_prefix = prefix | ((uint64_t)bin << shift);
+      }
     }
     mask |= (uint64_t)255 << shift;
     __syncthreads();

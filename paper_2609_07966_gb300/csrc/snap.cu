@@ -155,16 +155,36 @@ __global__ void __launch_bounds__(kSelThreads) rocket_select_kernel(const __half
     __syncthreads();
   }
   const int k = min(kp, ns);
-  uint64_t thr = ~0ull;
-  if (k > 0) thr = block_kth_largest(ns, k, [&](int i) { return rank_key(ssc[i], (uint32_t)i); }, hist);
   int base = 0;
-  for (int i0 = 0; i0 < ns; i0 += blockDim.x) {
-    const int i = i0 + threadIdx.x;
-    const int flag = (i < ns && k > 0 && rank_key(ssc[i], (uint32_t)i) >= thr) ? 1 : 0;
+  if (ns <= (int)blockDim.x) {
+    // few pages: each thread ranks its page by counting the pages ahead of it under
+    // (score desc, page asc)
+    const int i = threadIdx.x;
+    int flag = 0;
+    if (i < ns && k > 0) {
+      const float si = ssc[i];
+      int rank = 0;
+      for (int j = 0; j < ns; ++j) {
+        const float sj = ssc[j];
+        rank += (sj > si || (sj == si && j < i)) ? 1 : 0;
+      }
+      flag = rank < k;
+    }
     int total;
     const int before = block_exclusive_scan(flag, warp_sums, &total);
-    if (flag) out[bh * kp + base + before] = i;
-    base += total;
+    if (flag) out[bh * kp + before] = i;
+    base = total;
+  } else {
+    uint64_t thr = ~0ull;
+    if (k > 0) thr = block_kth_largest(ns, k, [&](int i) { return rank_key(ssc[i], (uint32_t)i); }, hist);
+    for (int i0 = 0; i0 < ns; i0 += blockDim.x) {
+      const int i = i0 + threadIdx.x;
+      const int flag = (i < ns && k > 0 && rank_key(ssc[i], (uint32_t)i) >= thr) ? 1 : 0;
+      int total;
+      const int before = block_exclusive_scan(flag, warp_sums, &total);
+      if (flag) out[bh * kp + base + before] = i;
+      base += total;
+    }
   }
   for (int i = base + threadIdx.x; i < kp; i += blockDim.x) out[bh * kp + i] = -1;
 }
