@@ -396,41 +396,52 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     }
     __syncthreads();
 
-    // ---- phase 2: warp w owns tokens 8w..8w+7 of the chunk and every output dim
-    {
+    // ---- phase 2: warps 0-3 each own 16 tokens of the chunk and every output dim
+    if (warp < 4) {
       const bool real = g < a.G;
-      const int base = warp >> 2;                            // tokens 0-31: base t0, 32-63: t0 + 32
+      const int base = warp >> 1;                            // tokens 0-31: base t0, 32-63: t0 + 32
       const uint2* qh2 = reinterpret_cast<const uint2*>(qhi + (base * 8 + (real ? g : 0)) * NP);
       const uint2* ql2 = reinterpret_cast<const uint2*>(qlo + (base * 8 + (real ? g : 0)) * NP);
-      float sc[4] = {0.f, 0.f, 0.f, 0.f};
-      // ldmatrix x4: lanes 0-15 address the hi tile, 16-31 the lo tile (dims kc*16 + 0..7 / 8..15)
-      const int mtx = lane >> 3, rowi = lane & 7;
-      const int tokk = warp * 8 + rowi;
-      const uint8_t* kt = (mtx < 2) ? khi_t : klo_t;
+      float sc[2][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) sc[0][i] = sc[1][i] = 0.f;
+      const int mi = lane >> 3, rowi = lane & 7;
+      const int t0w = warp * 16;
+      const int tokk = t0w + (mi >> 1) * 8 + rowi;
 #pragma unroll
       for (int kc = 0; kc < KC; ++kc) {
         const uint2 ah = real ? qh2[kc * 4 + r] : make_uint2(0u, 0u);
         const uint2 al = real ? ql2[kc * 4 + r] : make_uint2(0u, 0u);
-        uint32_t bk[4];
-        ldsm_x4(bk, kt + tile_off<D>(tokk, kc * 2 + (mtx & 1)));
-        mma16816(sc, ah.x, 0u, ah.y, 0u, bk[0], bk[1]);
-        mma16816(sc, ah.x, 0u, ah.y, 0u, bk[2], bk[3]);
-        mma16816(sc, al.x, 0u, al.y, 0u, bk[0], bk[1]);
+        uint32_t bh[4], bl[4];
+        const int ch = kc * 2 + (mi & 1);
+        ldsm_x4(bh, khi_t + tile_off<D>(tokk, ch));
+        ldsm_x4(bl, klo_t + tile_off<D>(tokk, ch));
+        mma16816(sc[0], ah.x, 0u, ah.y, 0u, bh[0], bh[1]);
+        mma16816(sc[1], ah.x, 0u, ah.y, 0u, bh[2], bh[3]);
+        mma16816(sc[0], ah.x, 0u, ah.y, 0u, bl[0], bl[1]);
+        mma16816(sc[1], ah.x, 0u, ah.y, 0u, bl[2], bl[3]);
+        mma16816(sc[0], al.x, 0u, al.y, 0u, bh[0], bh[1]);
+        mma16816(sc[1], al.x, 0u, al.y, 0u, bh[2], bh[3]);
       }
-      const int tk0 = warp * 8 + 2 * r;
-      float x0 = (t0 + tk0 < n_len) ? sc[0] * a.scale_log2 : -INFINITY;
-      float x1 = (t0 + tk0 + 1 < n_len) ? sc[1] * a.scale_log2 : -INFINITY;
-      float mx = fmaxf(x0, x1);
+      const int tk[4] = {t0w + 2 * r, t0w + 2 * r + 1, t0w + 8 + 2 * r, t0w + 9 + 2 * r};
+      float x[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
+      float mx = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        x[i] = (t0 + tk[i] < n_len) ? x[i] * a.scale_log2 : -INFINITY;
+        mx = fmaxf(mx, x[i]);
+      }
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
       mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
       const float m_new = fmaxf(m_run, mx);
-      float p0 = 0.f, p1 = 0.f, alpha = 1.f;
+      float p[4] = {0.f, 0.f, 0.f, 0.f};
+      float alpha = 1.f;
       if (m_new != -INFINITY) {
         alpha = exp2f(m_run - m_new);
-        p0 = exp2f(x0 - m_new);
-        p1 = exp2f(x1 - m_new);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) p[i] = exp2f(x[i] - m_new);
       }
-      l_part = l_part * alpha + p0 + p1;
+      l_part = l_part * alpha + (p[0] + p[1]) + (p[2] + p[3]);
       m_run = m_new;
       if (__any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll
@@ -439,19 +450,21 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
           o[i][1] *= alpha;
         }
       }
-      const uint32_t pa = pack_half2(p0, p1);
-      const int tokv = warp * 8 + rowi;
+      const uint32_t pa0 = pack_half2(p[0], p[1]);
+      const uint32_t pa2 = pack_half2(p[2], p[3]);
+      const int tokv = t0w + (mi & 1) * 8 + rowi;
 #pragma unroll
-      for (int dq = 0; dq < D / 32; ++dq) {                  // four 8-dim tiles per ldmatrix
+      for (int j = 0; j < D / 16; ++j) {
         uint32_t bv[4];
-        ldsm_x4_t(bv, v_t + tile_off<D>(tokv, dq * 4 + mtx));
-#pragma unroll
-        for (int m = 0; m < 4; ++m) {
-          float d[4] = {o[dq * 4 + m][0], o[dq * 4 + m][1], 0.f, 0.f};
-          mma1688(d, pa, 0u, bv[m]);
-          o[dq * 4 + m][0] = d[0];
-          o[dq * 4 + m][1] = d[1];
-        }
+        ldsm_x4_t(bv, v_t + tile_off<D>(tokv, 2 * j + (mi >> 1)));
+        float d0[4] = {o[2 * j][0], o[2 * j][1], 0.f, 0.f};
+        float d1[4] = {o[2 * j + 1][0], o[2 * j + 1][1], 0.f, 0.f};
+        mma16816(d0, pa0, 0u, pa2, 0u, bv[0], bv[1]);
+        mma16816(d1, pa0, 0u, pa2, 0u, bv[2], bv[3]);
+        o[2 * j][0] = d0[0];
+        o[2 * j][1] = d0[1];
+        o[2 * j + 1][0] = d1[0];
+        o[2 * j + 1][1] = d1[1];
       }
     }
   }
