@@ -151,7 +151,7 @@ typedef struct {
  *   v_tbl fp16 [Hkv][D][2^bits] value table per code: the NUQ centroid, or j
  *                               in uniform mode (filled by mkv_quant_prepare)
  *   rope fp32 [rope_len][D/2][2] (cos, sin) table from mkv_rope_table, with
- *                               rope_len >= the cache's T_cap; decode rotates
+ *                               rope_len >= max(the cache's T_cap, 64); decode rotates
  *                               each dequantized key by its position
  */
 typedef struct {

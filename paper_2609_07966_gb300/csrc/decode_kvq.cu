@@ -7,16 +7,26 @@
 //   v_t = lo_t + scale_t * tbl[code] with outliers restored,
 //   out_h = softmax_t(scale q_h . k_t) v_t.
 //
-// GB300 design: one CTA (8 warps) per (batch, kv-head, split); packed codes are
-// staged by cp.async (double buffer, 64 tokens per chunk).  Phase 1: each
-// thread dequantizes half of one token's key or value row from shared tables
-// (all lanes of a warp read the same channel's table -> conflict-free), rotates
-// key pairs (i, i + D/2) by the token's offset delta from its 32-token base,
-// and writes fp16 tiles (keys as hi + lo halves so the tensor-core product
-// keeps fp32 accuracy).  The base rotation R(tb) is applied to the query
-// instead (q . R(tb+d) k = (R(tb)^T q) . (R(d) k)), so only the 32-entry delta
-// table is needed.  Phase 2: tensor-core QK^T (hi*hi + hi*lo + lo*hi), online
-// softmax and PV as in the fp16 kernel.  Tile columns hold pair i at columns
+// GB300 design: one CTA of 20 warps per (batch, kv-head, split), one CTA per
+// SM, warp-specialised.  Sixteen producer warps stage packed codes by cp.async
+// (three 64-token chunks in flight) and dequantize chunk c into one of two
+// fp16 tile buffers while four consumer warps run the tensor-core attention on
+// the previous chunk from the other; named barriers (FULL / EMPTY per buffer)
+// hand the buffers over.
+//
+// Producers: thread (token row tok, pair group g) dequantizes QP = D/16 pairs
+// (i, i + D/2) of its token's key and value rows from shared per-channel tables
+// (all lanes of a warp read the same channel's table -> conflict-free).  Each
+// key pair is rotated by the token's offset d = tok from the chunk start with
+// a rotation held in registers for the whole kernel (the chunk start's own
+// rotation R(t0) is applied to the query instead:
+// q . R(t0 + d) k = (R(t0)^T q) . (R(d) k)) and written as fp16 hi plus the
+// negated fp16 remainder, so the tensor-core product keeps fp32 accuracy.
+// Dense-and-sparse outliers are restored afterwards in a fix-up pass over the
+// chunk's outlier entries (one thread per entry; key pairs recomputed from the
+// fp16 value(s), value entries overwritten); the key-outlier entries are read
+// one chunk ahead into shared memory.  Consumers: QK^T = q_hi k_hi - q_hi nk_lo + q_lo k_hi, online
+// softmax and PV on 16-token slabs.  Tile columns hold pair i at columns
 // (2i, 2i+1) = channels (i, i + D/2); the output is un-permuted at the end.
 #include <math.h>
 
@@ -28,7 +38,32 @@ namespace mkv {
 
 namespace {
 
-constexpr int kThr = 256;
+constexpr int kProdWarps = 16;                         // dequantize chunk c (+ stage loads)
+constexpr int kConsWarps = 4;                          // attention on chunk c-1 (tensor cores)
+constexpr int kProdThr = kProdWarps * 32;
+constexpr int kThr = (kProdWarps + kConsWarps) * 32;
+constexpr int kGroups = 8;                             // pair groups of a token row
+constexpr int kEntCap = kProdThr;                      // key-outlier entries of a chunk kept in smem
+// named barriers (0 is __syncthreads)
+constexpr int kBarProd = 1;                            // producers only
+constexpr int kBarFull = 2;                            // + buffer: tiles of a chunk are ready
+constexpr int kBarEmpty = 4;                           // + buffer: tiles may be overwritten
+// Register split: the kernel is compiled for (and launched with) kRegLaunch registers a
+// thread; producer warpgroups give registers back, the consumer warpgroup takes them.
+constexpr int kRegLaunch = 96, kRegProd = 88, kRegCons = 128;
+static_assert(kProdThr * kRegProd + (kThr - kProdThr) * kRegCons == kThr * kRegLaunch,
+              "the register split must add up to the launch allocation");
+static_assert(kProdThr % 128 == 0 && (kThr - kProdThr) % 128 == 0, "roles are whole warpgroups");
+
+// bar.sync / bar.arrive are warp-aligned: reconverge the warp first
+__device__ __forceinline__ void bar_sync(int id, int n) {
+  __syncwarp();
+  asm volatile("bar.sync %0, %1;\n" ::"r"(id), "r"(n) : "memory");
+}
+__device__ __forceinline__ void bar_arrive(int id, int n) {
+  __syncwarp();
+  asm volatile("bar.arrive %0, %1;\n" ::"r"(id), "r"(n) : "memory");
+}
 
 struct KvqArgs {
   const __half* q;        // [B][Hq][D]
@@ -44,7 +79,7 @@ struct KvqArgs {
   int64_t rope_len;
   const int32_t* T_len;
   int64_t T_cap, k_out_cap;
-  int Hq, Hkv, G, log2G, n_v;
+  int Hq, Hkv, G, n_v;
   int chunks_per_split, n_split;
   float scale_log2;
   float* part_m;
@@ -57,35 +92,41 @@ template <int D, int BITS>
 struct KvqLayout {
   static constexpr int NP = D / 2;
   static constexpr int K = 1 << BITS;
-  static constexpr int ROWB = D * BITS / 8;                  // packed bytes per token row
-  static constexpr int CP = (ROWB % 16 == 0) ? 16 : 8;       // cp.async granularity
-  static constexpr int SROW0 = (ROWB + 15) / 16 * 16;
-  static constexpr int SROW = ((SROW0 / 16) % 2 == 0) ? SROW0 + 16 : SROW0;   // odd # of 16B
+  static constexpr int ROWW = D * BITS / 32;                 // packed words per token row
+  static constexpr int SROWW = ROWW + 1;                     // staged row stride (odd: conflict-free)
+  static constexpr int QP = NP / kGroups;                    // pairs per producer thread
+  static constexpr int NWG = (QP * 2 * BITS + 31) / 32;      // words holding one group's codes
   static constexpr int TILE = kChunk * D * 2;                // fp16 tile bytes
   static constexpr int NVS = 4;                              // value outliers staged per token (<=)
-  static constexpr int KE_CAP = 128;                         // key outliers staged per chunk (<=)
-  // one pipeline stage: codes, then the chunk's per-token side data
-  static constexpr int S_KC = 0;                             // [64][SROW] key codes
-  static constexpr int S_VC = S_KC + kChunk * SROW;          // [64][SROW] value codes
-  static constexpr int S_VP = S_VC + kChunk * SROW;          // [64] float2 (lo, scale)
-  static constexpr int S_KE = S_VP + kChunk * 8;             // [KE_CAP] uint32 key outliers of the chunk
-  static constexpr int S_VO = S_KE + KE_CAP * 4;             // [64][NVS] uint32 value outliers
-  static constexpr int STAGE = S_VO + kChunk * NVS * 4;
-  // byte offsets
-  static constexpr int DTAB = 0;                             // [NP][32] float2
-  static constexpr int KDQ = DTAB + NP * 32 * 8;             // [D][K] float
+  static constexpr int NS = 4;                               // staged chunks (two in flight ahead)
+  static constexpr int QROW = NP + 8;                        // u32 per query row (padded)
+  // one pipeline stage: codes (row-major, odd word stride), then per-token side data
+  static constexpr int S_KC = 0;                             // [64][SROWW] u32 key codes
+  static constexpr int S_VC = S_KC + ((kChunk * SROWW * 4 + 15) / 16) * 16;
+  static constexpr int S_VP = S_VC + ((kChunk * SROWW * 4 + 15) / 16) * 16;   // [64] float2
+  static constexpr int S_KO = S_VP + kChunk * 8;             // [65] int32 key-outlier CSR offsets
+  static constexpr int S_VO = S_KO + 68 * 4;                 // [NVS][64] u32 value outliers
+  static constexpr int STAGE = S_VO + NVS * kChunk * 4;
+  // one tile buffer: keys (hi, negated lo), values, and the rotated query
+  static constexpr int B_KHI = 0;
+  static constexpr int B_KLO = B_KHI + TILE;
+  static constexpr int B_VT = B_KLO + TILE;
+  static constexpr int B_QH = B_VT + TILE;                   // [8][QROW] q_hi pairs, fragment order
+  static constexpr int B_QN = B_QH + 8 * QROW * 4;           // -q_hi
+  static constexpr int B_QL = B_QN + 8 * QROW * 4;           // q_lo
+  static constexpr int BUF = B_QL + 8 * QROW * 4;
+  // CTA layout
+  static constexpr int DTAB = 0;                             // [NP][64] float2 rotation by delta
+  static constexpr int KDQ = DTAB + NP * kChunk * 8;         // [D][K] float
   static constexpr int VTB = KDQ + D * K * 4;                // [D][K] float
-  static constexpr int QHI = VTB + D * K * 4;                // [2 bases][8][NP] half2 (rotated query, hi)
-  static constexpr int QLO = QHI + 2 * 8 * NP * 4;           // [2][8][NP] half2 (lo)
-  static constexpr int KOFF = QLO + 2 * 8 * NP * 4;          // [3 chunks][68] int32 key-outlier CSR offsets
-  static constexpr int STG = KOFF + 3 * 68 * 4;              // [2 stages][STAGE]
-  static constexpr int KHI = STG + 2 * STAGE;
-  static constexpr int KLO = KHI + TILE;
-  static constexpr int VT = KLO + TILE;
-  static constexpr int BYTES = VT + TILE;
+  static constexpr int ENTS = VTB + D * K * 4;               // [2][kEntCap] u32 key-outlier entries
+  static constexpr int OWNER = ENTS + 2 * kEntCap * 4;       // [kEntCap] u8 token of each entry
+  static constexpr int STG = OWNER + kEntCap;                // [NS][STAGE]
+  static constexpr int BUFS = STG + NS * STAGE;              // [2][BUF]
+  static constexpr int BYTES = BUFS + 2 * BUF;
 };
 
-// the `bits`-wide code of channel-in-pair `which` for pair j of a thread's word array
+// pair j's two `BITS`-wide codes from a group's realigned code words (j compile-time)
 template <int BITS, int NW>
 __device__ __forceinline__ void pair_codes(const uint32_t (&w)[NW], int j, int& lo, int& hi) {
   const int bit = 2 * BITS * j;
@@ -96,32 +137,43 @@ __device__ __forceinline__ void pair_codes(const uint32_t (&w)[NW], int j, int& 
   hi = (int)((x >> BITS) & ((1u << BITS) - 1u));
 }
 
-// pair j's codes read from a packed row in shared memory (any j)
+// pair i's codes read from a packed row in shared memory (any i; the row has a pad word)
 template <int BITS>
-__device__ __forceinline__ void pair_codes_row(const uint8_t* row, int j, int& lo, int& hi) {
-  const int bit = 2 * BITS * j;
+__device__ __forceinline__ void pair_codes_row(const uint32_t* row, int i, int& lo, int& hi) {
+  const int bit = 2 * BITS * i;
   const int wi = bit >> 5, sh = bit & 31;
-  const uint32_t w0 = reinterpret_cast<const uint32_t*>(row)[wi];
-  const uint32_t w1 = reinterpret_cast<const uint32_t*>(row)[wi + 1];
-  const uint32_t x = __funnelshift_r(w0, w1, sh);
+  const uint32_t x = __funnelshift_r(row[wi], row[wi + 1], sh);
   lo = (int)(x & ((1u << BITS) - 1u));
   hi = (int)((x >> BITS) & ((1u << BITS) - 1u));
 }
 
-__device__ __forceinline__ void split_hi_lo(float a, float b, uint32_t& hi, uint32_t& lo) {
-  const __half2 h = __floats2half2_rn(a, b);
-  const float2 hf = __half22float2(h);
-  const __half2 l = __floats2half2_rn(a - hf.x, b - hf.y);
-  hi = *reinterpret_cast<const uint32_t*>(&h);
-  lo = *reinterpret_cast<const uint32_t*>(&l);
+// the code words of pair group g of a staged row, shifted so the group starts at bit 0
+template <int BITS, int QP, int NW>
+__device__ __forceinline__ void group_words(const uint32_t* row, int g, uint32_t (&w)[NW]) {
+  const int bit0 = g * QP * 2 * BITS;
+  const int w0 = bit0 >> 5, sh = bit0 & 31;
+  if ((QP * 2 * BITS) % 32 == 0) {         // groups are word-aligned
+#pragma unroll
+    for (int k = 0; k < NW; ++k) w[k] = row[w0 + k];
+  } else {
+    uint32_t raw[NW + 1];
+#pragma unroll
+    for (int k = 0; k <= NW; ++k) raw[k] = row[w0 + k];
+#pragma unroll
+    for (int k = 0; k < NW; ++k) w[k] = __funnelshift_r(raw[k], raw[k + 1], sh);
+  }
 }
 
-// D(16x8 f32) += A(16x8 f16, row) * B(8x8 f16, col)
-__device__ __forceinline__ void mma1688(float c[4], uint32_t a0, uint32_t a1, uint32_t b0) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k8.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5}, {%6}, {%0,%1,%2,%3};\n"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a0), "r"(a1), "r"(b0));
+// (a, b) as fp16 hi and the negated fp16 remainder (hi - x), exact in fp32
+__device__ __forceinline__ void split_hi_nlo(float a, float b, uint32_t& hi, uint32_t& nlo) {
+  uint32_t h;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(h) : "f"(b), "f"(a));
+  float d0, d1;
+  asm("{.reg .f16 l, u;\n mov.b32 {l, u}, %2;\n sub.rn.f32.f16 %0, l, %3;\n sub.rn.f32.f16 %1, u, %4;\n}"
+      : "=f"(d0), "=f"(d1)
+      : "r"(h), "f"(a), "f"(b));
+  hi = h;
+  nlo = pack_half2(d0, d1);
 }
 
 // byte offset of (row, 16B chunk) in a swizzled fp16 tile of D columns
@@ -131,26 +183,19 @@ __device__ __forceinline__ int tile_off(int row, int ch) {
 }
 
 template <int D, int BITS>
-__global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
+__global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   using Lay = KvqLayout<D, BITS>;
-  constexpr int NP = Lay::NP, K = Lay::K, ROWB = Lay::ROWB, SROW = Lay::SROW;
+  constexpr int NP = Lay::NP, K = Lay::K, ROWW = Lay::ROWW, SROWW = Lay::SROWW, QP = Lay::QP;
+  constexpr int NWG = Lay::NWG, NS = Lay::NS, QROW = Lay::QROW;
   constexpr int KC = D / 16;
-  // Phase 1 splits each row's pairs into GROUPS groups of whole 32-bit words.
-  constexpr int GROUPS = ((NP / 4) * 2 * BITS) % 32 == 0 ? 4 : 2;
-  constexpr int QP = NP / GROUPS;                         // pairs per group
-  constexpr int NWQ = QP * 2 * BITS / 32;                 // code words per group
-  constexpr bool SPLIT_KV = GROUPS == 2;                  // then a thread does K or V, not both
   extern __shared__ __align__(128) uint8_t smem[];
   float2* dtab = reinterpret_cast<float2*>(smem + Lay::DTAB);
   float* kdq = reinterpret_cast<float*>(smem + Lay::KDQ);
   float* vtb = reinterpret_cast<float*>(smem + Lay::VTB);
-  uint32_t* qhi = reinterpret_cast<uint32_t*>(smem + Lay::QHI);
-  uint32_t* qlo = reinterpret_cast<uint32_t*>(smem + Lay::QLO);
+  uint32_t* ents = reinterpret_cast<uint32_t*>(smem + Lay::ENTS);
+  uint8_t* owner = smem + Lay::OWNER;
   uint8_t* stg = smem + Lay::STG;
-  int32_t* kring = reinterpret_cast<int32_t*>(smem + Lay::KOFF);
-  uint8_t* khi_t = smem + Lay::KHI;
-  uint8_t* klo_t = smem + Lay::KLO;
-  uint8_t* v_t = smem + Lay::VT;
+  uint8_t* bufs = smem + Lay::BUFS;
 
   const int split = blockIdx.x;
   const int64_t bh = blockIdx.y;
@@ -163,265 +208,286 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
   if (v_end > n_len) v_end = n_len;
   const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
 
-  const uint8_t* kc_base = a.k_codes + bh * a.T_cap * ROWB;
-  const uint8_t* vc_base = a.v_codes + bh * a.T_cap * ROWB;
-
-  const bool stage_vout = a.n_v <= Lay::NVS;
-  auto load_chunk = [&](int c, int stage) {
-    uint8_t* dst = stg + stage * Lay::STAGE;
-    const int64_t c0 = v_begin + (int64_t)c * kChunk;
-    constexpr int PER_ROW = ROWB / Lay::CP;
-    for (int e = tid; e < 2 * kChunk * PER_ROW; e += kThr) {
-      const int kv = e / (kChunk * PER_ROW);
-      const int rem = e % (kChunk * PER_ROW);
-      const int row = rem / PER_ROW, piece = rem % PER_ROW;
-      const int64_t s = c0 + row;
-      const bool ok = s < n_len;
-      const uint8_t* src = (kv ? vc_base : kc_base) + (ok ? s : 0) * ROWB + piece * Lay::CP;
-      uint8_t* d = dst + (kv ? Lay::S_VC : Lay::S_KC) + row * SROW + piece * Lay::CP;
-      if (Lay::CP == 16) {
-        cp_async16(d, src, ok ? 16 : 0);
-      } else {
-        cp_async8(d, src, ok ? 8 : 0);
-      }
-    }
-    if (tid < kChunk) {                          // value (lo, scale)
-      const int64_t s = c0 + tid;
-      const bool ok = s < n_len;
-      cp_async8(dst + Lay::S_VP + tid * 8, a.v_params + bh * a.T_cap + (ok ? s : 0), ok ? 8 : 0);
-    }
-    if (stage_vout && a.n_v > 0) {
-      for (int e = tid; e < kChunk * a.n_v; e += kThr) {
-        const int row = e / a.n_v, k = e % a.n_v;
-        const int64_t s = c0 + row;
-        const bool ok = s < n_len;
-        cp_async4(dst + Lay::S_VO + (row * Lay::NVS + k) * 4, a.v_out + (bh * a.T_cap + (ok ? s : 0)) * a.n_v + k,
-                  ok ? 4 : 0);
-      }
-    }
-  };
-
-  // key-outlier CSR offsets run one chunk ahead of the codes so that each
-  // chunk's outlier entries can be staged together with its codes
-  auto load_koff = [&](int c) {
-    if (tid <= kChunk) {
-      const int64_t s = min(v_begin + (int64_t)c * kChunk + tid, (int64_t)n_len);
-      cp_async4(kring + (c % 3) * 68 + tid, a.k_out_off + bh * (a.T_cap + 1) + s, 4);
-    }
-  };
-  auto load_kents = [&](int c, int stage) {      // needs chunk c's offsets in kring
-    const int32_t* ko = kring + (c % 3) * 68;
-    const int e0 = ko[0];
-    const int n = min((int)min((int64_t)ko[kChunk], a.k_out_cap) - e0, Lay::KE_CAP);
-    for (int e = tid; e < n; e += kThr)
-      cp_async4(stg + stage * Lay::STAGE + Lay::S_KE + e * 4, a.k_out + bh * a.k_out_cap + e0 + e, 4);
-  };
-  if (nchunks > 0) {
-    load_koff(0);
-    if (nchunks > 1) load_koff(1);
-    cp_async_commit();
-    cp_async_wait<0>();
-    __syncthreads();
-    load_chunk(0, 0);
-    load_kents(0, 0);
-    if (nchunks > 2) load_koff(2);
-    cp_async_commit();
-  }
-  // CTA-resident tables: rotations by delta in [0, 32), dequant tables of this kv-head
-  for (int e = tid; e < NP * 32; e += kThr) {      // coalesced read of rows 0..31, transposed
+  // CTA-resident tables: rotations by delta in [0, 64), dequant tables of this kv-head
+  for (int e = tid; e < NP * kChunk; e += kThr) {  // coalesced read of rope rows 0..63, transposed
     const int d = e / NP, i = e % NP;
-    dtab[i * 32 + d] = a.rope[(int64_t)d * NP + i];
+    dtab[i * kChunk + d] = a.rope[(int64_t)min((int64_t)d, a.rope_len - 1) * NP + i];
   }
   for (int e = tid; e < D * K; e += kThr) {
     kdq[e] = a.k_dq[(int64_t)kvh * D * K + e];
     vtb[e] = __half2float(__ushort_as_half(a.v_tbl[(int64_t)kvh * D * K + e]));
   }
-  // This thread's fixed share of the rotated-query table: element e = (base, head, pair) for
-  // e = tid + k*kThr.  Its raw query pair is loaded once; the rotation of its base is
-  // prefetched one chunk ahead.
-  constexpr int kQE = 2 * 8 * NP / kThr;                   // at most G = 8
-  float qx[kQE], qy[kQE];
-  float2 qcs[kQE];
-  const int nqe = 2 * a.G * NP;
-#pragma unroll
-  for (int k = 0; k < kQE; ++k) {
-    const int e = tid + k * kThr;
-    qx[k] = qy[k] = 0.f;
-    qcs[k] = make_float2(1.f, 0.f);
-    if (e < nqe) {
-      const int t = e / NP, i = e % NP;
-      const int gg = t & (a.G - 1), base = t >> a.log2G;
-      const __half* qr = a.q + ((int64_t)b * a.Hq + (int64_t)kvh * a.G + gg) * D;
-      qx[k] = __half2float(qr[i]);
-      qy[k] = __half2float(qr[i + NP]);
-      if (nchunks > 0) qcs[k] = a.rope[min(v_begin + 32 * base, a.rope_len - 1) * NP + i];
-    }
-  }
+  __syncthreads();
 
-  float o[D / 8][2];
-#pragma unroll
-  for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = 0.f;
-  float m_run = -INFINITY, l_part = 0.f;
-  const int t4 = warp & 3;                 // phase 1: pair group (or K/V role) of this warp
-  const int tok = (warp >> 2) * 32 + lane; // phase 1: this thread's token in the chunk
-  const int dl = tok & 31;                 // its offset from its 32-token base
+  // the four attention warps' (m, l, o) per query row, merged after both roles finish
+  float* wm = reinterpret_cast<float*>(stg);                // [4 warps][8 rows]
+  float* wl = wm + 32;                                       // [4][8]
+  float* wo = wl + 32;                                       // [4][8][D]  natural channel order
 
-  for (int c = 0; c < nchunks; ++c) {
-    cp_async_wait<0>();
-    __syncthreads();
-    if (c + 1 < nchunks) {
-      load_chunk(c + 1, (c + 1) & 1);
-      load_kents(c + 1, (c + 1) & 1);
-    }
-    if (c + 2 < nchunks) load_koff(c + 2);
-    cp_async_commit();
-    const int64_t t0 = v_begin + (int64_t)c * kChunk;      // position of the chunk's first token
-    const uint8_t* st = stg + (c & 1) * Lay::STAGE;
-    const float2* vpar = reinterpret_cast<const float2*>(st + Lay::S_VP);
-    const int32_t* koff = kring + (c % 3) * 68;
-    const uint32_t* kents = reinterpret_cast<const uint32_t*>(st + Lay::S_KE);
-    const int kbase = koff[0];
-    const int kstaged = min((int)min((int64_t)koff[kChunk], a.k_out_cap) - kbase, Lay::KE_CAP);
-    const uint32_t* vouts = reinterpret_cast<const uint32_t*>(st + Lay::S_VO);
+  if (warp < kProdWarps) {
+    // ======================= producers: stage, dequantize, rotate =======================
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegProd) : "memory");
+    const int ptid = tid;
+    const int tok = (warp & 1) * 32 + lane;   // this thread's token row in every chunk
+    const int grp = warp >> 1;                // its pairs: grp * QP .. grp * QP + QP - 1
+    const uint32_t* kc_base = reinterpret_cast<const uint32_t*>(a.k_codes) + bh * a.T_cap * ROWW;
+    const uint32_t* vc_base = reinterpret_cast<const uint32_t*>(a.v_codes) + bh * a.T_cap * ROWW;
+    const uint32_t* gents = a.k_out + bh * a.k_out_cap;
+    const bool stage_vout = a.n_v <= Lay::NVS;
 
-    // ---- query rotated back by each 32-token base tb: R(tb)^T q as hi/lo fp16 pairs, stored in
-    //      the order the mma fragments read: pair i = kc*8 + 4*hf + r at word kc*8 + 2*r + hf
-#pragma unroll
-    for (int k = 0; k < kQE; ++k) {
-      const int e = tid + k * kThr;
-      if (e < nqe) {
-        const int t = e / NP, i = e % NP;
-        const int gg = t & (a.G - 1), base = t >> a.log2G;
-        const float x = qx[k], y = qy[k];
-        const float2 cs = qcs[k];
-        const int wpos = (i / 8) * 8 + (i % 4) * 2 + ((i % 8) / 4);
-        split_hi_lo(x * cs.x + y * cs.y, y * cs.x - x * cs.y, qhi[(base * 8 + gg) * NP + wpos],
-                    qlo[(base * 8 + gg) * NP + wpos]);
-        if (c + 1 < nchunks) qcs[k] = a.rope[min(t0 + kChunk + 32 * base, a.rope_len - 1) * NP + i];
+    const int64_t off_base = bh * (a.T_cap + 1);
+
+    auto load_chunk = [&](int c, int stage) {
+      uint8_t* dst = stg + stage * Lay::STAGE;
+      const int64_t c0 = v_begin + (int64_t)c * kChunk;
+      for (int e = ptid; e < kChunk * ROWW; e += kProdThr) {        // row-contiguous: coalesced
+        const int row = e / ROWW, w = e % ROWW;
+        const int64_t s = c0 + row;
+        const bool ok = s < n_len;
+        const int64_t src = (ok ? s : 0) * ROWW + w;
+        const int d = (row * SROWW + w) * 4;
+        cp_async4(dst + Lay::S_KC + d, kc_base + src, ok ? 4 : 0);
+        cp_async4(dst + Lay::S_VC + d, vc_base + src, ok ? 4 : 0);
       }
+      if (ptid < kChunk) {                                          // value (lo, scale)
+        const int64_t s = c0 + ptid;
+        const bool ok = s < n_len;
+        cp_async8(dst + Lay::S_VP + ptid * 8, a.v_params + bh * a.T_cap + (ok ? s : 0), ok ? 8 : 0);
+      } else if (ptid <= 2 * kChunk) {                              // key-outlier offsets c0 .. c0+64
+        const int i = ptid - kChunk;
+        const int64_t s = min(c0 + i, (int64_t)n_len);
+        cp_async4(dst + Lay::S_KO + i * 4, a.k_out_off + off_base + s, 4);
+      } else if (stage_vout && ptid >= 3 * kChunk && ptid < (3 + Lay::NVS) * kChunk) {
+        const int k = (ptid - 3 * kChunk) / kChunk, row = ptid % kChunk;
+        if (k < a.n_v) {
+          const int64_t s = c0 + row;
+          const bool ok = s < n_len;
+          cp_async4(dst + Lay::S_VO + (k * kChunk + row) * 4, a.v_out + (bh * a.T_cap + (ok ? s : 0)) * a.n_v + k,
+                    ok ? 4 : 0);
+        }
+      }
+    };
+    // this thread's key rotations R(tok) for its pairs: the same in every chunk
+    float2 rot[QP];
+#pragma unroll
+    for (int j = 0; j < QP; ++j) rot[j] = dtab[(grp * QP + j) * kChunk + tok];
+
+    // this thread's element of the rotated-query table (head qg, pair qi)
+    const int nq = a.G * NP;
+    const int qg = ptid / NP, qi = ptid % NP;
+    float qx = 0.f, qy = 0.f;
+    float2 qcs = make_float2(1.f, 0.f);
+    if (ptid < nq) {
+      const __half* qr = a.q + ((int64_t)b * a.Hq + (int64_t)kvh * a.G + qg) * D;
+      qx = __half2float(qr[qi]);
+      qy = __half2float(qr[qi + NP]);
+      if (nchunks > 0) qcs = a.rope[min(v_begin, a.rope_len - 1) * NP + qi];
+    }
+    const int qpos = qg * QROW + (qi / 8) * 8 + (qi % 4) * 2 + ((qi % 8) / 4);
+
+    // key-outlier entries are fetched one chunk ahead, one per thread, into ents[c & 1]
+    if (nchunks > 0) {
+      const int64_t e0 = __ldg(a.k_out_off + off_base + min(v_begin, (int64_t)n_len));
+      const int64_t e1 = min((int64_t)__ldg(a.k_out_off + off_base + min(v_begin + kChunk, (int64_t)n_len)),
+                             a.k_out_cap);
+      ents[ptid] = e0 + ptid < e1 ? __ldg(gents + e0 + ptid) : 0u;
     }
 
-    // ---- phase 1: dequantize one pair group of the thread's token (keys and/or values)
-    {
-      const int64_t slot = t0 + tok;
-      const bool valid = slot < n_len;
-      const bool do_k = SPLIT_KV ? (t4 < 2) : true;
-      const bool do_v = SPLIT_KV ? (t4 >= 2) : true;
-      const int grp = SPLIT_KV ? (t4 & 1) : t4;
-      if (do_k) {
-        const uint8_t* rowfull = st + Lay::S_KC + tok * SROW;
-        uint32_t w[NWQ];
 #pragma unroll
-        for (int k = 0; k < NWQ; ++k) w[k] = reinterpret_cast<const uint32_t*>(rowfull)[grp * NWQ + k];
+    for (int s = 0; s < NS - 1; ++s) {
+      if (s < nchunks) load_chunk(s, s);
+      cp_async_commit();
+    }
+    for (int c = 0; c < nchunks; ++c) {
+      cp_async_wait<NS - 3>();                // this thread's copies of chunks c and c+1 landed
+      bar_sync(kBarProd, kProdThr);           // everyone's landed, ents[c & 1] written; stage c-1 free
+      if (c + NS - 1 < nchunks) load_chunk(c + NS - 1, (c + NS - 1) % NS);
+      cp_async_commit();
+      // read ahead: this thread's key-outlier entry of chunk c+1 (its offsets are staged)
+      uint32_t kent_n = 0u;
+      if (c + 1 < nchunks) {
+        const int32_t* koff_n = reinterpret_cast<const int32_t*>(stg + ((c + 1) % NS) * Lay::STAGE + Lay::S_KO);
+        const int e = koff_n[0] + ptid;
+        if (e < min((int64_t)koff_n[kChunk], a.k_out_cap)) kent_n = __ldg(gents + e);
+      }
+
+      const uint8_t* st = stg + (c % NS) * Lay::STAGE;
+      const int32_t* koff = reinterpret_cast<const int32_t*>(st + Lay::S_KO);
+      const uint32_t* ent_c = ents + (c & 1) * kEntCap;
+      const int E0 = koff[0];
+      const int E1 = (int)min((int64_t)koff[kChunk], a.k_out_cap);
+      // token of each of the chunk's first kEntCap key-outlier entries
+      if (ptid < kChunk) {
+        const int e_hi = min(min(koff[ptid + 1], E1), E0 + kEntCap);
+        for (int e = koff[ptid]; e < e_hi; ++e) owner[e - E0] = (uint8_t)ptid;
+      }
+      const int buf = c & 1;
+      if (c >= 2) bar_sync(kBarEmpty + buf, kThr);   // attention on chunk c-2 released the buffer
+      uint8_t* B_ = bufs + buf * Lay::BUF;
+      uint8_t* khi_t = B_ + Lay::B_KHI;
+      uint8_t* klo_t = B_ + Lay::B_KLO;
+      uint8_t* v_t = B_ + Lay::B_VT;
+      const int64_t t0 = v_begin + (int64_t)c * kChunk;
+
+      // query rotated back by the chunk start: R(t0)^T q as hi, -hi and lo fp16 pairs, stored in
+      // the order the mma fragments read (pair i = kc*8 + 4*hf + r at word kc*8 + 2*r + hf)
+      if (ptid < nq) {
+        const float xr = qx * qcs.x + qy * qcs.y, yr = qy * qcs.x - qx * qcs.y;
+        const uint32_t h = pack_half2(xr, yr);
+        const float2 hf = __half22float2(*reinterpret_cast<const __half2*>(&h));
+        reinterpret_cast<uint32_t*>(B_ + Lay::B_QH)[qpos] = h;
+        reinterpret_cast<uint32_t*>(B_ + Lay::B_QN)[qpos] = h ^ 0x80008000u;
+        reinterpret_cast<uint32_t*>(B_ + Lay::B_QL)[qpos] = pack_half2(xr - hf.x, yr - hf.y);
+        if (c + 1 < nchunks) qcs = a.rope[min(t0 + kChunk, a.rope_len - 1) * NP + qi];
+      }
+
+      // keys: dequantize, rotate by R(tok), split; rows past the cache end were zero-filled
+      // (finite keys, masked in the attention)
+      const uint32_t* krow = reinterpret_cast<const uint32_t*>(st + Lay::S_KC) + tok * SROWW;
+      {
+        uint32_t w[NWG];
+        group_words<BITS, QP, NWG>(krow, grp, w);
+        const float* kq = kdq + grp * QP * K;
 #pragma unroll
         for (int jj = 0; jj < QP; jj += 4) {
           uint32_t ph[4], pl[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const int j = jj + u, i = grp * QP + j;
+            const int j = jj + u;
             int clo, chi;
-            pair_codes<BITS, NWQ>(w, j, clo, chi);
-            // rows past the cache end were zero-filled: finite keys, masked in phase 2
-            const float x = kdq[i * K + clo];
-            const float y = kdq[(i + NP) * K + chi];
-            const float2 cs = dtab[i * 32 + dl];
-            split_hi_lo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph[u], pl[u]);
+            pair_codes<BITS, NWG>(w, j, clo, chi);
+            const float x = kq[j * K + clo];
+            const float y = kq[(j + NP) * K + chi];
+            split_hi_nlo(x * rot[j].x - y * rot[j].y, y * rot[j].x + x * rot[j].y, ph[u], pl[u]);
           }
           const int ch = (grp * QP + jj) / 4;
           *reinterpret_cast<uint4*>(khi_t + tile_off<D>(tok, ch)) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
           *reinterpret_cast<uint4*>(klo_t + tile_off<D>(tok, ch)) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
         }
-        // key outliers of this token in this group: recompute their pair exactly
-        if (valid) {
-          const int e0 = koff[tok], e1 = (int)min((int64_t)koff[tok + 1], a.k_out_cap);
-          const uint32_t* gents = a.k_out + bh * a.k_out_cap;
-          auto ent = [&](int e) { return e - kbase < kstaged ? kents[e - kbase] : gents[e]; };
-          for (int e = e0; e < e1; ++e) {
-            const int chn = (int)(ent(e) >> 16);
-            const int i = chn % NP;
-            if (i / QP != grp) continue;
-            int clo, chi;
-            pair_codes_row<BITS>(rowfull, i, clo, chi);
-            float x = kdq[i * K + clo], y = kdq[(i + NP) * K + chi];
-            for (int f = e0; f < e1; ++f) {
-              const uint32_t ef = ent(f);
-              const int cf = (int)(ef >> 16);
-              if (cf == i) x = h2f((uint16_t)(ef & 0xffffu));
-              if (cf == i + NP) y = h2f((uint16_t)(ef & 0xffffu));
-            }
-            const float2 cs = dtab[i * 32 + dl];
-            uint32_t ph, pl;
-            split_hi_lo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph, pl);
-            const int byte = tile_off<D>(tok, i / 4) + (i % 4) * 4;
-            *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
-            *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
-          }
-        }
       }
-      if (do_v) {
-        const uint8_t* rowfull = st + Lay::S_VC + tok * SROW;
-        uint32_t w[NWQ];
-#pragma unroll
-        for (int k = 0; k < NWQ; ++k) w[k] = reinterpret_cast<const uint32_t*>(rowfull)[grp * NWQ + k];
-        const float2 lp = vpar[tok];
+      // values: rows past the cache end have lo = scale = 0 (zero-filled): value 0
+      {
+        const uint32_t* row = reinterpret_cast<const uint32_t*>(st + Lay::S_VC) + tok * SROWW;
+        uint32_t w[NWG];
+        group_words<BITS, QP, NWG>(row, grp, w);
+        const float2 lp = reinterpret_cast<const float2*>(st + Lay::S_VP)[tok];
+        const float* vq = vtb + grp * QP * K;
 #pragma unroll
         for (int jj = 0; jj < QP; jj += 4) {
           uint32_t pv[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const int j = jj + u, i = grp * QP + j;
+            const int j = jj + u;
             int clo, chi;
-            pair_codes<BITS, NWQ>(w, j, clo, chi);
-            // rows past the cache end have lo = scale = 0 (zero-filled): value 0
-            const float x = fmaf(lp.y, vtb[i * K + clo], lp.x);
-            const float y = fmaf(lp.y, vtb[(i + NP) * K + chi], lp.x);
-            pv[u] = pack_half2(x, y);
+            pair_codes<BITS, NWG>(w, j, clo, chi);
+            pv[u] = pack_half2(fmaf(lp.y, vq[j * K + clo], lp.x), fmaf(lp.y, vq[(j + NP) * K + chi], lp.x));
           }
           const int ch = (grp * QP + jj) / 4;
           *reinterpret_cast<uint4*>(v_t + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
         }
-        if (valid) {
-          const uint32_t* ents = stage_vout ? vouts + tok * Lay::NVS : a.v_out + (bh * a.T_cap + slot) * a.n_v;
-          for (int e = 0; e < a.n_v; ++e) {
-            const uint32_t ev = ents[e];
-            const int chn = (int)(ev >> 16);
-            const int i = chn % NP;
-            if (i / QP != grp) continue;
-            const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
-            *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(tok, col / 8) + (col % 8) * 2) =
-                (uint16_t)(ev & 0xffffu);
+      }
+      ents[((c + 1) & 1) * kEntCap + ptid] = kent_n;   // read after the next barrier
+      bar_sync(kBarProd, kProdThr);           // chunk c's tiles and owner map written
+
+      // key outliers: the thread of entry e rewrites its pair (i, i + D/2) with the fp16 value(s)
+      for (int idx = E0 + ptid; idx < E1; idx += kProdThr) {
+        const uint32_t ev = idx - E0 < kEntCap ? ent_c[idx - E0] : __ldg(gents + idx);
+        int t;
+        if (idx - E0 < kEntCap) {
+          t = owner[idx - E0];
+        } else {                              // beyond the staged entries: search the offsets
+          t = 0;
+#pragma unroll
+          for (int step = kChunk / 2; step >= 1; step >>= 1)
+            if (koff[t + step] <= idx) t += step;
+        }
+        const int ch = (int)(ev >> 16);
+        if (ch >= D) continue;                // not a channel (never written by the quantizer)
+        const int i = ch < NP ? ch : ch - NP;
+        const int partner = ch < NP ? ch + NP : ch - NP;
+        const int f_hi = min(koff[t + 1], E1);
+        bool has_p = false;
+        float pval = 0.f;
+        for (int f = koff[t]; f < f_hi; ++f) {
+          const uint32_t ef = f - E0 < kEntCap ? ent_c[f - E0] : __ldg(gents + f);
+          if ((int)(ef >> 16) == partner) {
+            has_p = true;
+            pval = h2f((uint16_t)(ef & 0xffffu));
           }
         }
+        if (has_p && ch >= NP) continue;      // handled with its partner entry
+        int clo, chi;
+        pair_codes_row<BITS>(reinterpret_cast<const uint32_t*>(st + Lay::S_KC) + t * SROWW, i, clo, chi);
+        const float val = h2f((uint16_t)(ev & 0xffffu));
+        const float x = ch < NP ? val : (has_p ? pval : kdq[i * K + clo]);
+        const float y = ch >= NP ? val : (has_p ? pval : kdq[(i + NP) * K + chi]);
+        const float2 cs = dtab[i * kChunk + t];
+        uint32_t ph, pl;
+        split_hi_nlo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph, pl);
+        const int byte = tile_off<D>(t, i / 4) + (i % 4) * 4;
+        *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
+        *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
       }
+      // value outliers: exact fp16 values over the dequantized ones
+      {
+        const uint32_t* vouts = reinterpret_cast<const uint32_t*>(st + Lay::S_VO);
+        for (int e = ptid; e < kChunk * a.n_v; e += kProdThr) {
+          const int k = e / kChunk, t = e % kChunk;
+          if (t0 + t >= n_len) continue;
+          const uint32_t ev =
+              stage_vout ? vouts[k * kChunk + t] : __ldg(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
+          const int chn = (int)(ev >> 16);
+          if (chn >= D) continue;
+          const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
+          *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(t, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
+        }
+      }
+      bar_arrive(kBarFull + buf, kThr);       // chunk c's tiles are ready
     }
-    __syncthreads();
-
-    // ---- phase 2: warps 0-3 each own 16 tokens of the chunk and every output dim
-    if (warp < 4) {
-      const bool real = g < a.G;
-      const int base = warp >> 1;                            // tokens 0-31: base t0, 32-63: t0 + 32
-      const uint2* qh2 = reinterpret_cast<const uint2*>(qhi + (base * 8 + (real ? g : 0)) * NP);
-      const uint2* ql2 = reinterpret_cast<const uint2*>(qlo + (base * 8 + (real ? g : 0)) * NP);
+    cp_async_wait<0>();
+  } else {
+    // ======================= consumers: tensor-core attention =======================
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegCons) : "memory");
+    const int cw = warp - kProdWarps;        // tokens 16*cw .. 16*cw + 15 of each chunk
+    const bool real = g < a.G;
+    const int mi = lane >> 3, rowi = lane & 7;
+    const int t0w = cw * 16;
+    const int tokk = t0w + (mi >> 1) * 8 + rowi;
+    const int tokv = t0w + (mi & 1) * 8 + rowi;
+    float o[D / 8][2];
+#pragma unroll
+    for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = 0.f;
+    float m_run = -INFINITY, l_part = 0.f;
+    for (int c = 0; c < nchunks; ++c) {
+      const int buf = c & 1;
+      bar_sync(kBarFull + buf, kThr);
+      const uint8_t* B_ = bufs + buf * Lay::BUF;
+      const uint8_t* khi_t = B_ + Lay::B_KHI;
+      const uint8_t* klo_t = B_ + Lay::B_KLO;
+      const uint8_t* v_t = B_ + Lay::B_VT;
+      const int qrow = (real ? g : 0) * (QROW / 2);
+      const uint2* qh2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QH) + qrow;
+      const uint2* qn2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QN) + qrow;
+      const uint2* ql2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QL) + qrow;
+      const int64_t t0 = v_begin + (int64_t)c * kChunk;
       float sc[2][4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) sc[0][i] = sc[1][i] = 0.f;
-      const int mi = lane >> 3, rowi = lane & 7;
-      const int t0w = warp * 16;
-      const int tokk = t0w + (mi >> 1) * 8 + rowi;
 #pragma unroll
       for (int kc = 0; kc < KC; ++kc) {
         const uint2 ah = real ? qh2[kc * 4 + r] : make_uint2(0u, 0u);
+        const uint2 an = real ? qn2[kc * 4 + r] : make_uint2(0u, 0u);
         const uint2 al = real ? ql2[kc * 4 + r] : make_uint2(0u, 0u);
-        uint32_t bh[4], bl[4];
+        uint32_t bhi[4], bnl[4];
         const int ch = kc * 2 + (mi & 1);
-        ldsm_x4(bh, khi_t + tile_off<D>(tokk, ch));
-        ldsm_x4(bl, klo_t + tile_off<D>(tokk, ch));
-        mma16816(sc[0], ah.x, 0u, ah.y, 0u, bh[0], bh[1]);
-        mma16816(sc[1], ah.x, 0u, ah.y, 0u, bh[2], bh[3]);
-        mma16816(sc[0], ah.x, 0u, ah.y, 0u, bl[0], bl[1]);
-        mma16816(sc[1], ah.x, 0u, ah.y, 0u, bl[2], bl[3]);
-        mma16816(sc[0], al.x, 0u, al.y, 0u, bh[0], bh[1]);
-        mma16816(sc[1], al.x, 0u, al.y, 0u, bh[2], bh[3]);
+        ldsm_x4(bhi, khi_t + tile_off<D>(tokk, ch));
+        ldsm_x4(bnl, klo_t + tile_off<D>(tokk, ch));
+        mma16816(sc[0], ah.x, 0u, ah.y, 0u, bhi[0], bhi[1]);
+        mma16816(sc[1], ah.x, 0u, ah.y, 0u, bhi[2], bhi[3]);
+        mma16816(sc[0], an.x, 0u, an.y, 0u, bnl[0], bnl[1]);
+        mma16816(sc[1], an.x, 0u, an.y, 0u, bnl[2], bnl[3]);
+        mma16816(sc[0], al.x, 0u, al.y, 0u, bhi[0], bhi[1]);
+        mma16816(sc[1], al.x, 0u, al.y, 0u, bhi[2], bhi[3]);
       }
       const int tk[4] = {t0w + 2 * r, t0w + 2 * r + 1, t0w + 8 + 2 * r, t0w + 9 + 2 * r};
       float x[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
@@ -452,7 +518,6 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
       }
       const uint32_t pa0 = pack_half2(p[0], p[1]);
       const uint32_t pa2 = pack_half2(p[2], p[3]);
-      const int tokv = t0w + (mi & 1) * 8 + rowi;
 #pragma unroll
       for (int j = 0; j < D / 16; ++j) {
         uint32_t bv[4];
@@ -466,27 +531,23 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
         o[2 * j + 1][0] = d1[0];
         o[2 * j + 1][1] = d1[1];
       }
+      if (c + 2 < nchunks) bar_arrive(kBarEmpty + buf, kThr);   // producers may refill the buffer
     }
-  }
-  cp_async_wait<0>();
-  __syncthreads();
-
-  // ---- merge the eight warps' (m, l, o) per query row; o is in the permuted column order
-  l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
-  l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
-  float* wm = reinterpret_cast<float*>(khi_t);              // [8 warps][8 rows]
-  float* wl = wm + 64;                                       // [8][8]
-  float* wo = wl + 64;                                       // [8][8][D]  natural channel order
-  if (g < a.G) {
-    if (r == 0) {
-      wm[warp * 8 + g] = m_run;
-      wl[warp * 8 + g] = l_part;
-    }
+    // The producers are done with every stage once the last chunk was handed over (and no
+    // stage was filled when there are no chunks), so the stage area takes the partials.
+    l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
+    l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
+    if (g < a.G) {
+      if (r == 0) {
+        wm[cw * 8 + g] = m_run;
+        wl[cw * 8 + g] = l_part;
+      }
 #pragma unroll
-    for (int dt = 0; dt < D / 8; ++dt) {
-      const int chn = dt * 4 + r;                            // column dt*8 + 2r -> channel dt*4 + r
-      wo[(warp * 8 + g) * D + chn] = o[dt][0];
-      wo[(warp * 8 + g) * D + chn + NP] = o[dt][1];
+      for (int dt = 0; dt < D / 8; ++dt) {
+        const int chn = dt * 4 + r;                          // column dt*8 + 2r -> channel dt*4 + r
+        wo[(cw * 8 + g) * D + chn] = o[dt][0];
+        wo[(cw * 8 + g) * D + chn + NP] = o[dt][1];
+      }
     }
   }
   __syncthreads();
@@ -494,11 +555,11 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     const int row = e / D, d = e % D;
     float M = -INFINITY;
 #pragma unroll
-    for (int w = 0; w < 8; ++w) M = fmaxf(M, wm[w * 8 + row]);
+    for (int w = 0; w < kConsWarps; ++w) M = fmaxf(M, wm[w * 8 + row]);
     float L = 0.f, O = 0.f;
     if (M != -INFINITY) {
 #pragma unroll
-      for (int w = 0; w < 8; ++w) {
+      for (int w = 0; w < kConsWarps; ++w) {
         const float f = exp2f(wm[w * 8 + row] - M);
         L += wl[w * 8 + row] * f;
         O += wo[(w * 8 + row) * D + d] * f;
@@ -513,16 +574,24 @@ __global__ void __launch_bounds__(kThr, 2) decode_kvq_kernel(const KvqArgs a) {
     }
   }
   __syncthreads();                     // the stage buffers now serve as the merge's scratch
-  merge_if_last<D, kThr>(a.merge, bh, b, kvh, reinterpret_cast<float*>(stg), 2 * Lay::STAGE / 4);
+  merge_if_last<D, kThr>(a.merge, bh, b, kvh, reinterpret_cast<float*>(stg), Lay::NS * Lay::STAGE / 4);
 }
 
 template <int D, int BITS>
 cudaError_t launch_kvq_t(const KvqArgs& a, int units, int n_split, cudaStream_t st) {
   using Lay = KvqLayout<D, BITS>;
-  static_assert(Lay::BYTES <= 113 * 1024, "two CTAs per SM");
-  cudaError_t e = cudaFuncSetAttribute(decode_kvq_kernel<D, BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       Lay::BYTES);
-  if (e != cudaSuccess) return e;
+  static_assert(Lay::BYTES <= 227 * 1024, "one CTA per SM");
+  static int checked = 0;                 // 1: attributes set and register count verified
+  if (!checked) {
+    cudaFuncAttributes attr;
+    cudaError_t e = cudaFuncGetAttributes(&attr, decode_kvq_kernel<D, BITS>);
+    if (e != cudaSuccess) return e;
+    // the register split above assumes exactly kRegLaunch registers a thread at launch
+    if (attr.numRegs != kRegLaunch) return cudaErrorInvalidConfiguration;
+    e = cudaFuncSetAttribute(decode_kvq_kernel<D, BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, Lay::BYTES);
+    if (e != cudaSuccess) return e;
+    checked = 1;
+  }
   decode_kvq_kernel<D, BITS><<<dim3(n_split, units), kThr, Lay::BYTES, st>>>(a);
   return cudaPeekAtLastError();
 }
@@ -550,8 +619,7 @@ cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_
   a.Hq = c.Hq;
   a.Hkv = c.Hkv;
   a.G = c.Hq / c.Hkv;
-  a.log2G = a.G == 8 ? 3 : (a.G == 4 ? 2 : (a.G == 2 ? 1 : 0));
-  a.n_v = std::min(c.D, (int)ceil((double)c.outlier_frac * c.D));
+    a.n_v = std::min(c.D, (int)ceil((double)c.outlier_frac * c.D));
   a.chunks_per_split = sp.chunks_per_split;
   a.n_split = sp.n_split;
   const float scale = c.softmax_scale > 0.f ? c.softmax_scale : 1.0f / sqrtf((float)c.D);

@@ -28,10 +28,11 @@ Split decode_split(const mkv_config& c, int64_t T_cap) {
   s.v_tokens = c.method == MKV_ROCKET ? (int64_t)(c.topk_pages + 1) * kPage : T_cap;
   const int64_t chunks = std::max<int64_t>(1, ceil_div(s.v_tokens, kChunk));
   const int64_t units = (int64_t)c.B * c.Hkv;
-  // The decode kernels keep two CTAs resident per SM.  Pick the split count
-  // that minimises (waves of CTAs) x (chunks per CTA), i.e. the time of the
-  // busiest SM; among equals prefer fewer splits (smaller partials).
-  const int64_t slots = 2 * kNumSMs;
+  // The fp16-family decode kernels keep two CTAs resident per SM, the KVQuant
+  // kernel one.  Pick the split count that minimises (waves of CTAs) x
+  // (chunks per CTA), i.e. the time of the busiest SM; among equals prefer
+  // fewer splits (smaller partials).
+  const int64_t slots = (c.method == MKV_KVQUANT ? 1 : 2) * kNumSMs;
   int64_t best_n = 1, best_cost = INT64_MAX;
   for (int64_t n = 1; n <= std::min<int64_t>(chunks, 1024); ++n) {
     const int64_t cps = ceil_div(chunks, n);
@@ -324,8 +325,8 @@ mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_
   if (cfg->method == MKV_ROCKET) MKV_REQUIRE(page_idx != nullptr, MKV_ERR_INVALID_ARG, "ROCKET needs page_idx");
   if (cfg->method == MKV_KVQUANT) {
     MKV_TRY(check_qparams(cfg, qparams, true));
-    MKV_REQUIRE(qparams->rope && qparams->rope_len >= std::max<int64_t>(cache->T_cap, 32), MKV_ERR_INVALID_ARG,
-                "KVQUANT decode needs a rope table with rope_len >= max(T_cap, 32)");
+    MKV_REQUIRE(qparams->rope && qparams->rope_len >= std::max<int64_t>(cache->T_cap, 64), MKV_ERR_INVALID_ARG,
+                "KVQUANT decode needs a rope table with rope_len >= max(T_cap, 64)");
   }
   const DecodeWs need = decode_ws(*cfg, cache->T_cap, nullptr);
   MKV_REQUIRE(ws != nullptr && ws_bytes >= need.bytes, MKV_ERR_WORKSPACE,
