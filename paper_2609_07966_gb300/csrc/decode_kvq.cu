@@ -22,10 +22,11 @@
 // rotation R(t0) is applied to the query instead:
 // q . R(t0 + d) k = (R(t0)^T q) . (R(d) k)) and written as fp16 hi plus the
 // negated fp16 remainder, so the tensor-core product keeps fp32 accuracy.
-// Dense-and-sparse outliers are restored afterwards in a fix-up pass over the
-// chunk's outlier entries (one thread per entry; key pairs recomputed from the
-// fp16 value(s), value entries overwritten); the key-outlier entries are read
-// one chunk ahead into shared memory.  Consumers: QK^T = q_hi k_hi - q_hi nk_lo + q_lo k_hi, online
+// Dense-and-sparse outliers: value outliers are written over the dequantized
+// entries by the thread that owns them; key outliers are restored by the
+// consumers before the attention, one thread per outlier entry (the entries are
+// read one chunk ahead): the pair before the rotation is recovered from the
+// tile, the fp16 value(s) put in, and the pair rotated and split again.  Consumers: QK^T = q_hi k_hi - q_hi nk_lo + q_lo k_hi, online
 // softmax and PV on 16-token slabs.  Tile columns hold pair i at columns
 // (2i, 2i+1) = channels (i, i + D/2); the output is un-permuted at the end.
 #include <math.h>
@@ -48,6 +49,7 @@ constexpr int kEntCap = kProdThr;                      // key-outlier entries of
 constexpr int kBarProd = 1;                            // producers only
 constexpr int kBarFull = 2;                            // + buffer: tiles of a chunk are ready
 constexpr int kBarEmpty = 4;                           // + buffer: tiles may be overwritten
+constexpr int kBarCons = 6;                            // consumers only
 // Register split: the kernel is compiled for (and launched with) kRegLaunch registers a
 // thread; producer warpgroups give registers back, the consumer warpgroup takes them.
 constexpr int kRegLaunch = 96, kRegProd = 88, kRegCons = 128;
@@ -114,14 +116,15 @@ struct KvqLayout {
   static constexpr int B_QH = B_VT + TILE;                   // [8][QROW] q_hi pairs, fragment order
   static constexpr int B_QN = B_QH + 8 * QROW * 4;           // -q_hi
   static constexpr int B_QL = B_QN + 8 * QROW * 4;           // q_lo
-  static constexpr int BUF = B_QL + 8 * QROW * 4;
+  static constexpr int B_ENT = B_QL + 8 * QROW * 4;          // [kEntCap] u32 key-outlier entries
+  static constexpr int B_KO = B_ENT + kEntCap * 4;           // [68] int32 their CSR offsets
+  static constexpr int B_OWN = B_KO + 68 * 4;                // [kEntCap] u8 token of each entry
+  static constexpr int BUF = B_OWN + kEntCap;
   // CTA layout
   static constexpr int DTAB = 0;                             // [NP][64] float2 rotation by delta
   static constexpr int KDQ = DTAB + NP * kChunk * 8;         // [D][K] float
   static constexpr int VTB = KDQ + D * K * 4;                // [D][K] float
-  static constexpr int ENTS = VTB + D * K * 4;               // [2][kEntCap] u32 key-outlier entries
-  static constexpr int OWNER = ENTS + 2 * kEntCap * 4;       // [kEntCap] u8 token of each entry
-  static constexpr int STG = OWNER + kEntCap;                // [NS][STAGE]
+  static constexpr int STG = VTB + D * K * 4;                // [NS][STAGE]
   static constexpr int BUFS = STG + NS * STAGE;              // [2][BUF]
   static constexpr int BYTES = BUFS + 2 * BUF;
 };
@@ -192,8 +195,6 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   float2* dtab = reinterpret_cast<float2*>(smem + Lay::DTAB);
   float* kdq = reinterpret_cast<float*>(smem + Lay::KDQ);
   float* vtb = reinterpret_cast<float*>(smem + Lay::VTB);
-  uint32_t* ents = reinterpret_cast<uint32_t*>(smem + Lay::ENTS);
-  uint8_t* owner = smem + Lay::OWNER;
   uint8_t* stg = smem + Lay::STG;
   uint8_t* bufs = smem + Lay::BUFS;
 
@@ -285,12 +286,13 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     }
     const int qpos = qg * QROW + (qi / 8) * 8 + (qi % 4) * 2 + ((qi % 8) / 4);
 
-    // key-outlier entries are fetched one chunk ahead, one per thread, into ents[c & 1]
+    // key-outlier entries are fetched one chunk ahead, one per thread
+    uint32_t kent = 0u;
     if (nchunks > 0) {
       const int64_t e0 = __ldg(a.k_out_off + off_base + min(v_begin, (int64_t)n_len));
       const int64_t e1 = min((int64_t)__ldg(a.k_out_off + off_base + min(v_begin + kChunk, (int64_t)n_len)),
                              a.k_out_cap);
-      ents[ptid] = e0 + ptid < e1 ? __ldg(gents + e0 + ptid) : 0u;
+      if (e0 + ptid < e1) kent = __ldg(gents + e0 + ptid);
     }
 
 #pragma unroll
@@ -300,7 +302,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     }
     for (int c = 0; c < nchunks; ++c) {
       cp_async_wait<NS - 3>();                // this thread's copies of chunks c and c+1 landed
-      bar_sync(kBarProd, kProdThr);           // everyone's landed, ents[c & 1] written; stage c-1 free
+      bar_sync(kBarProd, kProdThr);           // everyone's landed; the stage of chunk c-1 is free
       if (c + NS - 1 < nchunks) load_chunk(c + NS - 1, (c + NS - 1) % NS);
       cp_async_commit();
       // read ahead: this thread's key-outlier entry of chunk c+1 (its offsets are staged)
@@ -313,14 +315,6 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
 
       const uint8_t* st = stg + (c % NS) * Lay::STAGE;
       const int32_t* koff = reinterpret_cast<const int32_t*>(st + Lay::S_KO);
-      const uint32_t* ent_c = ents + (c & 1) * kEntCap;
-      const int E0 = koff[0];
-      const int E1 = (int)min((int64_t)koff[kChunk], a.k_out_cap);
-      // token of each of the chunk's first kEntCap key-outlier entries
-      if (ptid < kChunk) {
-        const int e_hi = min(min(koff[ptid + 1], E1), E0 + kEntCap);
-        for (int e = koff[ptid]; e < e_hi; ++e) owner[e - E0] = (uint8_t)ptid;
-      }
       const int buf = c & 1;
       if (c >= 2) bar_sync(kBarEmpty + buf, kThr);   // attention on chunk c-2 released the buffer
       uint8_t* B_ = bufs + buf * Lay::BUF;
@@ -328,6 +322,15 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       uint8_t* klo_t = B_ + Lay::B_KLO;
       uint8_t* v_t = B_ + Lay::B_VT;
       const int64_t t0 = v_begin + (int64_t)c * kChunk;
+
+      // hand the chunk's key-outlier entries, their offsets and owners to the consumers
+      reinterpret_cast<uint32_t*>(B_ + Lay::B_ENT)[ptid] = kent;
+      if (ptid <= kChunk) reinterpret_cast<int32_t*>(B_ + Lay::B_KO)[ptid] = koff[ptid];
+      if (ptid < kChunk) {
+        const int E0 = koff[0];
+        const int e_hi = min((int)min((int64_t)koff[ptid + 1], a.k_out_cap), E0 + kEntCap);
+        for (int e = koff[ptid]; e < e_hi; ++e) (B_ + Lay::B_OWN)[e - E0] = (uint8_t)ptid;
+      }
 
       // query rotated back by the chunk start: R(t0)^T q as hi, -hi and lo fp16 pairs, stored in
       // the order the mma fragments read (pair i = kc*8 + 4*hf + r at word kc*8 + 2*r + hf)
@@ -386,62 +389,21 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
           *reinterpret_cast<uint4*>(v_t + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
         }
       }
-      ents[((c + 1) & 1) * kEntCap + ptid] = kent_n;   // read after the next barrier
-      bar_sync(kBarProd, kProdThr);           // chunk c's tiles and owner map written
-
-      // key outliers: the thread of entry e rewrites its pair (i, i + D/2) with the fp16 value(s)
-      for (int idx = E0 + ptid; idx < E1; idx += kProdThr) {
-        const uint32_t ev = idx - E0 < kEntCap ? ent_c[idx - E0] : __ldg(gents + idx);
-        int t;
-        if (idx - E0 < kEntCap) {
-          t = owner[idx - E0];
-        } else {                              // beyond the staged entries: search the offsets
-          t = 0;
-#pragma unroll
-          for (int step = kChunk / 2; step >= 1; step >>= 1)
-            if (koff[t + step] <= idx) t += step;
-        }
-        const int ch = (int)(ev >> 16);
-        if (ch >= D) continue;                // not a channel (never written by the quantizer)
-        const int i = ch < NP ? ch : ch - NP;
-        const int partner = ch < NP ? ch + NP : ch - NP;
-        const int f_hi = min(koff[t + 1], E1);
-        bool has_p = false;
-        float pval = 0.f;
-        for (int f = koff[t]; f < f_hi; ++f) {
-          const uint32_t ef = f - E0 < kEntCap ? ent_c[f - E0] : __ldg(gents + f);
-          if ((int)(ef >> 16) == partner) {
-            has_p = true;
-            pval = h2f((uint16_t)(ef & 0xffffu));
-          }
-        }
-        if (has_p && ch >= NP) continue;      // handled with its partner entry
-        int clo, chi;
-        pair_codes_row<BITS>(reinterpret_cast<const uint32_t*>(st + Lay::S_KC) + t * SROWW, i, clo, chi);
-        const float val = h2f((uint16_t)(ev & 0xffffu));
-        const float x = ch < NP ? val : (has_p ? pval : kdq[i * K + clo]);
-        const float y = ch >= NP ? val : (has_p ? pval : kdq[(i + NP) * K + chi]);
-        const float2 cs = dtab[i * kChunk + t];
-        uint32_t ph, pl;
-        split_hi_nlo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph, pl);
-        const int byte = tile_off<D>(t, i / 4) + (i % 4) * 4;
-        *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
-        *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
-      }
-      // value outliers: exact fp16 values over the dequantized ones
-      {
+      // value outliers of this token in this thread's pairs: exact fp16 values
+      if (t0 + tok < n_len) {
         const uint32_t* vouts = reinterpret_cast<const uint32_t*>(st + Lay::S_VO);
-        for (int e = ptid; e < kChunk * a.n_v; e += kProdThr) {
-          const int k = e / kChunk, t = e % kChunk;
-          if (t0 + t >= n_len) continue;
+        for (int k = 0; k < a.n_v; ++k) {
           const uint32_t ev =
-              stage_vout ? vouts[k * kChunk + t] : __ldg(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
+              stage_vout ? vouts[k * kChunk + tok] : __ldg(a.v_out + (bh * a.T_cap + t0 + tok) * a.n_v + k);
           const int chn = (int)(ev >> 16);
           if (chn >= D) continue;
+          const int i = chn < NP ? chn : chn - NP;
+          if ((unsigned)(i - grp * QP) >= (unsigned)QP) continue;
           const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
-          *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(t, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
+          *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(tok, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
         }
       }
+      kent = kent_n;
       bar_arrive(kBarFull + buf, kThr);       // chunk c's tiles are ready
     }
     cp_async_wait<0>();
@@ -461,10 +423,66 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     for (int c = 0; c < nchunks; ++c) {
       const int buf = c & 1;
       bar_sync(kBarFull + buf, kThr);
-      const uint8_t* B_ = bufs + buf * Lay::BUF;
-      const uint8_t* khi_t = B_ + Lay::B_KHI;
-      const uint8_t* klo_t = B_ + Lay::B_KLO;
+      uint8_t* B_ = bufs + buf * Lay::BUF;
+      uint8_t* khi_t = B_ + Lay::B_KHI;
+      uint8_t* klo_t = B_ + Lay::B_KLO;
       const uint8_t* v_t = B_ + Lay::B_VT;
+      // key outliers: the thread of entry e recovers its pair before the rotation from the
+      // tile (hi - nlo, then R(d)^T), puts in the fp16 value(s), rotates and splits again
+      {
+        const int32_t* ko = reinterpret_cast<const int32_t*>(B_ + Lay::B_KO);
+        const uint32_t* ents = reinterpret_cast<const uint32_t*>(B_ + Lay::B_ENT);
+        const uint8_t* own = B_ + Lay::B_OWN;
+        const uint32_t* gents = a.k_out + bh * a.k_out_cap;
+        const int E0 = ko[0];
+        const int E1 = (int)min((int64_t)ko[kChunk], a.k_out_cap);
+        for (int idx = E0 + (tid - kProdThr); idx < E1; idx += kThr - kProdThr) {
+          const bool staged = idx - E0 < kEntCap;
+          const uint32_t ev = staged ? ents[idx - E0] : __ldg(gents + idx);
+          int t;
+          if (staged) {
+            t = own[idx - E0];
+          } else {                            // beyond the staged entries: search the offsets
+            t = 0;
+#pragma unroll
+            for (int step = kChunk / 2; step >= 1; step >>= 1)
+              if (ko[t + step] <= idx) t += step;
+          }
+          const int ch = (int)(ev >> 16);
+          if (ch >= D) continue;              // not a channel (never written by the quantizer)
+          const int i = ch < NP ? ch : ch - NP;
+          const int partner = ch < NP ? ch + NP : ch - NP;
+          const int f_hi = min(ko[t + 1], E1);
+          bool has_p = false;
+          float pval = 0.f;
+          for (int f = ko[t]; f < f_hi; ++f) {
+            const uint32_t ef = f - E0 < kEntCap ? ents[f - E0] : __ldg(gents + f);
+            if ((int)(ef >> 16) == partner) {
+              has_p = true;
+              pval = h2f((uint16_t)(ef & 0xffffu));
+            }
+          }
+          if (has_p && ch >= NP) continue;    // handled with its partner entry
+          const int byte = tile_off<D>(t, i / 4) + (i % 4) * 4;
+          const float2 hf = __half22float2(*reinterpret_cast<const __half2*>(khi_t + byte));
+          const float2 nf = __half22float2(*reinterpret_cast<const __half2*>(klo_t + byte));
+          const float kx = hf.x - nf.x, ky = hf.y - nf.y;
+          const float2 cs = dtab[i * kChunk + t];
+          float x = kx * cs.x + ky * cs.y, y = ky * cs.x - kx * cs.y;
+          const float val = h2f((uint16_t)(ev & 0xffffu));
+          if (ch < NP) {
+            x = val;
+            if (has_p) y = pval;
+          } else {
+            y = val;
+          }
+          uint32_t ph, pl;
+          split_hi_nlo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph, pl);
+          *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
+          *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
+        }
+        bar_sync(kBarCons, kThr - kProdThr);  // every consumer warp reads every row
+      }
       const int qrow = (real ? g : 0) * (QROW / 2);
       const uint2* qh2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QH) + qrow;
       const uint2* qn2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QN) + qrow;
