@@ -22,11 +22,11 @@
 // rotation R(t0) is applied to the query instead:
 // q . R(t0 + d) k = (R(t0)^T q) . (R(d) k)) and written as fp16 hi plus the
 // negated fp16 remainder, so the tensor-core product keeps fp32 accuracy.
-// Dense-and-sparse outliers: value outliers are written over the dequantized
-// entries by the thread that owns them; key outliers are restored by the
-// consumers before the attention, one thread per outlier entry (the entries are
-// read one chunk ahead): the pair before the rotation is recovered from the
-// tile, the fp16 value(s) put in, and the pair rotated and split again.  Consumers: QK^T = q_hi k_hi - q_hi nk_lo + q_lo k_hi, online
+// Dense-and-sparse outliers are restored by the consumers before the
+// attention, one thread per outlier entry (key entries are read one chunk
+// ahead): a value outlier overwrites its tile entry; for a key outlier the
+// pair before the rotation is recovered from the tile, the fp16 value(s) put
+// in, and the pair rotated and split again.  Consumers: QK^T = q_hi k_hi - q_hi nk_lo + q_lo k_hi, online
 // softmax and PV on 16-token slabs.  Tile columns hold pair i at columns
 // (2i, 2i+1) = channels (i, i + D/2); the output is un-permuted at the end.
 #include <math.h>
@@ -119,7 +119,8 @@ struct KvqLayout {
   static constexpr int B_ENT = B_QL + 8 * QROW * 4;          // [kEntCap] u32 key-outlier entries
   static constexpr int B_KO = B_ENT + kEntCap * 4;           // [68] int32 their CSR offsets
   static constexpr int B_OWN = B_KO + 68 * 4;                // [kEntCap] u8 token of each entry
-  static constexpr int BUF = B_OWN + kEntCap;
+  static constexpr int B_VO = B_OWN + kEntCap;               // [NVS][64] u32 value outliers
+  static constexpr int BUF = B_VO + NVS * kChunk * 4;
   // CTA layout
   static constexpr int DTAB = 0;                             // [NP][64] float2 rotation by delta
   static constexpr int KDQ = DTAB + NP * kChunk * 8;         // [D][K] float
@@ -177,6 +178,13 @@ __device__ __forceinline__ void split_hi_nlo(float a, float b, uint32_t& hi, uin
       : "r"(h), "f"(a), "f"(b));
   hi = h;
   nlo = pack_half2(d0, d1);
+}
+
+__device__ __forceinline__ void cp_async4s(uint32_t saddr, const void* gmem, int src_bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(saddr), "l"(gmem), "r"(src_bytes));
+}
+__device__ __forceinline__ void cp_async8s(uint32_t saddr, const void* gmem, int src_bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(saddr), "l"(gmem), "r"(src_bytes));
 }
 
 // byte offset of (row, 16B chunk) in a swizzled fp16 tile of D columns
@@ -238,33 +246,39 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
 
     const int64_t off_base = bh * (a.T_cap + 1);
 
+    const uint32_t stg_s = smem_addr(stg);
+    constexpr int NCW = kChunk * ROWW;                       // code words per chunk (keys or values)
+    constexpr int NIT = (NCW + kProdThr - 1) / kProdThr;
     auto load_chunk = [&](int c, int stage) {
-      uint8_t* dst = stg + stage * Lay::STAGE;
-      const int64_t c0 = v_begin + (int64_t)c * kChunk;
-      for (int e = ptid; e < kChunk * ROWW; e += kProdThr) {        // row-contiguous: coalesced
-        const int row = e / ROWW, w = e % ROWW;
-        const int64_t s = c0 + row;
-        const bool ok = s < n_len;
-        const int64_t src = (ok ? s : 0) * ROWW + w;
-        const int d = (row * SROWW + w) * 4;
-        cp_async4(dst + Lay::S_KC + d, kc_base + src, ok ? 4 : 0);
-        cp_async4(dst + Lay::S_VC + d, vc_base + src, ok ? 4 : 0);
+      const uint32_t dst = stg_s + stage * Lay::STAGE;
+      const int64_t c0 = v_begin + (int64_t)c * kChunk;     // < n_len: the chunk has a first row
+      const int lim = (int)min((int64_t)kChunk, (int64_t)n_len - c0);
+      const uint32_t* kc = kc_base + c0 * ROWW;
+      const uint32_t* vc = vc_base + c0 * ROWW;
+#pragma unroll
+      for (int k = 0; k < NIT; ++k) {                        // row-contiguous: coalesced
+        const int e = ptid + k * kProdThr;
+        if (NCW % kProdThr == 0 || e < NCW) {
+          const int row = e / ROWW, w = e % ROWW;
+          const bool ok = row < lim;
+          const int src = ok ? e : 0;
+          const uint32_t d = dst + (row * SROWW + w) * 4;
+          cp_async4s(d + Lay::S_KC, kc + src, ok ? 4 : 0);
+          cp_async4s(d + Lay::S_VC, vc + src, ok ? 4 : 0);
+        }
       }
       if (ptid < kChunk) {                                          // value (lo, scale)
-        const int64_t s = c0 + ptid;
-        const bool ok = s < n_len;
-        cp_async8(dst + Lay::S_VP + ptid * 8, a.v_params + bh * a.T_cap + (ok ? s : 0), ok ? 8 : 0);
+        const bool ok = ptid < lim;
+        cp_async8s(dst + Lay::S_VP + ptid * 8, a.v_params + bh * a.T_cap + c0 + (ok ? ptid : 0), ok ? 8 : 0);
       } else if (ptid <= 2 * kChunk) {                              // key-outlier offsets c0 .. c0+64
         const int i = ptid - kChunk;
-        const int64_t s = min(c0 + i, (int64_t)n_len);
-        cp_async4(dst + Lay::S_KO + i * 4, a.k_out_off + off_base + s, 4);
+        cp_async4s(dst + Lay::S_KO + i * 4, a.k_out_off + off_base + c0 + min(i, lim), 4);
       } else if (stage_vout && ptid >= 3 * kChunk && ptid < (3 + Lay::NVS) * kChunk) {
         const int k = (ptid - 3 * kChunk) / kChunk, row = ptid % kChunk;
         if (k < a.n_v) {
-          const int64_t s = c0 + row;
-          const bool ok = s < n_len;
-          cp_async4(dst + Lay::S_VO + (k * kChunk + row) * 4, a.v_out + (bh * a.T_cap + (ok ? s : 0)) * a.n_v + k,
-                    ok ? 4 : 0);
+          const bool ok = row < lim;
+          cp_async4s(dst + Lay::S_VO + (k * kChunk + row) * 4, a.v_out + (bh * a.T_cap + c0 + (ok ? row : 0)) * a.n_v + k,
+                     ok ? 4 : 0);
         }
       }
     };
@@ -326,6 +340,8 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       // hand the chunk's key-outlier entries, their offsets and owners to the consumers
       reinterpret_cast<uint32_t*>(B_ + Lay::B_ENT)[ptid] = kent;
       if (ptid <= kChunk) reinterpret_cast<int32_t*>(B_ + Lay::B_KO)[ptid] = koff[ptid];
+      if (stage_vout && ptid < kChunk * a.n_v)
+        reinterpret_cast<uint32_t*>(B_ + Lay::B_VO)[ptid] = reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[ptid];
       if (ptid < kChunk) {
         const int E0 = koff[0];
         const int e_hi = min((int)min((int64_t)koff[ptid + 1], a.k_out_cap), E0 + kEntCap);
@@ -389,20 +405,6 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
           *reinterpret_cast<uint4*>(v_t + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
         }
       }
-      // value outliers of this token in this thread's pairs: exact fp16 values
-      if (t0 + tok < n_len) {
-        const uint32_t* vouts = reinterpret_cast<const uint32_t*>(st + Lay::S_VO);
-        for (int k = 0; k < a.n_v; ++k) {
-          const uint32_t ev =
-              stage_vout ? vouts[k * kChunk + tok] : __ldg(a.v_out + (bh * a.T_cap + t0 + tok) * a.n_v + k);
-          const int chn = (int)(ev >> 16);
-          if (chn >= D) continue;
-          const int i = chn < NP ? chn : chn - NP;
-          if ((unsigned)(i - grp * QP) >= (unsigned)QP) continue;
-          const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
-          *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(tok, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
-        }
-      }
       kent = kent_n;
       bar_arrive(kBarFull + buf, kThr);       // chunk c's tiles are ready
     }
@@ -426,7 +428,8 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       uint8_t* B_ = bufs + buf * Lay::BUF;
       uint8_t* khi_t = B_ + Lay::B_KHI;
       uint8_t* klo_t = B_ + Lay::B_KLO;
-      const uint8_t* v_t = B_ + Lay::B_VT;
+      uint8_t* v_t = B_ + Lay::B_VT;
+      const int64_t t0 = v_begin + (int64_t)c * kChunk;
       // key outliers: the thread of entry e recovers its pair before the rotation from the
       // tile (hi - nlo, then R(d)^T), puts in the fp16 value(s), rotates and splits again
       {
@@ -481,13 +484,24 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
           *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
           *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
         }
+        // value outliers: exact fp16 values over the dequantized ones
+        const bool stage_vout = a.n_v <= Lay::NVS;
+        const uint32_t* vo = reinterpret_cast<const uint32_t*>(B_ + Lay::B_VO);
+        for (int e = tid - kProdThr; e < kChunk * a.n_v; e += kThr - kProdThr) {
+          const int k = e / kChunk, t = e % kChunk;
+          if (t0 + t >= n_len) continue;
+          const uint32_t ev = stage_vout ? vo[e] : __ldg(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
+          const int chn = (int)(ev >> 16);
+          if (chn >= D) continue;
+          const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
+          *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(t, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
+        }
         bar_sync(kBarCons, kThr - kProdThr);  // every consumer warp reads every row
       }
       const int qrow = (real ? g : 0) * (QROW / 2);
       const uint2* qh2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QH) + qrow;
       const uint2* qn2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QN) + qrow;
       const uint2* ql2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QL) + qrow;
-      const int64_t t0 = v_begin + (int64_t)c * kChunk;
       float sc[2][4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) sc[0][i] = sc[1][i] = 0.f;
