@@ -338,6 +338,22 @@ def time_e2e(runner, steps, warmup):
     return dt, h2d, d2h
 
 
+def captured_traffic(workload: str):
+    """DRAM bytes (read + write) of one decode launch from the committed ncu capture of this workload,
+    or None when there is none or the kernel source changed since it was taken."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    ent = json.load(open(path)).get(workload)
+    if ent is None:
+        return None
+    src = os.path.join(ROOT, ent["source"])
+    if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest() != ent["source_sha256"]:
+        return None
+    return ent["dram_bytes_read"] + ent["dram_bytes_write"]
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -497,7 +513,7 @@ def main():
             "e2e": {"value": w.B * world / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                         "frac": achieved / peak, "traffic": None,
+                         "frac": achieved / peak, "traffic": captured_traffic(args.workload),
                          "kernel": "mkv_decode_attention (one fused split-KV decode kernel), one layer",
                          "peak_kind": peak_kind, "frac_of_8000": achieved / 8000.0,
                          "alg_bytes_per_launch": alg_bytes, "context_at_measure": T_now,
