@@ -104,7 +104,7 @@ typedef struct {
  *         pos int32 [B][Hkv][T_cap] (position held by each slot, -1 = empty);
  *         acc fp32 [B][Hkv][T_cap] accumulated attention score;
  *         slot int32 [B][Hkv] the slot the next append writes.
- *  ROCKET: kmin, kmax fp16 [B][Hkv][D][T_cap/page_size] per-page per-dim key
+ *  ROCKET: kmin, kmax fp16 [B][Hkv][D][T_cap/page_size] (16-byte aligned) per-page per-dim key
  *         min/max (dim-major), valid for every completed page.
  *  KVQUANT (keys stored before rotation; Section 2.1, KVQuant paragraph):
  *         k_codes, v_codes uint8 [B][Hkv][T_cap][D*bits/8]: per token, the

@@ -193,6 +193,8 @@ mkv_status check_cache(const mkv_config* c, const mkv_cache* k) {
       MKV_REQUIRE(k->k && k->v && k->kmin && k->kmax, MKV_ERR_INVALID_ARG,
                   "ROCKET cache needs k, v, kmin, kmax");
       MKV_REQUIRE(k->T_cap % kPage == 0, MKV_ERR_INVALID_ARG, "ROCKET T_cap must be a multiple of 16");
+      MKV_REQUIRE(((uintptr_t)k->kmin & 15) == 0 && ((uintptr_t)k->kmax & 15) == 0, MKV_ERR_INVALID_ARG,
+                  "ROCKET kmin/kmax must be 16-byte aligned");
       break;
     case MKV_KVQUANT:
       MKV_REQUIRE(k->k_codes && k->v_codes && k->v_params && k->k_out_off && k->k_out &&

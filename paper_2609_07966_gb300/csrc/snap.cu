@@ -19,6 +19,9 @@ namespace mkv {
 namespace {
 
 constexpr int kSelThreads = 1024;
+constexpr int kSelPages = 256;          // page selection: pages whose bounds are prefetched for every dim
+constexpr int kSelRow = kSelPages + 8;  // halves per prefetched row (room for the 16-byte alignment offset)
+constexpr int kSelChunks = kSelRow / 8; // 16-byte copies per prefetched row
 
 __device__ __forceinline__ float pooled_at(const float* s, int64_t n, int64_t j, int r) {
   float m = -INFINITY;
@@ -94,22 +97,49 @@ __global__ void page_meta_kernel(const __half* __restrict__ k, int64_t T_cap, in
 }
 
 // One CTA per (batch, kv-head): dims, page scores, top-k pages.
+// Page selection (RocketKV stage 2).  With max(q kmin, q kmax) = q kmax for q >= 0 and q kmin
+// otherwise (kmin <= kmax), a page's score over the selected dims t is
+//   sum_t (kmax_t P_t + kmin_t N_t),  P_t = sum_h max(q_h,t, 0),  N_t = sum_h min(q_h,t, 0).
+// Up to kSelPages candidate pages (the common case) the bounds of every dim are prefetched into
+// shared memory while the dims are being chosen; larger caches stage the chosen dims' bounds
+// 256 pages at a time.
 __global__ void __launch_bounds__(kSelThreads) rocket_select_kernel(const __half* __restrict__ q, const __half* __restrict__ kmin,
                                                                     const __half* __restrict__ kmax,
                                                                     const int32_t* __restrict__ T_len, int Hkv, int G, int D,
                                                                     int64_t T_cap, int kp, int rd, int32_t* __restrict__ out) {
-  extern __shared__ float sm[];
+  extern __shared__ __align__(16) float sm[];
+  const int64_t npc = T_cap / kPage;
   float* qs = sm;                       // [G][D]
   float* ssc = qs + G * D;              // [npc] page scores
+  float* part = ssc + ((npc + 3) & ~3ll);                     // [4][kSelPages] partial scores
+  __half* bmn = reinterpret_cast<__half*>(part + 4 * kSelPages);   // fast path: [D][kSelRow]
+  __half* bmx = bmn + D * kSelRow;
   __shared__ int hist[256];
   __shared__ int warp_sums[32];
   __shared__ int dims[128];
-  __shared__ float a_dim[128];
+  __shared__ __align__(16) float a_dim[128];
+  __shared__ float pn[2][128];          // P_t, N_t of the selected dims
   const int64_t bh = blockIdx.x;
   const int b = (int)(bh / Hkv), kvh = (int)(bh % Hkv);
-  const int64_t npc = T_cap / kPage;
   const int n = (int)min((int64_t)T_len[b], T_cap);
   const int ns = n > 0 ? (n - 1) / kPage : 0;
+  const bool fast = ns <= kSelPages;
+  if (fast && ns > 0) {
+    // every dim's bounds of pages [0, ns): 16-byte copies from the row start rounded down to
+    // 16 bytes (the first copy may begin in the previous row), the last one cut at the row end
+    for (int e = threadIdx.x; e < 2 * D * kSelChunks; e += blockDim.x) {
+      const int which = e / (D * kSelChunks), rem = e % (D * kSelChunks);
+      const int dim = rem / kSelChunks, ch = rem % kSelChunks;
+      const int64_t start = (bh * D + dim) * npc;           // first half of the row
+      const int64_t h0 = (start & ~7ll) + ch * 8;
+      const int64_t end = start + ns;
+      if (h0 < end) {
+        const int bytes = (int)min((int64_t)16, (end - h0) * 2);
+        cp_async16((which ? bmx : bmn) + dim * kSelRow + ch * 8, (which ? kmax : kmin) + h0, bytes);
+      }
+    }
+    cp_async_commit();
+  }
   for (int e = threadIdx.x; e < G * D; e += blockDim.x) qs[e] = __half2float(q[((int64_t)b * Hkv * G + (int64_t)kvh * G) * D + e]);
   __syncthreads();
   if (threadIdx.x < D) {
@@ -119,40 +149,80 @@ __global__ void __launch_bounds__(kSelThreads) rocket_select_kernel(const __half
   }
   __syncthreads();
   if (threadIdx.x < D) {
-    const uint64_t mine = rank_key(a_dim[threadIdx.x], (uint32_t)threadIdx.x);
+    // rank under (sum |q| desc, dim asc): four dims per shared-memory read, unrolled so the
+    // reads overlap
+    const int i = threadIdx.x;
+    const float ai = a_dim[i];
     int rank = 0;
-    for (int j = 0; j < D; ++j) rank += rank_key(a_dim[j], (uint32_t)j) > mine ? 1 : 0;
-    if (rank < rd) dims[rank] = threadIdx.x;
+#pragma unroll 4
+    for (int j = 0; j < D; j += 4) {
+      const float4 v = *reinterpret_cast<const float4*>(a_dim + j);
+      rank += (v.x > ai || (v.x == ai && j < i)) + (v.y > ai || (v.y == ai && j + 1 < i)) +
+              (v.z > ai || (v.z == ai && j + 2 < i)) + (v.w > ai || (v.w == ai && j + 3 < i));
+    }
+    if (rank < rd) dims[rank] = i;
   }
   __syncthreads();
-  // page scores, 256 pages at a time: the selected dims' min/max rows are staged with
-  // coalesced loads (dim-major layout), then each thread scores one page from shared memory
-  __half* bmin = reinterpret_cast<__half*>(ssc + npc);          // [rd][256]
-  __half* bmax = bmin + rd * 256;
-  for (int p0 = 0; p0 < ns; p0 += 256) {
-    const int np = min(256, ns - p0);
-    for (int e = threadIdx.x; e < rd * 256; e += blockDim.x) {
-      const int t = e / 256, pp = e % 256;
-      if (pp < np) {
-        const int64_t src = (bh * D + dims[t]) * npc + p0 + pp;
-        bmin[e] = kmin[src];
-        bmax[e] = kmax[src];
-      }
+  if (threadIdx.x < rd) {
+    const int d = dims[threadIdx.x];
+    float P = 0.f, N = 0.f;
+    for (int h = 0; h < G; ++h) {
+      const float v = qs[h * D + d];
+      P += fmaxf(v, 0.f);
+      N += fminf(v, 0.f);
     }
+    pn[0][threadIdx.x] = P;
+    pn[1][threadIdx.x] = N;
+  }
+  if (fast) {
+    cp_async_wait<0>();
     __syncthreads();
-    if (threadIdx.x < np) {
-      float sc = 0.f;
-      for (int h = 0; h < G; ++h) {
-        for (int t = 0; t < rd; ++t) {
-          const float qv = qs[h * D + dims[t]];
-          const float lo = __half2float(bmin[t * 256 + threadIdx.x]) * qv;
-          const float hi = __half2float(bmax[t * 256 + threadIdx.x]) * qv;
-          sc += fmaxf(lo, hi);
+    // thread (page p, slice sl) sums the dims t = sl, sl + 4, ...; the four slices are added after
+    const int p = threadIdx.x % kSelPages, sl = threadIdx.x / kSelPages;
+    if (sl < 4) {
+      float acc = 0.f;
+      if (p < ns) {
+        for (int t = sl; t < rd; t += 4) {
+          const int d = dims[t];
+          const int off = (int)(((bh * D + d) * npc) & 7);
+          const int i = d * kSelRow + off + p;
+          acc += __half2float(bmx[i]) * pn[0][t] + __half2float(bmn[i]) * pn[1][t];
         }
       }
-      ssc[p0 + threadIdx.x] = sc;
+      part[sl * kSelPages + p] = acc;
     }
     __syncthreads();
+    if (threadIdx.x < ns)
+      ssc[threadIdx.x] = (part[threadIdx.x] + part[kSelPages + threadIdx.x]) +
+                         (part[2 * kSelPages + threadIdx.x] + part[3 * kSelPages + threadIdx.x]);
+    else if (threadIdx.x < ((ns + 3) & ~3))
+      ssc[threadIdx.x] = -INFINITY;       // pads the last group of four; never ranks ahead
+    __syncthreads();
+  } else {
+    __syncthreads();
+    // the selected dims' min/max rows staged 256 pages at a time with coalesced loads (dim-major
+    // layout), then each thread scores one page from shared memory
+    __half* smn = bmn;                                          // [rd][256]
+    __half* smx = smn + rd * 256;
+    for (int p0 = 0; p0 < ns; p0 += 256) {
+      const int np = min(256, ns - p0);
+      for (int e = threadIdx.x; e < rd * 256; e += blockDim.x) {
+        const int t = e / 256, pp = e % 256;
+        if (pp < np) {
+          const int64_t src = (bh * D + dims[t]) * npc + p0 + pp;
+          smn[e] = kmin[src];
+          smx[e] = kmax[src];
+        }
+      }
+      __syncthreads();
+      if (threadIdx.x < np) {
+        float sc = 0.f;
+        for (int t = 0; t < rd; ++t)
+          sc += __half2float(smx[t * 256 + threadIdx.x]) * pn[0][t] + __half2float(smn[t * 256 + threadIdx.x]) * pn[1][t];
+        ssc[p0 + threadIdx.x] = sc;
+      }
+      __syncthreads();
+    }
   }
   const int k = min(kp, ns);
   int base = 0;
@@ -164,9 +234,18 @@ __global__ void __launch_bounds__(kSelThreads) rocket_select_kernel(const __half
     if (i < ns && k > 0) {
       const float si = ssc[i];
       int rank = 0;
-      for (int j = 0; j < ns; ++j) {
-        const float sj = ssc[j];
-        rank += (sj > si || (sj == si && j < i)) ? 1 : 0;
+      if (fast) {                         // scores padded to a multiple of four with -inf
+#pragma unroll 4
+        for (int j = 0; j < ns; j += 4) {
+          const float4 v = *reinterpret_cast<const float4*>(ssc + j);
+          rank += (v.x > si || (v.x == si && j < i)) + (v.y > si || (v.y == si && j + 1 < i)) +
+                  (v.z > si || (v.z == si && j + 2 < i)) + (v.w > si || (v.w == si && j + 3 < i));
+        }
+      } else {
+        for (int j = 0; j < ns; ++j) {
+          const float sj = ssc[j];
+          rank += (sj > si || (sj == si && j < i)) ? 1 : 0;
+        }
       }
       flag = rank < k;
     }
@@ -219,7 +298,9 @@ cudaError_t launch_snap_keep(const mkv_config& c, const void* full_k, const void
 cudaError_t launch_rocket_select(const mkv_config& c, const void* q, const mkv_cache& cache, int32_t* page_idx,
                                  cudaStream_t st) {
   const int G = c.Hq / c.Hkv;
-  const size_t smem = ((size_t)G * c.D + cache.T_cap / kPage) * sizeof(float) + 2 * (size_t)c.topq_dims * 256 * 2;
+  const int64_t npc = cache.T_cap / kPage;
+  const size_t smem = ((size_t)G * c.D + ((npc + 3) & ~3ll) + 4 * kSelPages) * sizeof(float) +
+                      std::max<size_t>(2 * (size_t)c.D * kSelRow * 2, 2 * (size_t)c.topq_dims * 256 * 2);
   cudaError_t e = cudaFuncSetAttribute(rocket_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   rocket_select_kernel<<<c.B * c.Hkv, kSelThreads, smem, st>>>(
