@@ -193,18 +193,18 @@ class Runner:
         cache, qp = self.layers[l]
         q = self.q[l] if q is None else q
         out = self.out[l] if out is None else out
-        pidx = self.pidx[l].data_ptr() if self.method == "rocket" else 0
-        mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, qp.c if qp else None, pidx, out.data_ptr(),
+        if self.method == "rocket":           # page choice + sparse attention in one launch
+            mkv.mkv_rocket_decode(self.cfg, q.data_ptr(), cache.c, 0, out.data_ptr())
+            return
+        mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, qp.c if qp else None, 0, out.data_ptr(),
                                  self.ws.data_ptr(), self.nws)
 
     def layer_step(self, l, q=None, kn=None, vn=None, out=None):
-        """One layer of one decode step: append the token, (select pages,) attend, (update scores)."""
+        """One layer of one decode step: append the token, attend (RocketKV: choose pages and attend),
+        (update scores)."""
         mkv = self.mkv
         cache, _ = self.layers[l]
         self.append(l, kn, vn)
-        if self.method == "rocket":
-            mkv.mkv_rocket_select(self.cfg, (self.q[l] if q is None else q).data_ptr(), cache.c,
-                                  self.pidx[l].data_ptr())
         self.decode(l, q, out)
         if self.method == "h2o":
             mkv.mkv_h2o_update(self.cfg, cache.c, self.ws.data_ptr(), self.nws)
@@ -233,9 +233,9 @@ class Runner:
             self.step()
 
     def launches_per_step(self):
-        # per layer: append (KVQuant: quantize + length advance), (page select), decode,
-        # (score update)
-        per = {"fp16": 2, "kvquant": 3, "h2o": 3, "rocket": 3}[self.method]
+        # per layer: append (KVQuant: quantize + length advance), decode (RocketKV: page choice
+        # and attention fused), (H2O: score update)
+        per = {"fp16": 2, "kvquant": 3, "h2o": 3, "rocket": 2}[self.method]
         return per * self.w.L
 
     def decode_bytes(self):
@@ -256,8 +256,10 @@ class Runner:
             # K and V rows, the slot's position (mask) and the G logits written for the update
             return units * slots * (w.D * 2 * 2 + 4 + 4 * w.G), int(cache.t["pos"][0, 0].ge(0).sum())
         n = T
-        tail = n - 16 * ((n - 1) // 16)
-        return units * ((w.topk_pages * 16 + tail) * w.D * 2 * 2 + 4 * w.topk_pages), n
+        ns = (n - 1) // 16
+        tail = n - 16 * ns
+        # the attended pages' K and V rows, and every dim's min/max of every candidate page
+        return units * ((min(w.topk_pages, ns) * 16 + tail) * w.D * 2 * 2 + ns * w.D * 2 * 2), n
 
 
 def time_steps(runner, steps, warmup):

@@ -315,6 +315,20 @@ mkv_status mkv_snap_compress(const mkv_config* cfg, const void* q_window, const 
 mkv_status mkv_rocket_select(const mkv_config* cfg, const void* q, const mkv_cache* cache,
                              int32_t* page_idx_out, void* stream);
 
+/* RocketKV decode step in one launch: the page choice of mkv_rocket_select
+ * and the sparse exact attention of mkv_decode_attention over the chosen
+ * pages plus the newest token's page (Section 2.1, RocketKV paragraph, stage
+ * 2).  One cluster of 8 CTAs per (batch, kv-head) exchanges page scores and
+ * attention partials through distributed shared memory, so no workspace is
+ * needed.  q fp16 [B][Hq][D]; out fp16 [B][Hq][D]; page_idx_out (optional,
+ * NULL to skip) int32 [B][Hkv][topk_pages] as mkv_rocket_select writes it.
+ * The page scores are the same sums in another fp32 order, so a near-tie
+ * may pick another page than mkv_rocket_select.  MKV_ERR_UNSUPPORTED when
+ * T_cap is too long for the step's shared memory (about 32K slots at D=128);
+ * use the two calls then. */
+mkv_status mkv_rocket_decode(const mkv_config* cfg, const void* q, const mkv_cache* cache,
+                             int32_t* page_idx_out, void* out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

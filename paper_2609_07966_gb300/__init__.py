@@ -79,6 +79,7 @@ _SIGS = {
     "mkv_h2o_update": [_CFG, _CACHE, _P, ctypes.c_size_t, _P],
     "mkv_snap_compress": [_CFG, _P, _P, _P, ctypes.c_int64, _CACHE, _P, _P, ctypes.c_size_t, _P],
     "mkv_rocket_select": [_CFG, _P, _CACHE, _P, _P],
+    "mkv_rocket_decode": [_CFG, _P, _CACHE, _P, _P, _P],
     "mkv_decode_attention_noalloc": [_CFG, _P, _CACHE, _P, _P],
 }
 
@@ -210,6 +211,11 @@ def mkv_snap_compress(cfg, q_window: int, full_k: int, full_v: int, T: int, cach
 
 def mkv_rocket_select(cfg, q: int, cache: mkv_cache, page_idx_out: int, stream=None):
     _call("mkv_rocket_select", ctypes.byref(cfg), q, ctypes.byref(cache), page_idx_out, _stream(stream))
+
+
+def mkv_rocket_decode(cfg, q: int, cache: mkv_cache, page_idx_out, out: int, stream=None):
+    _call("mkv_rocket_decode", ctypes.byref(cfg), q, ctypes.byref(cache), page_idx_out or None, out,
+          _stream(stream))
 
 
 def n_value_outliers(D: int, frac: float) -> int:

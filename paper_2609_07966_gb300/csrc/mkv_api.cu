@@ -440,4 +440,17 @@ mkv_status mkv_rocket_select(const mkv_config* cfg, const void* q, const mkv_cac
   return MKV_OK;
 }
 
+mkv_status mkv_rocket_decode(const mkv_config* cfg, const void* q, const mkv_cache* cache, int32_t* page_idx_out,
+                             void* out, void* stream) {
+  MKV_TRY(check_config(cfg));
+  MKV_REQUIRE(cfg->method == MKV_ROCKET, MKV_ERR_INVALID_ARG, "rocket_decode is for ROCKET");
+  MKV_TRY(check_cache(cfg, cache));
+  MKV_REQUIRE(q && out, MKV_ERR_INVALID_ARG, "q/out NULL");
+  MKV_REQUIRE(rocket_fused_smem(*cfg, cache->T_cap) <= 227 * 1024, MKV_ERR_UNSUPPORTED,
+              "T_cap = %lld is too long for the fused step; use mkv_rocket_select + mkv_decode_attention",
+              (long long)cache->T_cap);
+  MKV_CUDA(launch_rocket_fused(*cfg, q, *cache, page_idx_out, out, as_stream(stream)));
+  return MKV_OK;
+}
+
 }  // extern "C"

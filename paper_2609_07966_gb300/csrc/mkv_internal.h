@@ -97,6 +97,10 @@ cudaError_t launch_snap_keep(const mkv_config& c, const void* full_k, const void
                              cudaStream_t st);
 cudaError_t launch_rocket_select(const mkv_config& c, const void* q, const mkv_cache& cache,
                                  int32_t* page_idx, cudaStream_t st);
+// Fused RocketKV step (page choice + sparse attention, one cluster per (batch, kv-head)).
+size_t rocket_fused_smem(const mkv_config& c, int64_t T_cap);
+cudaError_t launch_rocket_fused(const mkv_config& c, const void* q, const mkv_cache& cache, int32_t* page_idx,
+                                void* out, cudaStream_t st);
 
 // Host-side argument checks of an FP16 decode call (config, cache, q/out pointers).
 mkv_status check_fp16_decode_args(const mkv_config* cfg, const mkv_cache* cache, const void* q, const void* out);

@@ -101,3 +101,23 @@ def test_pointer_checks_reject_before_launch(L):
     assert st == mkv.MKV_ERR_INVALID_ARG
     st = L.mkv_rope_table(96, 10000.0, 10, 8, None)
     assert st == mkv.MKV_ERR_UNSUPPORTED
+
+
+def test_rocket_fused_step_checks(L):
+    """The fused RocketKV step is ROCKET-only, needs q/out, aligned page bounds, and a cache short
+    enough for its shared memory; every rejection happens on the host."""
+    rc = mkv.config(mkv.MKV_ROCKET, 1, 32, 8, 128, snap_window=32, snap_pool=7, snap_keep=4096, page_size=16,
+                    topk_pages=64, topq_dims=32)
+    cache = mkv.mkv_cache()
+    cache.T_cap, cache.T_len, cache.k, cache.v, cache.kmin, cache.kmax = 4208, 8, 256, 512, 768, 1024
+    st = L.mkv_rocket_decode(ctypes.byref(_cfg()), 64, ctypes.byref(cache), None, 128, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG
+    st = L.mkv_rocket_decode(ctypes.byref(rc), None, ctypes.byref(cache), None, 128, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG
+    cache.kmin = 770                                   # not 16-byte aligned
+    st = L.mkv_rocket_decode(ctypes.byref(rc), 64, ctypes.byref(cache), None, 128, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG and "aligned" in mkv.mkv_last_error()
+    cache.kmin = 768
+    cache.T_cap = 1 << 20                              # 65536 pages: beyond the fused step
+    st = L.mkv_rocket_decode(ctypes.byref(rc), 64, ctypes.byref(cache), None, 128, None)
+    assert st == mkv.MKV_ERR_UNSUPPORTED and "mkv_rocket_select" in mkv.mkv_last_error()

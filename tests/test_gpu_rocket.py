@@ -1,4 +1,6 @@
-"""GPU parity: SnapKV prefill compression, page metadata, page selection and sparse decode."""
+"""GPU parity: SnapKV prefill compression, page metadata, page selection and sparse decode,
+both as two calls (mkv_rocket_select + mkv_decode_attention) and as the fused step
+(mkv_rocket_decode)."""
 import numpy as np
 import pytest
 
@@ -13,7 +15,7 @@ from lockstep import check_topk, tiny_seed
 pytestmark = pytest.mark.gpu
 
 
-def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev, exact, units, tag):
+def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev, exact, units, tag, fused=False):
     """K, V [B,Hkv,T+steps,D]; QW [B,Hq,W,D] window queries; Q [steps,B,Hq,D] (device tensors)."""
     torch = torch_cuda()
     G = Hq // Hkv
@@ -60,9 +62,13 @@ def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev,
         q = Q[s].contiguous()
         out = torch.empty_like(q)
         mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
-        mkv.mkv_rocket_select(cfg, q.data_ptr(), cache.c, page_idx.data_ptr())
-        mkv.mkv_decode_attention(cfg, q.data_ptr(), cache.c, None, page_idx.data_ptr(), out.data_ptr(), ws.data_ptr(),
-                                 nws)
+        if fused:
+            page_idx.fill_(-7)
+            mkv.mkv_rocket_decode(cfg, q.data_ptr(), cache.c, page_idx.data_ptr(), out.data_ptr())
+        else:
+            mkv.mkv_rocket_select(cfg, q.data_ptr(), cache.c, page_idx.data_ptr())
+            mkv.mkv_decode_attention(cfg, q.data_ptr(), cache.c, None, page_idx.data_ptr(), out.data_ptr(),
+                                     ws.data_ptr(), nws)
         got = out.float().cpu().numpy()
         pidx = page_idx.cpu().numpy()
         for (b, h) in units:
@@ -83,7 +89,8 @@ def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev,
     return near
 
 
-def test_tiny_exact():
+@pytest.mark.parametrize("fused", [False, True])
+def test_tiny_exact(fused):
     torch = torch_cuda()
     dev = torch.device("cuda")
     w = synth.tiny()
@@ -92,11 +99,12 @@ def test_tiny_exact():
     QW = to_dev(x["q_prompt"][0, :, :, w.T - w.snap_window:], dev)
     Q = to_dev(x["q"][:, 0], dev)
     near = run_rocket(w.B, w.Hq, w.Hkv, w.D, w.T, w.steps, w.snap_window, w.snap_pool, w.snap_keep, w.topk_pages,
-                      w.topq_dims, K, V, QW, Q, dev, True, [(0, 0), (0, 1)], "tiny")
+                      w.topq_dims, K, V, QW, Q, dev, True, [(0, 0), (0, 1)], "tiny", fused)
     assert near == 0
 
 
-def test_keep_everything_is_full_attention():
+@pytest.mark.parametrize("fused", [False, True])
+def test_keep_everything_is_full_attention(fused):
     """keep >= T and k_p >= pages: every step attends the whole cache."""
     torch = torch_cuda()
     dev = torch.device("cuda")
@@ -107,11 +115,12 @@ def test_keep_everything_is_full_attention():
     QW = rng.standard_normal((B, Hq, 8, D)).astype(np.float16)
     Q = rng.standard_normal((steps, B, Hq, D)).astype(np.float16)
     run_rocket(B, Hq, Hkv, D, T, steps, 8, 7, 160, 64, 16, to_dev(K, dev), to_dev(V, dev), to_dev(QW, dev),
-               to_dev(Q, dev), dev, False, [(0, 0), (1, 1)], "all")
+               to_dev(Q, dev), dev, False, [(0, 0), (1, 1)], "all", fused)
 
 
-@pytest.mark.parametrize("G,D", [(1, 128), (8, 64)])
-def test_shapes_lockstep(G, D):
+@pytest.mark.parametrize("G,D,fused", [(1, 128, False), (8, 64, False), (1, 128, True), (8, 64, True),
+                                       (4, 128, True), (2, 64, True)])
+def test_shapes_lockstep(G, D, fused):
     torch = torch_cuda()
     dev = torch.device("cuda")
     rng = np.random.default_rng(G + D)
@@ -122,10 +131,11 @@ def test_shapes_lockstep(G, D):
     QW = rng.standard_normal((B, Hq, W, D)).astype(np.float16)
     Q = rng.standard_normal((steps, B, Hq, D)).astype(np.float16)
     run_rocket(B, Hq, Hkv, D, T, steps, W, 7, 300, 6, D // 4, to_dev(K, dev), to_dev(V, dev), to_dev(QW, dev),
-               to_dev(Q, dev), dev, False, [(0, 1), (1, 0)], f"G{G}D{D}")
+               to_dev(Q, dev), dev, False, [(0, 1), (1, 0)], f"G{G}D{D}", fused)
 
 
-def test_full_size_lockstep():
+@pytest.mark.parametrize("fused", [False, True])
+def test_full_size_lockstep(fused):
     """B=4, T=32768 -> keep 4096, W=32, pool 7, top-64 pages over top-32 dims: one layer,
     16 steps, two (batch, kv-head) units in lockstep with the oracle."""
     torch = torch_cuda()
@@ -134,5 +144,48 @@ def test_full_size_lockstep():
     x = synth.device_layer_inputs(w, seed=12, layer=0, device=dev, n_tokens=w.T + 16, with_prompt_queries=True)
     QW = x["q_prompt"][:, :, w.T - w.snap_window:].contiguous()
     near = run_rocket(w.B, w.Hq, w.Hkv, w.D, w.T, 16, w.snap_window, w.snap_pool, w.snap_keep, w.topk_pages,
-                      w.topq_dims, x["k"], x["v"], QW, x["q"][:16], dev, False, [(0, 0), (3, 7)], "rocket32k")
+                      w.topq_dims, x["k"], x["v"], QW, x["q"][:16], dev, False, [(0, 0), (3, 7)], "rocket32k", fused)
     print(f"near-ties adopted: {near}")
+
+
+def test_fused_short_contexts():
+    """T_len of 0, 1, 16, 17 and 40 in one batch (no candidate page, one partial page, a full page
+    plus the newest token's page...): the fused step against the oracle, page list -1 padded."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(31)
+    lens = [0, 1, 16, 17, 40]
+    B, Hq, Hkv, D, kp, rd = len(lens), 8, 2, 64, 2, 16
+    G = Hq // Hkv
+    T_cap = 48
+    cfg = mkv.config(mkv.MKV_ROCKET, B, Hq, Hkv, D, snap_window=8, snap_pool=7, snap_keep=64, page_size=16,
+                     topk_pages=kp, topq_dims=rd)
+    cache = caches.alloc_cache(cfg, T_cap, device=dev)
+    K = rng.standard_normal((B, Hkv, T_cap, D)).astype(np.float16)
+    V = rng.standard_normal((B, Hkv, T_cap, D)).astype(np.float16)
+    cache.t["k"].copy_(to_dev(K, dev))
+    cache.t["v"].copy_(to_dev(V, dev))
+    for b in range(B):
+        for h in range(Hkv):
+            npg = T_cap // 16
+            kmin, kmax = rocket.page_minmax(K[b, h], 16, npg)
+            cache.t["kmin"][b, h] = to_dev(kmin.T.astype(np.float16), dev)
+            cache.t["kmax"][b, h] = to_dev(kmax.T.astype(np.float16), dev)
+    cache.t["T_len"].copy_(torch.tensor(lens, dtype=torch.int32))
+    q = to_dev(rng.standard_normal((B, Hq, D)).astype(np.float16), dev)
+    out = torch.full_like(q, float("nan"))
+    page_idx = torch.full((B, Hkv, kp), -7, dtype=torch.int32, device=dev)
+    mkv.mkv_rocket_decode(cfg, q.data_ptr(), cache.c, page_idx.data_ptr(), out.data_ptr())
+    got = out.float().cpu().numpy()
+    pidx = page_idx.cpu().numpy()
+    for b, n in enumerate(lens):
+        for h in range(Hkv):
+            qh = q[b, h * G:(h + 1) * G].cpu().numpy()
+            if n == 0:
+                assert np.all(got[b, h * G:(h + 1) * G] == 0) and np.all(pidx[b, h] == -1)
+                continue
+            sel, _ = rocket.select_pages(qh, K[b, h, :n], n, 16, kp, rd)
+            assert pidx[b, h][pidx[b, h] >= 0].tolist() == sel.tolist()
+            assert np.all(pidx[b, h][len(sel):] == -1)
+            ref, _, _ = rocket.decode(qh, K[b, h, :n], V[b, h, :n], n, 16, kp, rd)
+            assert_close(got[b, h * G:(h + 1) * G], ref, f"n={n} h{h}")
