@@ -121,14 +121,14 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
   const int64_t bh = blockIdx.y;
   const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int n = (int)min((int64_t)a.T_len[b], a.T_cap);
-  const int ns = n > 0 ? (n - 1) / kPage : 0;          // candidate (full) pages
-  const int sp = (ns + kCl - 1) / kCl;                  // pages scored per CTA
-  const int p0 = min(ns, rank * sp), np = min(ns, p0 + sp) - p0;
+  // this CTA's share of the pages, fixed by the capacity so the prefetch need not wait for T_len
+  const int sp = (int)((a.npc + kCl - 1) / kCl);        // pages per CTA
+  const int p0 = min((int)a.npc, rank * sp), npf = min((int)a.npc, p0 + sp) - p0;
 
   // ---- 1. prefetch every dim's bounds of this CTA's pages (16-byte copies from the row start
   // rounded down to 16 bytes, the last one cut at the end of the pages)
-  if (np > 0) {
+  if (npf > 0) {
+    const int np = npf;
     const int nch = (7 + np + 7) / 8;                   // copies per row (covers the offset)
     for (int e = tid; e < 2 * D * nch; e += kRfThreads) {
       const int which = e / (D * nch), rem = e % (D * nch);
@@ -143,6 +143,9 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
     }
   }
   cp_async_commit();
+  const int n = (int)min((int64_t)a.T_len[b], a.T_cap);
+  const int ns = n > 0 ? (n - 1) / kPage : 0;          // candidate (full) pages
+  const int np = max(0, min(ns, p0 + sp) - p0);        // of them, this CTA's
   for (int e = tid; e < G * D; e += kRfThreads)
     qs[e] = __half2float(a.q[((int64_t)b * a.Hq + (int64_t)kvh * G) * D + e]);
   for (int e = tid; e < G * (D / 2); e += kRfThreads)
@@ -353,6 +356,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
   }
   __syncthreads();
   float* cp = reinterpret_cast<float*>(smem + L.cpart);   // CTA 0: [kCl][G][D + 2]
+  const uint32_t cp0 = cluster_addr(cp, 0);
   for (int e = tid; e < G * D; e += kRfThreads) {
     const int row = e / D, d = e % D;
     float M = -INFINITY;
@@ -365,11 +369,11 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
         O += wo[(w * G + row) * D + d] * f;
       }
     }
-    float* slot = cp + (rank * G + row) * (D + 2);
-    st_cluster(cluster_addr(slot + 2 + d, 0), O);
+    const uint32_t slot = cp0 + (uint32_t)((rank * G + row) * (D + 2)) * 4u;
+    st_cluster(slot + (2 + d) * 4u, O);
     if (d == 0) {
-      st_cluster(cluster_addr(slot, 0), M);
-      st_cluster(cluster_addr(slot + 1, 0), Lsum);
+      st_cluster(slot, M);
+      st_cluster(slot + 4u, Lsum);
     }
   }
   cluster_sync();
