@@ -13,6 +13,7 @@
 
 #include "mkv_common.cuh"
 #include "mkv_internal.h"
+#include "mkv_h2o.cuh"
 #include "mkv_select.cuh"
 
 namespace mkv {
@@ -86,84 +87,7 @@ __global__ void __launch_bounds__(1024) h2o_update_kernel(const float* __restric
                                                          int H, int R, const int32_t* __restrict__ T_len,
                                                          int32_t* __restrict__ pos, float* __restrict__ acc,
                                                          int32_t* __restrict__ slot_out) {
-  const int64_t bh = blockIdx.x;
-  const int b = (int)(bh / Hkv), kvh = (int)(bh % Hkv);
-  const int64_t newest = (int64_t)T_len[b] - 1;
-  float m[8], il[8];
-  for (int h = 0; h < G; ++h) {
-    const int64_t hq = (int64_t)b * Hkv * G + (int64_t)kvh * G + h;
-    m[h] = m_tot[hq];
-    il[h] = l_tot[hq] > 0.f ? 1.f / l_tot[hq] : 0.f;
-  }
-  int held = 0;
-  uint64_t best = ~0ull;          // minimum key among candidates -> evicted
-  int best_slot = -1, first_free = INT32_MAX;
-  for (int64_t s = threadIdx.x; s < T_cap; s += blockDim.x) {
-    const int32_t p = pos[bh * T_cap + s];
-    if (p < 0) {
-      first_free = min(first_free, (int)s);
-      continue;
-    }
-    ++held;
-    float add = 0.f;
-    const float* lg = logits + (bh * T_cap + s) * G;
-    if (G == 4) {
-      const float4 x = *reinterpret_cast<const float4*>(lg);
-      add = exp2f(x.x - m[0]) * il[0] + exp2f(x.y - m[1]) * il[1] + exp2f(x.z - m[2]) * il[2] +
-            exp2f(x.w - m[3]) * il[3];
-    } else {
-      for (int h = 0; h < G; ++h) add += exp2f(lg[h] - m[h]) * il[h];
-    }
-    const float a2 = acc[bh * T_cap + s] + add;
-    acc[bh * T_cap + s] = a2;
-    if ((int64_t)p <= newest - R) {
-      const uint64_t key = rank_key(a2, (uint32_t)p);
-      if (key < best) {
-        best = key;
-        best_slot = (int)s;
-      }
-    }
-  }
-  // block reductions: held count, first free slot, min key (with its slot)
-  __shared__ int s_held[32], s_free[32];
-  __shared__ uint64_t s_key[32];
-  __shared__ int s_slot[32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int o = 16; o > 0; o >>= 1) {
-    held += __shfl_xor_sync(0xffffffffu, held, o);
-    first_free = min(first_free, __shfl_xor_sync(0xffffffffu, first_free, o));
-    const uint64_t ok = __shfl_xor_sync(0xffffffffu, best, o);
-    const int os = __shfl_xor_sync(0xffffffffu, best_slot, o);
-    if (ok < best) {
-      best = ok;
-      best_slot = os;
-    }
-  }
-  if (lane == 0) {
-    s_held[warp] = held;
-    s_free[warp] = first_free;
-    s_key[warp] = best;
-    s_slot[warp] = best_slot;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    int hsum = 0, ff = INT32_MAX, bs = -1;
-    uint64_t bk = ~0ull;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
-      hsum += s_held[w];
-      ff = min(ff, s_free[w]);
-      if (s_key[w] < bk) {
-        bk = s_key[w];
-        bs = s_slot[w];
-      }
-    }
-    if (hsum > H + R && bs >= 0) {
-      pos[bh * T_cap + bs] = -1;
-      slot_out[bh] = bs;
-    } else {
-      slot_out[bh] = ff == INT32_MAX ? -1 : ff;
-    }
-  }
+  h2o_update_unit(logits, m_tot, l_tot, Hkv, G, T_cap, H, R, T_len, pos, acc, slot_out, blockIdx.x);
 }
 
 }  // namespace
