@@ -37,8 +37,9 @@ Split decode_split(const mkv_config& c, int64_t T_cap) {
   for (int64_t n = 1; n <= std::min<int64_t>(chunks, 1024); ++n) {
     const int64_t cps = ceil_div(chunks, n);
     if (ceil_div(chunks, cps) != n) continue;      // n is not the split count of any cps
-    // + 2: a CTA's fixed cost (query load, table load, pipeline fill, merge) in chunk units
-    const int64_t cost = ceil_div(units * n, slots) * (cps + 2);
+    // + 6: a CTA's fixed cost (query and table loads, pipeline fill and drain, merge) in chunk
+    // units, fitted to measured split sweeps of the FP16 and KVQuant kernels
+    const int64_t cost = ceil_div(units * n, slots) * (cps + 6);
     if (cost < best_cost) {
       best_cost = cost;
       best_n = n;
