@@ -179,6 +179,36 @@ mkv_status mkv_workspace_size(const mkv_config* cfg, int64_t T_cap, size_t* byte
  * peak-memory figure the paper's selector predicts (Section 2.3).  Host only. */
 mkv_status mkv_cache_bytes(const mkv_config* cfg, int64_t T, size_t* resident, size_t* peak);
 
+/* ------------------------------------------------------------ selector */
+
+/* One candidate configuration for mkv_select_config: its method, its level
+ * of compression within the method (larger = less compressed: KVQuant bits,
+ * H2O budget percent, RocketKV minus its compression ratio), and its
+ * predicted end-to-end latency, peak memory and probability of a correct
+ * answer.  Latency and memory use the units of the budgets they are compared
+ * with. */
+typedef struct {
+  int32_t method;   /* mkv_method */
+  int32_t level;
+  double latency;
+  double memory;
+  double accuracy;
+} mkv_candidate;
+
+/* The configuration choice of MetaKV (Section 2.3), fed by measured or
+ * predicted costs: keep the candidates with latency <= L_max and memory <=
+ * M_max; if FP16 is among them choose it (the first FP16 candidate); else
+ * keep the least compressed candidate of each method (largest level, ties:
+ * lower index) and choose it if it is alone, otherwise the one with the
+ * highest accuracy (ties: lower index).  If no candidate is within both
+ * budgets, choose the smallest violation v_c = latency/L_max +
+ * memory/M_max (ties: higher accuracy, then lower index).  *chosen gets the
+ * index into `cands`, *within_budget 1 or 0 for the fallback.  Host only;
+ * MKV_ERR_INVALID_ARG for n < 1, a budget <= 0, a non-finite or negative
+ * cost, or a method out of range. */
+mkv_status mkv_select_config(const mkv_candidate* cands, int32_t n, double L_max, double M_max,
+                             int32_t* chosen, int32_t* within_budget);
+
 /* ------------------------------------------------------------ utilities */
 
 /* table fp32 [T_max][D/2][2]: (cos, sin) of p * theta^(-2i/D), computed in

@@ -22,6 +22,7 @@ Modules
   snapkv     -- observation-window scores, pooling, keep selection       (O5)
   rocket     -- page min/max, dims, page scores, sparse decode           (O6)
   order      -- the total orders used for every ranking decision        (O7)
+  selector   -- the configuration choice over predicted costs (Section 2.3) (O8)
 
 Parity status: every function is pinned by tests in ``tests/test_oracle_*``
 against closed forms, invariants, brute force or an independent library

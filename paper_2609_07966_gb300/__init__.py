@@ -36,6 +36,11 @@ class mkv_config(ctypes.Structure):
                 ("page_size", ctypes.c_int32), ("topk_pages", ctypes.c_int32), ("topq_dims", ctypes.c_int32)]
 
 
+class mkv_candidate(ctypes.Structure):
+    _fields_ = [("method", ctypes.c_int32), ("level", ctypes.c_int32), ("latency", ctypes.c_double),
+                ("memory", ctypes.c_double), ("accuracy", ctypes.c_double)]
+
+
 class mkv_cache(ctypes.Structure):
     _fields_ = [("T_cap", ctypes.c_int64), ("T_len", ctypes.c_void_p), ("k", ctypes.c_void_p),
                 ("v", ctypes.c_void_p), ("pos", ctypes.c_void_p), ("acc", ctypes.c_void_p),
@@ -80,6 +85,8 @@ _SIGS = {
     "mkv_snap_compress": [_CFG, _P, _P, _P, ctypes.c_int64, _CACHE, _P, _P, ctypes.c_size_t, _P],
     "mkv_rocket_select": [_CFG, _P, _CACHE, _P, _P],
     "mkv_rocket_decode": [_CFG, _P, _CACHE, _P, _P, _P],
+    "mkv_select_config": [ctypes.POINTER(mkv_candidate), ctypes.c_int32, ctypes.c_double, ctypes.c_double,
+                          ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32)],
     "mkv_decode_attention_noalloc": [_CFG, _P, _CACHE, _P, _P],
 }
 
@@ -222,3 +229,13 @@ def n_value_outliers(D: int, frac: float) -> int:
     import ctypes as _ct
     f32 = _ct.c_float(frac).value
     return min(D, int(math.ceil(f32 * D)))
+
+
+def mkv_select_config(cands, L_max: float, M_max: float):
+    """cands: sequence of (method, level, latency, memory, accuracy).  Returns (index, within_budget)."""
+    arr = (mkv_candidate * len(cands))(*[mkv_candidate(int(m), int(lv), float(l), float(mm), float(a))
+                                          for (m, lv, l, mm, a) in cands])
+    chosen, within = ctypes.c_int32(-1), ctypes.c_int32(-1)
+    _call("mkv_select_config", arr, len(cands), float(L_max), float(M_max), ctypes.byref(chosen),
+          ctypes.byref(within))
+    return chosen.value, bool(within.value)
