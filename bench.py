@@ -340,6 +340,24 @@ def time_e2e(runner, steps, warmup):
     return dt, h2d, d2h
 
 
+def slowest_rank_ms(ms: float, dev) -> float:
+    """Step time of the slowest rank: every rank gets the max over ranks (one rank: unchanged).
+    Ranks are independent replicas (each decodes its own batch, no collective on the data path),
+    so the whole-job value is the units of all ranks over this time."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return ms
+    t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_tokens_per_s(batch: int, world: int, ms: float) -> float:
+    """Tokens per second of the whole job: every rank decodes `batch` tokens per step."""
+    return batch * world / (ms * 1e-3)
+
+
 def captured_traffic(workload: str):
     """DRAM bytes (read + write) of one decode launch from the committed ncu capture of this workload,
     or None when there is none or the kernel source changed since it was taken."""
@@ -494,10 +512,8 @@ def main():
     ms = time_steps(runner, args.steps, args.warmup)
     clk = clocks.stop()
     clk["window"] = "sampled every 50 ms from just before the warm-up to the end of the timed steps"
+    ms = slowest_rank_ms(ms, dev)
     if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
         torch.distributed.barrier()
 
     alg_bytes, T_now = runner.decode_bytes()
@@ -505,7 +521,7 @@ def main():
     e2e_s, h2d, d2h = time_e2e(runner, max(1, min(args.steps, 5)), 1)
     peak, peak_kind = peaks()
     achieved = alg_bytes / (dec_ms * 1e-3) / 1e9
-    value = w.B * world / (ms * 1e-3)
+    value = whole_job_tokens_per_s(w.B, world, ms)
     res, pk = runner.mkv.mkv_cache_bytes(runner.cfg, w.T)
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",

@@ -41,15 +41,6 @@ __device__ __forceinline__ void qrow_map(const ScoreArgs& a, int rb, int q, int&
   i = (int64_t)rb * a.rpb + q % a.rpb;
 }
 
-template <int D>
-__device__ __forceinline__ void load_rows_async(uint8_t* tile, const __half* base_of_row0, int64_t stride_rows,
-                                                int nrows_valid, int row_of[64]) {
-  (void)base_of_row0;
-  (void)stride_rows;
-  (void)nrows_valid;
-  (void)row_of;
-}
-
 // ---------------------------------------------------------------- pass 1
 template <int D>
 __global__ void __launch_bounds__(kT) rowstats_kernel(const ScoreArgs a) {
