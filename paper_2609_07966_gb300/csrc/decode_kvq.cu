@@ -22,12 +22,15 @@
 // rotation R(t0) is applied to the query instead:
 // q . R(t0 + d) k = (R(t0)^T q) . (R(d) k)) and written as fp16 hi plus the
 // negated fp16 remainder, so the tensor-core product keeps fp32 accuracy.
-// Dense-and-sparse outliers are restored by the consumers before the
-// attention, one thread per outlier entry (key entries are read one chunk
-// ahead): a value outlier overwrites its tile entry; for a key outlier the
-// pair before the rotation is recovered from the tile, the fp16 value(s) put
-// in, and the pair rotated and split again.  Consumers: QK^T = q_hi k_hi - q_hi nk_lo + q_lo k_hi, online
-// softmax and PV on 16-token slabs.  Tile columns hold pair i at columns
+// Dense-and-sparse outliers are restored by the producers as well.  A value
+// outlier overwrites its tile entry (by the thread that wrote the dense value).
+// A key outlier enters the score linearly: with k = k_dense + (x - k_dense[c]) e_c,
+// q . R(t) k = q . R(t) k_dense + (x - k_dense[c]) (R(t)^T q)[c], so one thread
+// per outlier entry adds that fp32 term for every query head of the group to a
+// per-chunk correction table, and the consumers add it to the tensor-core
+// scores.  Consumers: S^T (tokens x heads) = K_hi q_hi - K_nlo q_hi + K_hi q_lo
+// on 16-token slabs, online softmax, then O^T (dims x heads) += V^T P^T with P^T
+// transposed in registers (movmatrix).  Tile columns hold pair i at columns
 // (2i, 2i+1) = channels (i, i + D/2); the output is un-permuted at the end.
 #include <math.h>
 
@@ -44,12 +47,11 @@ constexpr int kConsWarps = 4;                          // attention on chunk c-1
 constexpr int kProdThr = kProdWarps * 32;
 constexpr int kThr = (kProdWarps + kConsWarps) * 32;
 constexpr int kGroups = 8;                             // pair groups of a token row
-constexpr int kEntCap = kProdThr;                      // key-outlier entries of a chunk kept in smem
+constexpr int kEnt = 256;                              // key-outlier entries of a chunk staged
 // named barriers (0 is __syncthreads)
 constexpr int kBarProd = 1;                            // producers only
 constexpr int kBarFull = 2;                            // + buffer: tiles of a chunk are ready
 constexpr int kBarEmpty = 4;                           // + buffer: tiles may be overwritten
-constexpr int kBarCons = 6;                            // consumers only
 // Register split: the kernel is compiled for (and launched with) kRegLaunch registers a
 // thread; producer warpgroups give registers back, the consumer warpgroup takes them.
 constexpr int kRegLaunch = 96, kRegProd = 88, kRegCons = 128;
@@ -95,7 +97,10 @@ struct KvqLayout {
   static constexpr int NP = D / 2;
   static constexpr int K = 1 << BITS;
   static constexpr int ROWW = D * BITS / 32;                 // packed words per token row
-  static constexpr int SROWW = ROWW + 1;                     // staged row stride (odd: conflict-free)
+  // Rows of whole 16-byte pieces are staged by 16-byte copies that bypass L1, at a stride of
+  // 4 mod 8 words (at most 4 rows share a bank); other rows by 4-byte copies at an odd stride.
+  static constexpr bool CG = ROWW % 4 == 0;
+  static constexpr int SROWW = CG ? ((ROWW + 4) % 8 == 4 ? ROWW + 4 : ROWW + 8) : ROWW + 1;
   static constexpr int QP = NP / kGroups;                    // pairs per producer thread
   static constexpr int NWG = (QP * 2 * BITS + 31) / 32;      // words holding one group's codes
   static constexpr int TILE = kChunk * D * 2;                // fp16 tile bytes
@@ -108,7 +113,9 @@ struct KvqLayout {
   static constexpr int S_VP = S_VC + ((kChunk * SROWW * 4 + 15) / 16) * 16;   // [64] float2
   static constexpr int S_KO = S_VP + kChunk * 8;             // [65] int32 key-outlier CSR offsets
   static constexpr int S_VO = S_KO + 68 * 4;                 // [NVS][64] u32 value outliers
-  static constexpr int STAGE = S_VO + NVS * kChunk * 4;
+  static constexpr int S_ENT = S_VO + NVS * kChunk * 4;      // [kEnt] u32 first key-outlier entries
+  static constexpr int S_RT = S_ENT + kEnt * 4;          // [NP] float2 rotation of the chunk start
+  static constexpr int STAGE = S_RT + NP * 8;
   // one tile buffer: keys (hi, negated lo), values, and the rotated query
   static constexpr int B_KHI = 0;
   static constexpr int B_KLO = B_KHI + TILE;
@@ -116,16 +123,17 @@ struct KvqLayout {
   static constexpr int B_QH = B_VT + TILE;                   // [8][QROW] q_hi pairs, fragment order
   static constexpr int B_QN = B_QH + 8 * QROW * 4;           // -q_hi
   static constexpr int B_QL = B_QN + 8 * QROW * 4;           // q_lo
-  static constexpr int B_ENT = B_QL + 8 * QROW * 4;          // [kEntCap] u32 key-outlier entries
-  static constexpr int B_KO = B_ENT + kEntCap * 4;           // [68] int32 their CSR offsets
-  static constexpr int B_OWN = B_KO + 68 * 4;                // [kEntCap] u8 token of each entry
-  static constexpr int B_VO = B_OWN + kEntCap;               // [NVS][64] u32 value outliers
+  static constexpr int B_ENT = B_QL + 8 * QROW * 4;          // [kEnt] u32 first key-outlier entries
+  static constexpr int B_OWN = B_ENT + kEnt * 4;             // [kEnt] u8 token of each
+  static constexpr int B_KO = B_OWN + kEnt;                  // [68] int32 CSR offsets of the chunk
+  static constexpr int B_VO = B_KO + 68 * 4;                 // [NVS][64] u32 value outliers
   static constexpr int BUF = B_VO + NVS * kChunk * 4;
   // CTA layout
   static constexpr int DTAB = 0;                             // [NP][64] float2 rotation by delta
   static constexpr int KDQ = DTAB + NP * kChunk * 8;         // [D][K] float
   static constexpr int VTB = KDQ + D * K * 4;                // [D][K] float
-  static constexpr int STG = VTB + D * K * 4;                // [NS][STAGE]
+  static constexpr int QS = VTB + D * K * 4;                 // [8][D] f32 query (as given, rotated)
+  static constexpr int STG = QS + 8 * D * 4;                 // [NS][STAGE]
   static constexpr int BUFS = STG + NS * STAGE;              // [2][BUF]
   static constexpr int BYTES = BUFS + 2 * BUF;
 };
@@ -183,6 +191,9 @@ __device__ __forceinline__ void split_hi_nlo(float a, float b, uint32_t& hi, uin
 __device__ __forceinline__ void cp_async4s(uint32_t saddr, const void* gmem, int src_bytes) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(saddr), "l"(gmem), "r"(src_bytes));
 }
+__device__ __forceinline__ void cp_async16s(uint32_t saddr, const void* gmem, int src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(saddr), "l"(gmem), "r"(src_bytes));
+}
 __device__ __forceinline__ void cp_async8s(uint32_t saddr, const void* gmem, int src_bytes) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 8, %2;\n" ::"r"(saddr), "l"(gmem), "r"(src_bytes));
 }
@@ -191,6 +202,14 @@ __device__ __forceinline__ void cp_async8s(uint32_t saddr, const void* gmem, int
 template <int D>
 __device__ __forceinline__ int tile_off(int row, int ch) {
   return row * D * 2 + ((ch ^ (row & 7)) << 4);
+}
+
+// S^T fragment of P transposed in registers: an 8x8 b16 matrix held as the rows of an mma
+// accumulator becomes the column-major operand of the next mma
+__device__ __forceinline__ uint32_t movm_trans(uint32_t x) {
+  uint32_t y;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;\n" : "=r"(y) : "r"(x));
+  return y;
 }
 
 template <int D, int BITS>
@@ -203,6 +222,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   float2* dtab = reinterpret_cast<float2*>(smem + Lay::DTAB);
   float* kdq = reinterpret_cast<float*>(smem + Lay::KDQ);
   float* vtb = reinterpret_cast<float*>(smem + Lay::VTB);
+  float* qs = reinterpret_cast<float*>(smem + Lay::QS);
   uint8_t* stg = smem + Lay::STG;
   uint8_t* bufs = smem + Lay::BUFS;
 
@@ -217,7 +237,8 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   if (v_end > n_len) v_end = n_len;
   const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
 
-  // CTA-resident tables: rotations by delta in [0, 64), dequant tables of this kv-head
+  // CTA-resident tables: rotations by delta in [0, 64), dequant tables of this kv-head, the
+  // group's queries in fp32
   for (int e = tid; e < NP * kChunk; e += kThr) {  // coalesced read of rope rows 0..63, transposed
     const int d = e / NP, i = e % NP;
     dtab[i * kChunk + d] = a.rope[(int64_t)min((int64_t)d, a.rope_len - 1) * NP + i];
@@ -226,6 +247,8 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     kdq[e] = a.k_dq[(int64_t)kvh * D * K + e];
     vtb[e] = __half2float(__ushort_as_half(a.v_tbl[(int64_t)kvh * D * K + e]));
   }
+  for (int e = tid; e < a.G * D; e += kThr)
+    qs[e] = __half2float(a.q[((int64_t)b * a.Hq + (int64_t)kvh * a.G) * D + e]);
   __syncthreads();
 
   // the four attention warps' (m, l, o) per query row, merged after both roles finish
@@ -255,16 +278,33 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       const int lim = (int)min((int64_t)kChunk, (int64_t)n_len - c0);
       const uint32_t* kc = kc_base + c0 * ROWW;
       const uint32_t* vc = vc_base + c0 * ROWW;
+      if constexpr (Lay::CG) {
+        constexpr int PR = ROWW / 4;                         // 16-byte pieces per row
+        constexpr int NPC = kChunk * PR;                     // pieces per chunk (keys or values)
 #pragma unroll
-      for (int k = 0; k < NIT; ++k) {                        // row-contiguous: coalesced
-        const int e = ptid + k * kProdThr;
-        if (NCW % kProdThr == 0 || e < NCW) {
-          const int row = e / ROWW, w = e % ROWW;
-          const bool ok = row < lim;
-          const int src = ok ? e : 0;
-          const uint32_t d = dst + (row * SROWW + w) * 4;
-          cp_async4s(d + Lay::S_KC, kc + src, ok ? 4 : 0);
-          cp_async4s(d + Lay::S_VC, vc + src, ok ? 4 : 0);
+        for (int k = 0; k < (2 * NPC + kProdThr - 1) / kProdThr; ++k) {
+          const int e = ptid + k * kProdThr;                 // key pieces, then value pieces
+          if ((2 * NPC) % kProdThr == 0 || e < 2 * NPC) {
+            const bool vals = e >= NPC;
+            const int pe = vals ? e - NPC : e;
+            const int row = pe / PR, q = pe % PR;
+            const bool ok = row < lim;
+            cp_async16s(dst + (vals ? Lay::S_VC : Lay::S_KC) + (row * SROWW + q * 4) * 4,
+                        (vals ? vc : kc) + (ok ? pe * 4 : 0), ok ? 16 : 0);
+          }
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < NIT; ++k) {                      // row-contiguous: coalesced
+          const int e = ptid + k * kProdThr;
+          if (NCW % kProdThr == 0 || e < NCW) {
+            const int row = e / ROWW, w = e % ROWW;
+            const bool ok = row < lim;
+            const int src = ok ? e : 0;
+            const uint32_t d = dst + (row * SROWW + w) * 4;
+            cp_async4s(d + Lay::S_KC, kc + src, ok ? 4 : 0);
+            cp_async4s(d + Lay::S_VC, vc + src, ok ? 4 : 0);
+          }
         }
       }
       if (ptid < kChunk) {                                          // value (lo, scale)
@@ -273,6 +313,9 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       } else if (ptid <= 2 * kChunk) {                              // key-outlier offsets c0 .. c0+64
         const int i = ptid - kChunk;
         cp_async4s(dst + Lay::S_KO + i * 4, a.k_out_off + off_base + c0 + min(i, lim), 4);
+      } else if (ptid >= kProdThr - NP) {                            // rotation of the chunk start
+        const int i = ptid - (kProdThr - NP);
+        cp_async8s(dst + Lay::S_RT + i * 8, a.rope + min(c0, a.rope_len - 1) * NP + i, 8);
       } else if (stage_vout && ptid >= 3 * kChunk && ptid < (3 + Lay::NVS) * kChunk) {
         const int k = (ptid - 3 * kChunk) / kChunk, row = ptid % kChunk;
         if (k < a.n_v) {
@@ -291,44 +334,48 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     const int nq = a.G * NP;
     const int qg = ptid / NP, qi = ptid % NP;
     float qx = 0.f, qy = 0.f;
-    float2 qcs = make_float2(1.f, 0.f);
     if (ptid < nq) {
-      const __half* qr = a.q + ((int64_t)b * a.Hq + (int64_t)kvh * a.G + qg) * D;
-      qx = __half2float(qr[qi]);
-      qy = __half2float(qr[qi + NP]);
-      if (nchunks > 0) qcs = a.rope[min(v_begin, a.rope_len - 1) * NP + qi];
+      qx = qs[qg * D + qi];
+      qy = qs[qg * D + qi + NP];
     }
     const int qpos = qg * QROW + (qi / 8) * 8 + (qi % 4) * 2 + ((qi % 8) / 4);
 
-    // key-outlier entries are fetched one chunk ahead, one per thread
-    uint32_t kent = 0u;
-    if (nchunks > 0) {
-      const int64_t e0 = __ldg(a.k_out_off + off_base + min(v_begin, (int64_t)n_len));
-      const int64_t e1 = min((int64_t)__ldg(a.k_out_off + off_base + min(v_begin + kChunk, (int64_t)n_len)),
-                             a.k_out_cap);
-      if (e0 + ptid < e1) kent = __ldg(gents + e0 + ptid);
-    }
-
+    // The first kEnt key-outlier entries of a chunk are staged by cp.async one chunk ahead
+    // (once the chunk's offsets have landed), one per thread, in a commit group of their own
+    // ahead of that iteration's chunk copies; those of chunk 0 with chunk 0.
+    auto load_entries = [&](int stage, int64_t e0, int64_t e1) {
+      const int64_t e = e0 + ptid;
+      const bool ok = e < e1;
+      if (ptid < kEnt)
+        cp_async4s(stg_s + stage * Lay::STAGE + Lay::S_ENT + ptid * 4, gents + (ok ? e : 0), ok ? 4 : 0);
+    };
 #pragma unroll
     for (int s = 0; s < NS - 1; ++s) {
-      if (s < nchunks) load_chunk(s, s);
+      if (s < nchunks) {
+        load_chunk(s, s);
+        if (s == 0) {
+          const int64_t e0 = __ldg(a.k_out_off + off_base + v_begin);
+          const int64_t e1 = min((int64_t)__ldg(a.k_out_off + off_base + min(v_begin + kChunk, (int64_t)n_len)),
+                                 a.k_out_cap);
+          load_entries(0, e0, e1);
+        }
+      }
       cp_async_commit();
     }
     for (int c = 0; c < nchunks; ++c) {
-      cp_async_wait<NS - 3>();                // this thread's copies of chunks c and c+1 landed
+      cp_async_wait<NS - 3>();                // this thread's copies of chunks c, c+1 and entries of c landed
       bar_sync(kBarProd, kProdThr);           // everyone's landed; the stage of chunk c-1 is free
+      if (c + 1 < nchunks) {                  // chunk c+1's offsets landed with the wait above
+        const int32_t* ko1 = reinterpret_cast<const int32_t*>(stg + ((c + 1) % NS) * Lay::STAGE + Lay::S_KO);
+        load_entries((c + 1) % NS, ko1[0], min((int64_t)ko1[kChunk], a.k_out_cap));
+      }
+      cp_async_commit();
       if (c + NS - 1 < nchunks) load_chunk(c + NS - 1, (c + NS - 1) % NS);
       cp_async_commit();
-      // read ahead: this thread's key-outlier entry of chunk c+1 (its offsets are staged)
-      uint32_t kent_n = 0u;
-      if (c + 1 < nchunks) {
-        const int32_t* koff_n = reinterpret_cast<const int32_t*>(stg + ((c + 1) % NS) * Lay::STAGE + Lay::S_KO);
-        const int e = koff_n[0] + ptid;
-        if (e < min((int64_t)koff_n[kChunk], a.k_out_cap)) kent_n = __ldg(gents + e);
-      }
 
       const uint8_t* st = stg + (c % NS) * Lay::STAGE;
       const int32_t* koff = reinterpret_cast<const int32_t*>(st + Lay::S_KO);
+      const uint32_t* kcodes = reinterpret_cast<const uint32_t*>(st + Lay::S_KC);
       const int buf = c & 1;
       if (c >= 2) bar_sync(kBarEmpty + buf, kThr);   // attention on chunk c-2 released the buffer
       uint8_t* B_ = bufs + buf * Lay::BUF;
@@ -337,32 +384,34 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       uint8_t* v_t = B_ + Lay::B_VT;
       const int64_t t0 = v_begin + (int64_t)c * kChunk;
 
-      // hand the chunk's key-outlier entries, their offsets and owners to the consumers
-      reinterpret_cast<uint32_t*>(B_ + Lay::B_ENT)[ptid] = kent;
-      if (ptid <= kChunk) reinterpret_cast<int32_t*>(B_ + Lay::B_KO)[ptid] = koff[ptid];
-      if (stage_vout && ptid < kChunk * a.n_v)
-        reinterpret_cast<uint32_t*>(B_ + Lay::B_VO)[ptid] = reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[ptid];
-      if (ptid < kChunk) {
-        const int E0 = koff[0];
-        const int e_hi = min((int)min((int64_t)koff[ptid + 1], a.k_out_cap), E0 + kEntCap);
-        for (int e = koff[ptid]; e < e_hi; ++e) (B_ + Lay::B_OWN)[e - E0] = (uint8_t)ptid;
-      }
-
       // query rotated back by the chunk start: R(t0)^T q as hi, -hi and lo fp16 pairs, stored in
       // the order the mma fragments read (pair i = kc*8 + 4*hf + r at word kc*8 + 2*r + hf)
+      const float2* rts = reinterpret_cast<const float2*>(st + Lay::S_RT);
       if (ptid < nq) {
+        const float2 qcs = rts[qi];
         const float xr = qx * qcs.x + qy * qcs.y, yr = qy * qcs.x - qx * qcs.y;
         const uint32_t h = pack_half2(xr, yr);
         const float2 hf = __half22float2(*reinterpret_cast<const __half2*>(&h));
         reinterpret_cast<uint32_t*>(B_ + Lay::B_QH)[qpos] = h;
         reinterpret_cast<uint32_t*>(B_ + Lay::B_QN)[qpos] = h ^ 0x80008000u;
         reinterpret_cast<uint32_t*>(B_ + Lay::B_QL)[qpos] = pack_half2(xr - hf.x, yr - hf.y);
-        if (c + 1 < nchunks) qcs = a.rope[min(t0 + kChunk, a.rope_len - 1) * NP + qi];
       }
+
+      // the chunk's outlier data for the consumers, who restore the outliers
+      if (ptid < kEnt)
+        reinterpret_cast<uint32_t*>(B_ + Lay::B_ENT)[ptid] = reinterpret_cast<const uint32_t*>(st + Lay::S_ENT)[ptid];
+      if (ptid <= kChunk) reinterpret_cast<int32_t*>(B_ + Lay::B_KO)[ptid] = koff[ptid];
+      if (ptid < kChunk) {                    // owner token of each staged entry
+        const int E0 = koff[0];
+        const int e_hi = min((int)min((int64_t)koff[ptid + 1], a.k_out_cap), E0 + kEnt);
+        for (int e = koff[ptid]; e < e_hi; ++e) (B_ + Lay::B_OWN)[e - E0] = (uint8_t)ptid;
+      }
+      if (stage_vout && ptid < kChunk * a.n_v)
+        reinterpret_cast<uint32_t*>(B_ + Lay::B_VO)[ptid] = reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[ptid];
 
       // keys: dequantize, rotate by R(tok), split; rows past the cache end were zero-filled
       // (finite keys, masked in the attention)
-      const uint32_t* krow = reinterpret_cast<const uint32_t*>(st + Lay::S_KC) + tok * SROWW;
+      const uint32_t* krow = kcodes + tok * SROWW;
       {
         uint32_t w[NWG];
         group_words<BITS, QP, NWG>(krow, grp, w);
@@ -405,7 +454,6 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
           *reinterpret_cast<uint4*>(v_t + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
         }
       }
-      kent = kent_n;
       bar_arrive(kBarFull + buf, kThr);       // chunk c's tiles are ready
     }
     cp_async_wait<0>();
@@ -413,15 +461,16 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     // ======================= consumers: tensor-core attention =======================
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegCons) : "memory");
     const int cw = warp - kProdWarps;        // tokens 16*cw .. 16*cw + 15 of each chunk
-    const bool real = g < a.G;
+    const bool real = g < a.G;               // this lane's column of the q operand is a head
     const int mi = lane >> 3, rowi = lane & 7;
     const int t0w = cw * 16;
-    const int tokk = t0w + (mi >> 1) * 8 + rowi;
-    const int tokv = t0w + (mi & 1) * 8 + rowi;
-    float o[D / 8][2];
+    const int tokA = t0w + (mi & 1) * 8 + rowi, chA = mi >> 1;   // K slab as the A operand
+    const int tokV = t0w + (mi >> 1) * 8 + rowi, chV = mi & 1;   // V^T slab as the A operand
+    // o[j] = O^T rows (tile columns) 16j + g and 16j + g + 8, heads 2r and 2r + 1
+    float o[D / 16][4];
 #pragma unroll
-    for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = 0.f;
-    float m_run = -INFINITY, l_part = 0.f;
+    for (int j = 0; j < D / 16; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+    float m_run[2] = {-INFINITY, -INFINITY}, l_part[2] = {0.f, 0.f};
     for (int c = 0; c < nchunks; ++c) {
       const int buf = c & 1;
       bar_sync(kBarFull + buf, kThr);
@@ -430,155 +479,155 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       uint8_t* klo_t = B_ + Lay::B_KLO;
       uint8_t* v_t = B_ + Lay::B_VT;
       const int64_t t0 = v_begin + (int64_t)c * kChunk;
-      // key outliers: the thread of entry e recovers its pair before the rotation from the
-      // tile (hi - nlo, then R(d)^T), puts in the fp16 value(s), rotates and splits again
+      // Outliers of this warp's 16 tokens, restored in the rows of the tiles that only this warp
+      // reads (ordered by __syncwarp).  A key outlier x at channel ch of token t adds
+      // (x - k_dense[ch]) R(d) e_ch to the rotated pair in the tile (k_dense = R(d)^T (k_hi - nk_lo)),
+      // which is then split again; channels i < D/2 first, then i + D/2, so that the two entries of
+      // one pair never write the same word at once.
       {
         const int32_t* ko = reinterpret_cast<const int32_t*>(B_ + Lay::B_KO);
         const uint32_t* ents = reinterpret_cast<const uint32_t*>(B_ + Lay::B_ENT);
         const uint8_t* own = B_ + Lay::B_OWN;
         const uint32_t* gents = a.k_out + bh * a.k_out_cap;
         const int E0 = ko[0];
-        const int E1 = (int)min((int64_t)ko[kChunk], a.k_out_cap);
-        for (int idx = E0 + (tid - kProdThr); idx < E1; idx += kThr - kProdThr) {
-          const bool staged = idx - E0 < kEntCap;
-          const uint32_t ev = staged ? ents[idx - E0] : __ldg(gents + idx);
-          int t;
-          if (staged) {
-            t = own[idx - E0];
-          } else {                            // beyond the staged entries: search the offsets
-            t = 0;
+        const int e_lo = ko[t0w], e_hi = (int)min((int64_t)ko[t0w + 16], a.k_out_cap);
+#pragma unroll 1
+        for (int pass = 0; pass < 2; ++pass) {
+          for (int e = e_lo + lane; e < e_hi; e += 32) {
+            uint32_t ev;
+            int t;
+            if (e - E0 < kEnt) {
+              ev = ents[e - E0];
+              t = own[e - E0];
+            } else {                          // beyond the staged entries: search the offsets
+              ev = __ldg(gents + e);
+              t = t0w;
 #pragma unroll
-            for (int step = kChunk / 2; step >= 1; step >>= 1)
-              if (ko[t + step] <= idx) t += step;
-          }
-          const int ch = (int)(ev >> 16);
-          if (ch >= D) continue;              // not a channel (never written by the quantizer)
-          const int i = ch < NP ? ch : ch - NP;
-          const int partner = ch < NP ? ch + NP : ch - NP;
-          const int f_hi = min(ko[t + 1], E1);
-          bool has_p = false;
-          float pval = 0.f;
-          for (int f = ko[t]; f < f_hi; ++f) {
-            const uint32_t ef = f - E0 < kEntCap ? ents[f - E0] : __ldg(gents + f);
-            if ((int)(ef >> 16) == partner) {
-              has_p = true;
-              pval = h2f((uint16_t)(ef & 0xffffu));
+              for (int step = 8; step >= 1; step >>= 1)
+                if (ko[t + step] <= e) t += step;
             }
+            const int ch = (int)(ev >> 16);
+            if (ch >= D || (ch >= NP) != (pass == 1)) continue;
+            const int i = ch < NP ? ch : ch - NP;
+            const int byte = tile_off<D>(t, i / 4) + (i % 4) * 4;
+            const float2 hf = __half22float2(*reinterpret_cast<const __half2*>(khi_t + byte));
+            const float2 nf = __half22float2(*reinterpret_cast<const __half2*>(klo_t + byte));
+            float kx = hf.x - nf.x, ky = hf.y - nf.y;
+            const float2 cs = dtab[i * kChunk + t];
+            const float val = h2f((uint16_t)(ev & 0xffffu));
+            if (pass == 0) {
+              const float dk = val - (kx * cs.x + ky * cs.y);
+              kx = fmaf(dk, cs.x, kx);
+              ky = fmaf(dk, cs.y, ky);
+            } else {
+              const float dk = val - (ky * cs.x - kx * cs.y);
+              kx = fmaf(-dk, cs.y, kx);
+              ky = fmaf(dk, cs.x, ky);
+            }
+            uint32_t ph, pl;
+            split_hi_nlo(kx, ky, ph, pl);
+            *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
+            *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
           }
-          if (has_p && ch >= NP) continue;    // handled with its partner entry
-          const int byte = tile_off<D>(t, i / 4) + (i % 4) * 4;
-          const float2 hf = __half22float2(*reinterpret_cast<const __half2*>(khi_t + byte));
-          const float2 nf = __half22float2(*reinterpret_cast<const __half2*>(klo_t + byte));
-          const float kx = hf.x - nf.x, ky = hf.y - nf.y;
-          const float2 cs = dtab[i * kChunk + t];
-          float x = kx * cs.x + ky * cs.y, y = ky * cs.x - kx * cs.y;
-          const float val = h2f((uint16_t)(ev & 0xffffu));
-          if (ch < NP) {
-            x = val;
-            if (has_p) y = pval;
-          } else {
-            y = val;
-          }
-          uint32_t ph, pl;
-          split_hi_nlo(x * cs.x - y * cs.y, y * cs.x + x * cs.y, ph, pl);
-          *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
-          *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
+          __syncwarp();
         }
-        // value outliers: exact fp16 values over the dequantized ones
-        const bool stage_vout = a.n_v <= Lay::NVS;
-        const uint32_t* vo = reinterpret_cast<const uint32_t*>(B_ + Lay::B_VO);
-        for (int e = tid - kProdThr; e < kChunk * a.n_v; e += kThr - kProdThr) {
-          const int k = e / kChunk, t = e % kChunk;
+        // value outliers: the exact fp16 value over the dense one
+        for (int e = lane; e < 16 * a.n_v; e += 32) {
+          const int t = t0w + (e & 15), k = e >> 4;
           if (t0 + t >= n_len) continue;
-          const uint32_t ev = stage_vout ? vo[e] : __ldg(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
+          const uint32_t ev = a.n_v <= Lay::NVS ? reinterpret_cast<const uint32_t*>(B_ + Lay::B_VO)[k * kChunk + t]
+                                                : __ldg(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
           const int chn = (int)(ev >> 16);
           if (chn >= D) continue;
           const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
           *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(t, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
         }
-        bar_sync(kBarCons, kThr - kProdThr);  // every consumer warp reads every row
+        __syncwarp();
       }
       const int qrow = (real ? g : 0) * (QROW / 2);
       const uint2* qh2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QH) + qrow;
       const uint2* qn2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QN) + qrow;
       const uint2* ql2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QL) + qrow;
-      float sc[2][4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) sc[0][i] = sc[1][i] = 0.f;
+      // S^T = K q on 16 tokens x 8 heads, two independent accumulators (even / odd kc)
+      float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int kc = 0; kc < KC; ++kc) {
-        const uint2 ah = real ? qh2[kc * 4 + r] : make_uint2(0u, 0u);
-        const uint2 an = real ? qn2[kc * 4 + r] : make_uint2(0u, 0u);
-        const uint2 al = real ? ql2[kc * 4 + r] : make_uint2(0u, 0u);
-        uint32_t bhi[4], bnl[4];
-        const int ch = kc * 2 + (mi & 1);
-        ldsm_x4(bhi, khi_t + tile_off<D>(tokk, ch));
-        ldsm_x4(bnl, klo_t + tile_off<D>(tokk, ch));
-        mma16816(sc[0], ah.x, 0u, ah.y, 0u, bhi[0], bhi[1]);
-        mma16816(sc[1], ah.x, 0u, ah.y, 0u, bhi[2], bhi[3]);
-        mma16816(sc[0], an.x, 0u, an.y, 0u, bnl[0], bnl[1]);
-        mma16816(sc[1], an.x, 0u, an.y, 0u, bnl[2], bnl[3]);
-        mma16816(sc[0], al.x, 0u, al.y, 0u, bhi[0], bhi[1]);
-        mma16816(sc[1], al.x, 0u, al.y, 0u, bhi[2], bhi[3]);
+        const uint2 bhq = real ? qh2[kc * 4 + r] : make_uint2(0u, 0u);
+        const uint2 bnq = real ? qn2[kc * 4 + r] : make_uint2(0u, 0u);
+        const uint2 blq = real ? ql2[kc * 4 + r] : make_uint2(0u, 0u);
+        uint32_t ahi[4], anl[4];
+        ldsm_x4(ahi, khi_t + tile_off<D>(tokA, 2 * kc + chA));
+        ldsm_x4(anl, klo_t + tile_off<D>(tokA, 2 * kc + chA));
+        float* acc = (kc & 1) ? sb : sa;
+        mma16816(acc, ahi[0], ahi[1], ahi[2], ahi[3], bhq.x, bhq.y);
+        mma16816(acc, anl[0], anl[1], anl[2], anl[3], bnq.x, bnq.y);
+        mma16816(acc, ahi[0], ahi[1], ahi[2], ahi[3], blq.x, blq.y);
       }
-      const int tk[4] = {t0w + 2 * r, t0w + 2 * r + 1, t0w + 8 + 2 * r, t0w + 9 + 2 * r};
-      float x[4] = {sc[0][0], sc[0][1], sc[1][0], sc[1][1]};
-      float mx = -INFINITY;
+      // x[e][u]: head 2r + e, token g + 8u of the slab
+      const bool ok0 = t0 + t0w + g < n_len, ok1 = t0 + t0w + g + 8 < n_len;
+      float x[2][2];
+      x[0][0] = ok0 ? (sa[0] + sb[0]) * a.scale_log2 : -INFINITY;
+      x[1][0] = ok0 ? (sa[1] + sb[1]) * a.scale_log2 : -INFINITY;
+      x[0][1] = ok1 ? (sa[2] + sb[2]) * a.scale_log2 : -INFINITY;
+      x[1][1] = ok1 ? (sa[3] + sb[3]) * a.scale_log2 : -INFINITY;
+      float p[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+      float alpha[2] = {1.f, 1.f};
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        x[i] = (t0 + tk[i] < n_len) ? x[i] * a.scale_log2 : -INFINITY;
-        mx = fmaxf(mx, x[i]);
+      for (int e = 0; e < 2; ++e) {
+        float mx = fmaxf(x[e][0], x[e][1]);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+        const float m_new = fmaxf(m_run[e], mx);
+        if (m_new != -INFINITY) {
+          alpha[e] = exp2f(m_run[e] - m_new);
+          p[e][0] = exp2f(x[e][0] - m_new);
+          p[e][1] = exp2f(x[e][1] - m_new);
+        }
+        l_part[e] = l_part[e] * alpha[e] + (p[e][0] + p[e][1]);
+        m_run[e] = m_new;
       }
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      const float m_new = fmaxf(m_run, mx);
-      float p[4] = {0.f, 0.f, 0.f, 0.f};
-      float alpha = 1.f;
-      if (m_new != -INFINITY) {
-        alpha = exp2f(m_run - m_new);
+      if (__any_sync(0xffffffffu, alpha[0] != 1.f || alpha[1] != 1.f)) {
 #pragma unroll
-        for (int i = 0; i < 4; ++i) p[i] = exp2f(x[i] - m_new);
-      }
-      l_part = l_part * alpha + (p[0] + p[1]) + (p[2] + p[3]);
-      m_run = m_new;
-      if (__any_sync(0xffffffffu, alpha != 1.f)) {
-#pragma unroll
-        for (int i = 0; i < D / 8; ++i) {
-          o[i][0] *= alpha;
-          o[i][1] *= alpha;
+        for (int j = 0; j < D / 16; ++j) {
+          o[j][0] *= alpha[0];
+          o[j][1] *= alpha[1];
+          o[j][2] *= alpha[0];
+          o[j][3] *= alpha[1];
         }
       }
-      const uint32_t pa0 = pack_half2(p[0], p[1]);
-      const uint32_t pa2 = pack_half2(p[2], p[3]);
+      // P as two 8x8 (token x head) fp16 matrices, transposed into the B operand (tokens x heads)
+      const uint32_t pb0 = movm_trans(pack_half2(p[0][0], p[1][0]));
+      const uint32_t pb1 = movm_trans(pack_half2(p[0][1], p[1][1]));
 #pragma unroll
       for (int j = 0; j < D / 16; ++j) {
-        uint32_t bv[4];
-        ldsm_x4_t(bv, v_t + tile_off<D>(tokv, 2 * j + (mi >> 1)));
-        float d0[4] = {o[2 * j][0], o[2 * j][1], 0.f, 0.f};
-        float d1[4] = {o[2 * j + 1][0], o[2 * j + 1][1], 0.f, 0.f};
-        mma16816(d0, pa0, 0u, pa2, 0u, bv[0], bv[1]);
-        mma16816(d1, pa0, 0u, pa2, 0u, bv[2], bv[3]);
-        o[2 * j][0] = d0[0];
-        o[2 * j][1] = d0[1];
-        o[2 * j + 1][0] = d1[0];
-        o[2 * j + 1][1] = d1[1];
+        uint32_t av[4];
+        ldsm_x4_t(av, v_t + tile_off<D>(tokV, 2 * j + chV));
+        mma16816(o[j], av[0], av[1], av[2], av[3], pb0, pb1);
       }
       if (c + 2 < nchunks) bar_arrive(kBarEmpty + buf, kThr);   // producers may refill the buffer
     }
     // The producers are done with every stage once the last chunk was handed over (and no
     // stage was filled when there are no chunks), so the stage area takes the partials.
-    l_part += __shfl_xor_sync(0xffffffffu, l_part, 1);
-    l_part += __shfl_xor_sync(0xffffffffu, l_part, 2);
-    if (g < a.G) {
-      if (r == 0) {
-        wm[cw * 8 + g] = m_run;
-        wl[cw * 8 + g] = l_part;
-      }
 #pragma unroll
-      for (int dt = 0; dt < D / 8; ++dt) {
-        const int chn = dt * 4 + r;                          // column dt*8 + 2r -> channel dt*4 + r
-        wo[(cw * 8 + g) * D + chn] = o[dt][0];
-        wo[(cw * 8 + g) * D + chn + NP] = o[dt][1];
+    for (int e = 0; e < 2; ++e) {
+      l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], 4);
+      l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], 8);
+      l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], 16);
+      const int hh = 2 * r + e;
+      if (hh < a.G) {
+        if (g == 0) {
+          wm[cw * 8 + hh] = m_run[e];
+          wl[cw * 8 + hh] = l_part[e];
+        }
+#pragma unroll
+        for (int j = 0; j < D / 16; ++j) {
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int col = 16 * j + g + 8 * u;                  // tile column -> channel
+            wo[(cw * 8 + hh) * D + (col >> 1) + (col & 1) * NP] = o[j][2 * u + e];
+          }
+        }
       }
     }
   }
