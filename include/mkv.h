@@ -118,7 +118,8 @@ typedef struct {
  *         k_out_off int32 [B][Hkv][T_cap + 1]: CSR offsets of key outliers
  *           per token (k_out_off[..][0] = 0).
  *         k_out uint32 [B][Hkv][k_out_cap]: key outliers of token t at
- *           [k_out_off[t], k_out_off[t+1]), (channel << 16) | fp16 bits.
+ *           [k_out_off[t], k_out_off[t+1]), in channel order, each
+ *           ((t mod 64) << 24) | (channel << 16) | fp16 bits.
  */
 typedef struct {
   int64_t T_cap;

@@ -21,17 +21,17 @@
 // a rotation held in registers for the whole kernel (the chunk start's own
 // rotation R(t0) is applied to the query instead:
 // q . R(t0 + d) k = (R(t0)^T q) . (R(d) k)) and written as fp16 hi plus the
-// negated fp16 remainder, so the tensor-core product keeps fp32 accuracy.
-// Dense-and-sparse outliers are restored by the producers as well.  A value
-// outlier overwrites its tile entry (by the thread that wrote the dense value).
-// A key outlier enters the score linearly: with k = k_dense + (x - k_dense[c]) e_c,
-// q . R(t) k = q . R(t) k_dense + (x - k_dense[c]) (R(t)^T q)[c], so one thread
-// per outlier entry adds that fp32 term for every query head of the group to a
-// per-chunk correction table, and the consumers add it to the tensor-core
-// scores.  Consumers: S^T (tokens x heads) = K_hi q_hi - K_nlo q_hi + K_hi q_lo
-// on 16-token slabs, online softmax, then O^T (dims x heads) += V^T P^T with P^T
-// transposed in registers (movmatrix).  Tile columns hold pair i at columns
-// (2i, 2i+1) = channels (i, i + D/2); the output is un-permuted at the end.
+// fp16 remainder lo, so the tensor-core product keeps fp32 accuracy.  The same
+// thread restores its token's value outliers in its pairs (exact fp16 values).
+// Consumers: each of the four attention warps owns 16 token rows of a chunk.  It
+// first restores the key outliers of its rows in the key tiles (an outlier x at
+// channel ch adds (x - k_dense[ch]) R(d) e_ch to the rotated pair, which is split
+// again; x-channels before y-channels so the two entries of a pair never write
+// one word at once; __syncwarp orders it, as only this warp reads those rows),
+// then computes S^T (tokens x heads) = K_hi q_hi + K_lo q_hi + K_hi q_lo, the
+// online softmax, and O^T (dims x heads) += V^T P^T with P^T transposed in
+// registers (movmatrix).  Tile columns hold pair i at columns (2i, 2i+1) =
+// channels (i, i + D/2); the output is un-permuted at the end.
 #include <math.h>
 
 #include "mkv_common.cuh"
@@ -116,18 +116,15 @@ struct KvqLayout {
   static constexpr int S_ENT = S_VO + NVS * kChunk * 4;      // [kEnt] u32 first key-outlier entries
   static constexpr int S_RT = S_ENT + kEnt * 4;          // [NP] float2 rotation of the chunk start
   static constexpr int STAGE = S_RT + NP * 8;
-  // one tile buffer: keys (hi, negated lo), values, and the rotated query
+  // one tile buffer: keys (hi, lo), values, the rotated query and the chunk's key outliers
   static constexpr int B_KHI = 0;
   static constexpr int B_KLO = B_KHI + TILE;
   static constexpr int B_VT = B_KLO + TILE;
   static constexpr int B_QH = B_VT + TILE;                   // [8][QROW] q_hi pairs, fragment order
-  static constexpr int B_QN = B_QH + 8 * QROW * 4;           // -q_hi
-  static constexpr int B_QL = B_QN + 8 * QROW * 4;           // q_lo
+  static constexpr int B_QL = B_QH + 8 * QROW * 4;           // q_lo
   static constexpr int B_ENT = B_QL + 8 * QROW * 4;          // [kEnt] u32 first key-outlier entries
-  static constexpr int B_OWN = B_ENT + kEnt * 4;             // [kEnt] u8 token of each
-  static constexpr int B_KO = B_OWN + kEnt;                  // [68] int32 CSR offsets of the chunk
-  static constexpr int B_VO = B_KO + 68 * 4;                 // [NVS][64] u32 value outliers
-  static constexpr int BUF = B_VO + NVS * kChunk * 4;
+  static constexpr int B_KO = B_ENT + kEnt * 4;              // [68] int32 CSR offsets of the chunk
+  static constexpr int BUF = B_KO + 68 * 4;
   // CTA layout
   static constexpr int DTAB = 0;                             // [NP][64] float2 rotation by delta
   static constexpr int KDQ = DTAB + NP * kChunk * 8;         // [D][K] float
@@ -176,8 +173,8 @@ __device__ __forceinline__ void group_words(const uint32_t* row, int g, uint32_t
   }
 }
 
-// (a, b) as fp16 hi and the negated fp16 remainder (hi - x), exact in fp32
-__device__ __forceinline__ void split_hi_nlo(float a, float b, uint32_t& hi, uint32_t& nlo) {
+// (a, b) as fp16 hi and the fp16 remainder lo = x - hi (exact in fp32 before its rounding)
+__device__ __forceinline__ void split_hi_lo(float a, float b, uint32_t& hi, uint32_t& lo) {
   uint32_t h;
   asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(h) : "f"(b), "f"(a));
   float d0, d1;
@@ -185,7 +182,7 @@ __device__ __forceinline__ void split_hi_nlo(float a, float b, uint32_t& hi, uin
       : "=f"(d0), "=f"(d1)
       : "r"(h), "f"(a), "f"(b));
   hi = h;
-  nlo = pack_half2(d0, d1);
+  lo = pack_half2(-d0, -d1);
 }
 
 __device__ __forceinline__ void cp_async4s(uint32_t saddr, const void* gmem, int src_bytes) {
@@ -377,37 +374,37 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       const int32_t* koff = reinterpret_cast<const int32_t*>(st + Lay::S_KO);
       const uint32_t* kcodes = reinterpret_cast<const uint32_t*>(st + Lay::S_KC);
       const int buf = c & 1;
+      const int64_t t0 = v_begin + (int64_t)c * kChunk;
+      // staged words this thread hands on or uses late, read before the wait for the buffer: its
+      // key-outlier entry and offset for the consumers, its part of the chunk-start rotation, and
+      // its token's value outliers
+      const uint32_t my_ent = ptid < kEnt ? reinterpret_cast<const uint32_t*>(st + Lay::S_ENT)[ptid] : 0u;
+      const int32_t my_ko = ptid <= kChunk ? koff[ptid] : 0;
+      const float2 qcs = reinterpret_cast<const float2*>(st + Lay::S_RT)[qi];
+      uint32_t vo[Lay::NVS];
+#pragma unroll
+      for (int k = 0; k < Lay::NVS; ++k)
+        vo[k] = (stage_vout && k < a.n_v) ? reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[k * kChunk + tok]
+                                          : 0xffff0000u;
       if (c >= 2) bar_sync(kBarEmpty + buf, kThr);   // attention on chunk c-2 released the buffer
       uint8_t* B_ = bufs + buf * Lay::BUF;
       uint8_t* khi_t = B_ + Lay::B_KHI;
       uint8_t* klo_t = B_ + Lay::B_KLO;
       uint8_t* v_t = B_ + Lay::B_VT;
-      const int64_t t0 = v_begin + (int64_t)c * kChunk;
 
       // query rotated back by the chunk start: R(t0)^T q as hi, -hi and lo fp16 pairs, stored in
       // the order the mma fragments read (pair i = kc*8 + 4*hf + r at word kc*8 + 2*r + hf)
-      const float2* rts = reinterpret_cast<const float2*>(st + Lay::S_RT);
       if (ptid < nq) {
-        const float2 qcs = rts[qi];
         const float xr = qx * qcs.x + qy * qcs.y, yr = qy * qcs.x - qx * qcs.y;
         const uint32_t h = pack_half2(xr, yr);
         const float2 hf = __half22float2(*reinterpret_cast<const __half2*>(&h));
         reinterpret_cast<uint32_t*>(B_ + Lay::B_QH)[qpos] = h;
-        reinterpret_cast<uint32_t*>(B_ + Lay::B_QN)[qpos] = h ^ 0x80008000u;
         reinterpret_cast<uint32_t*>(B_ + Lay::B_QL)[qpos] = pack_half2(xr - hf.x, yr - hf.y);
       }
 
-      // the chunk's outlier data for the consumers, who restore the outliers
-      if (ptid < kEnt)
-        reinterpret_cast<uint32_t*>(B_ + Lay::B_ENT)[ptid] = reinterpret_cast<const uint32_t*>(st + Lay::S_ENT)[ptid];
-      if (ptid <= kChunk) reinterpret_cast<int32_t*>(B_ + Lay::B_KO)[ptid] = koff[ptid];
-      if (ptid < kChunk) {                    // owner token of each staged entry
-        const int E0 = koff[0];
-        const int e_hi = min((int)min((int64_t)koff[ptid + 1], a.k_out_cap), E0 + kEnt);
-        for (int e = koff[ptid]; e < e_hi; ++e) (B_ + Lay::B_OWN)[e - E0] = (uint8_t)ptid;
-      }
-      if (stage_vout && ptid < kChunk * a.n_v)
-        reinterpret_cast<uint32_t*>(B_ + Lay::B_VO)[ptid] = reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[ptid];
+      // the chunk's key-outlier entries for the consumers, who restore them
+      if (ptid < kEnt) reinterpret_cast<uint32_t*>(B_ + Lay::B_ENT)[ptid] = my_ent;
+      if (ptid <= kChunk) reinterpret_cast<int32_t*>(B_ + Lay::B_KO)[ptid] = my_ko;
 
       // keys: dequantize, rotate by R(tok), split; rows past the cache end were zero-filled
       // (finite keys, masked in the attention)
@@ -426,7 +423,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
             pair_codes<BITS, NWG>(w, j, clo, chi);
             const float x = kq[j * K + clo];
             const float y = kq[(j + NP) * K + chi];
-            split_hi_nlo(x * rot[j].x - y * rot[j].y, y * rot[j].x + x * rot[j].y, ph[u], pl[u]);
+            split_hi_lo(x * rot[j].x - y * rot[j].y, y * rot[j].x + x * rot[j].y, ph[u], pl[u]);
           }
           const int ch = (grp * QP + jj) / 4;
           *reinterpret_cast<uint4*>(khi_t + tile_off<D>(tok, ch)) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
@@ -454,6 +451,23 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
           *reinterpret_cast<uint4*>(v_t + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
         }
       }
+      // value outliers of this thread's token in its pairs: the exact fp16 value over the dense one
+      if (t0 + tok < n_len) {
+        auto put = [&](uint32_t ev) {
+          const int chn = (int)(ev >> 16);
+          const int i = chn < NP ? chn : chn - NP;
+          if (chn < D && i / QP == grp) {
+            const int col = 2 * i + (chn >= NP ? 1 : 0);
+            *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(tok, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
+          }
+        };
+        if (stage_vout) {
+#pragma unroll
+          for (int k = 0; k < Lay::NVS; ++k) put(vo[k]);
+        } else {
+          for (int k = 0; k < a.n_v; ++k) put(__ldg(a.v_out + (bh * a.T_cap + t0 + tok) * a.n_v + k));
+        }
+      }
       bar_arrive(kBarFull + buf, kThr);       // chunk c's tiles are ready
     }
     cp_async_wait<0>();
@@ -479,88 +493,73 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       uint8_t* klo_t = B_ + Lay::B_KLO;
       uint8_t* v_t = B_ + Lay::B_VT;
       const int64_t t0 = v_begin + (int64_t)c * kChunk;
-      // Outliers of this warp's 16 tokens, restored in the rows of the tiles that only this warp
-      // reads (ordered by __syncwarp).  A key outlier x at channel ch of token t adds
-      // (x - k_dense[ch]) R(d) e_ch to the rotated pair in the tile (k_dense = R(d)^T (k_hi - nk_lo)),
+      // Key outliers of this warp's 16 tokens, restored in the rows of the key tiles that only this
+      // warp reads (ordered by __syncwarp).  An outlier x at channel ch of token t adds
+      // (x - k_dense[ch]) R(d) e_ch to the rotated pair in the tile (k_dense = R(d)^T (k_hi + k_lo)),
       // which is then split again; channels i < D/2 first, then i + D/2, so that the two entries of
-      // one pair never write the same word at once.
+      // one pair never write the same word at once.  Each entry carries its token within the chunk.
       {
         const int32_t* ko = reinterpret_cast<const int32_t*>(B_ + Lay::B_KO);
         const uint32_t* ents = reinterpret_cast<const uint32_t*>(B_ + Lay::B_ENT);
-        const uint8_t* own = B_ + Lay::B_OWN;
         const uint32_t* gents = a.k_out + bh * a.k_out_cap;
         const int E0 = ko[0];
         const int e_lo = ko[t0w], e_hi = (int)min((int64_t)ko[t0w + 16], a.k_out_cap);
-#pragma unroll 1
-        for (int pass = 0; pass < 2; ++pass) {
-          for (int e = e_lo + lane; e < e_hi; e += 32) {
-            uint32_t ev;
-            int t;
-            if (e - E0 < kEnt) {
-              ev = ents[e - E0];
-              t = own[e - E0];
-            } else {                          // beyond the staged entries: search the offsets
-              ev = __ldg(gents + e);
-              t = t0w;
-#pragma unroll
-              for (int step = 8; step >= 1; step >>= 1)
-                if (ko[t + step] <= e) t += step;
-            }
-            const int ch = (int)(ev >> 16);
-            if (ch >= D || (ch >= NP) != (pass == 1)) continue;
-            const int i = ch < NP ? ch : ch - NP;
-            const int byte = tile_off<D>(t, i / 4) + (i % 4) * 4;
-            const float2 hf = __half22float2(*reinterpret_cast<const __half2*>(khi_t + byte));
-            const float2 nf = __half22float2(*reinterpret_cast<const __half2*>(klo_t + byte));
-            float kx = hf.x - nf.x, ky = hf.y - nf.y;
-            const float2 cs = dtab[i * kChunk + t];
-            const float val = h2f((uint16_t)(ev & 0xffffu));
-            if (pass == 0) {
-              const float dk = val - (kx * cs.x + ky * cs.y);
-              kx = fmaf(dk, cs.x, kx);
-              ky = fmaf(dk, cs.y, ky);
-            } else {
-              const float dk = val - (ky * cs.x - kx * cs.y);
-              kx = fmaf(-dk, cs.y, kx);
-              ky = fmaf(dk, cs.x, ky);
-            }
-            uint32_t ph, pl;
-            split_hi_nlo(kx, ky, ph, pl);
-            *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
-            *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
+        auto fetch = [&](int e) -> uint32_t {
+          if (e >= e_hi) return 0xffff0000u;  // no entry: not a channel
+          if (e - E0 < kEnt) return ents[e - E0];
+          return __ldg(gents + e);            // beyond the staged entries
+        };
+        auto fix = [&](uint32_t ev, int pass) {
+          const int ch = (int)((ev >> 16) & 0xffu);
+          if (ch >= D || (ch >= NP) != (pass == 1)) return;
+          const int t = (int)(ev >> 24) & (kChunk - 1);
+          const int i = ch < NP ? ch : ch - NP;
+          const int byte = tile_off<D>(t, i / 4) + (i % 4) * 4;
+          const float2 hf = __half22float2(*reinterpret_cast<const __half2*>(khi_t + byte));
+          const float2 lf = __half22float2(*reinterpret_cast<const __half2*>(klo_t + byte));
+          float kx = hf.x + lf.x, ky = hf.y + lf.y;
+          const float2 cs = dtab[i * kChunk + t];
+          const float val = h2f((uint16_t)(ev & 0xffffu));
+          if (pass == 0) {
+            const float dk = val - (kx * cs.x + ky * cs.y);
+            kx = fmaf(dk, cs.x, kx);
+            ky = fmaf(dk, cs.y, ky);
+          } else {
+            const float dk = val - (ky * cs.x - kx * cs.y);
+            kx = fmaf(-dk, cs.y, kx);
+            ky = fmaf(dk, cs.x, ky);
           }
-          __syncwarp();
-        }
-        // value outliers: the exact fp16 value over the dense one
-        for (int e = lane; e < 16 * a.n_v; e += 32) {
-          const int t = t0w + (e & 15), k = e >> 4;
-          if (t0 + t >= n_len) continue;
-          const uint32_t ev = a.n_v <= Lay::NVS ? reinterpret_cast<const uint32_t*>(B_ + Lay::B_VO)[k * kChunk + t]
-                                                : __ldg(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
-          const int chn = (int)(ev >> 16);
-          if (chn >= D) continue;
-          const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
-          *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(t, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
-        }
+          uint32_t ph, pl;
+          split_hi_lo(kx, ky, ph, pl);
+          *reinterpret_cast<uint32_t*>(khi_t + byte) = ph;
+          *reinterpret_cast<uint32_t*>(klo_t + byte) = pl;
+        };
+        const uint32_t ea = fetch(e_lo + lane), eb = fetch(e_lo + 32 + lane);
+        fix(ea, 0);
+        fix(eb, 0);
+        for (int e = e_lo + 64 + lane; e < e_hi; e += 32) fix(fetch(e), 0);
+        __syncwarp();
+        fix(ea, 1);
+        fix(eb, 1);
+        for (int e = e_lo + 64 + lane; e < e_hi; e += 32) fix(fetch(e), 1);
         __syncwarp();
       }
       const int qrow = (real ? g : 0) * (QROW / 2);
       const uint2* qh2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QH) + qrow;
-      const uint2* qn2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QN) + qrow;
       const uint2* ql2 = reinterpret_cast<const uint2*>(B_ + Lay::B_QL) + qrow;
-      // S^T = K q on 16 tokens x 8 heads, two independent accumulators (even / odd kc)
+      // S^T = K_hi q_hi + K_lo q_hi + K_hi q_lo on 16 tokens x 8 heads, two independent accumulators
+      // (even / odd kc)
       float sa[4] = {0.f, 0.f, 0.f, 0.f}, sb[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int kc = 0; kc < KC; ++kc) {
         const uint2 bhq = real ? qh2[kc * 4 + r] : make_uint2(0u, 0u);
-        const uint2 bnq = real ? qn2[kc * 4 + r] : make_uint2(0u, 0u);
         const uint2 blq = real ? ql2[kc * 4 + r] : make_uint2(0u, 0u);
-        uint32_t ahi[4], anl[4];
+        uint32_t ahi[4], alo[4];
         ldsm_x4(ahi, khi_t + tile_off<D>(tokA, 2 * kc + chA));
-        ldsm_x4(anl, klo_t + tile_off<D>(tokA, 2 * kc + chA));
+        ldsm_x4(alo, klo_t + tile_off<D>(tokA, 2 * kc + chA));
         float* acc = (kc & 1) ? sb : sa;
         mma16816(acc, ahi[0], ahi[1], ahi[2], ahi[3], bhq.x, bhq.y);
-        mma16816(acc, anl[0], anl[1], anl[2], anl[3], bnq.x, bnq.y);
+        mma16816(acc, alo[0], alo[1], alo[2], alo[3], bhq.x, bhq.y);
         mma16816(acc, ahi[0], ahi[1], ahi[2], ahi[3], blq.x, blq.y);
       }
       // x[e][u]: head 2r + e, token g + 8u of the slab

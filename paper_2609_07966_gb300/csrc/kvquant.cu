@@ -139,7 +139,9 @@ __global__ void quantize_kernel(const QuantArgs a) {
     if (kout) {
       const int64_t e = (int64_t)off + before + __popc(bal & ((1u << lane) - 1u));
       if (e < a.k_out_cap) {
-        a.k_out[(int64_t)bh * a.k_out_cap + e] = ((uint32_t)c << 16) | __half_as_ushort(a.k_pre[src]);
+        // (token position within its 64-token block << 24) | (channel << 16) | fp16 bits
+        a.k_out[(int64_t)bh * a.k_out_cap + e] =
+            ((uint32_t)(t & 63) << 24) | ((uint32_t)c << 16) | __half_as_ushort(a.k_pre[src]);
       } else {
         atomicOr(&g_status_kvquant, MKV_FLAG_K_OUTLIER_OVERFLOW);
       }

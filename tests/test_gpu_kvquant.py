@@ -141,7 +141,8 @@ def test_quantize_bit_exact(bits, mode, D):
             assert np.array_equal(vpar[b, h, :, 1].view(np.uint32), qh.v_scale.view(np.uint32))
             for t in range(n):
                 ents = kout[b, h, off[b, h, t]:off[b, h, t + 1]]
-                got = {(int(e >> 16), int(e & 0xffff)) for e in ents}
+                assert all(int(e >> 24) == t % 64 for e in ents), f"key outlier token field b{b} h{h} t{t}"
+                got = {(int((e >> 16) & 0xff), int(e & 0xffff)) for e in ents}
                 chans = np.nonzero(qh.k_mask[t])[0]
                 ref = {(int(c), int(k[b, h, t, c].view(np.uint16))) for c in chans}
                 assert got == ref, f"key outliers b{b} h{h} t{t}"
