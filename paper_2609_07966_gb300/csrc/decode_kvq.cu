@@ -569,24 +569,22 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       x[1][0] = ok0 ? (sa[1] + sb[1]) * a.scale_log2 : -INFINITY;
       x[0][1] = ok1 ? (sa[2] + sb[2]) * a.scale_log2 : -INFINITY;
       x[1][1] = ok1 ? (sa[3] + sb[3]) * a.scale_log2 : -INFINITY;
-      float p[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
-      float alpha[2] = {1.f, 1.f};
+      float p[2][2];
+      // the running maxima move only when a score exceeds them: then (rarely, after the first
+      // chunks) reduce the slab's maxima across the lanes of each head and rescale
+      if (__any_sync(0xffffffffu, fmaxf(x[0][0], x[0][1]) > m_run[0] || fmaxf(x[1][0], x[1][1]) > m_run[1])) {
+        float alpha[2] = {1.f, 1.f};
 #pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        float mx = fmaxf(x[e][0], x[e][1]);
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-        const float m_new = fmaxf(m_run[e], mx);
-        if (m_new != -INFINITY) {
-          alpha[e] = exp2f(m_run[e] - m_new);
-          p[e][0] = exp2f(x[e][0] - m_new);
-          p[e][1] = exp2f(x[e][1] - m_new);
+        for (int e = 0; e < 2; ++e) {
+          float mx = fmaxf(x[e][0], x[e][1]);
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+          const float m_new = fmaxf(m_run[e], mx);
+          if (m_new != -INFINITY) alpha[e] = exp2f(m_run[e] - m_new);
+          l_part[e] *= alpha[e];
+          m_run[e] = m_new;
         }
-        l_part[e] = l_part[e] * alpha[e] + (p[e][0] + p[e][1]);
-        m_run[e] = m_new;
-      }
-      if (__any_sync(0xffffffffu, alpha[0] != 1.f || alpha[1] != 1.f)) {
 #pragma unroll
         for (int j = 0; j < D / 16; ++j) {
           o[j][0] *= alpha[0];
@@ -594,6 +592,13 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
           o[j][2] *= alpha[0];
           o[j][3] *= alpha[1];
         }
+      }
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        // exp2(-inf - m) = 0 for masked tokens; a head with no score yet (m = -inf) has none
+        p[e][0] = m_run[e] != -INFINITY ? exp2f(x[e][0] - m_run[e]) : 0.f;
+        p[e][1] = m_run[e] != -INFINITY ? exp2f(x[e][1] - m_run[e]) : 0.f;
+        l_part[e] += p[e][0] + p[e][1];
       }
       // P as two 8x8 (token x head) fp16 matrices, transposed into the B operand (tokens x heads)
       const uint32_t pb0 = movm_trans(pack_half2(p[0][0], p[1][0]));
