@@ -84,7 +84,9 @@ struct KvqArgs {
   const int32_t* T_len;
   int64_t T_cap, k_out_cap;
   int Hq, Hkv, G, n_v;
-  int chunks_per_split, n_split;
+  int n_split;             // partial slots per (batch, kv-head)
+  int n_cta;               // CTA i covers virtual chunks [i * c_tot / n_cta, (i + 1) * c_tot / n_cta)
+  int64_t cpu, c_tot;      // virtual chunks per (batch, kv-head), and of all of them
   float scale_log2;
   float* part_m;
   float* part_l;
@@ -223,35 +225,107 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   uint8_t* stg = smem + Lay::STG;
   uint8_t* bufs = smem + Lay::BUFS;
 
-  const int split = blockIdx.x;
-  const int64_t bh = blockIdx.y;
-  const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
+  const int cta = blockIdx.x;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, r = lane & 3;
-  const int n_len = (int)min((int64_t)a.T_len[b], a.T_cap);
-  const int64_t v_begin = (int64_t)split * a.chunks_per_split * kChunk;
-  int64_t v_end = v_begin + (int64_t)a.chunks_per_split * kChunk;
-  if (v_end > n_len) v_end = n_len;
-  const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
+  // this CTA's virtual chunks of the concatenated (batch, kv-head) units: one segment per unit
+  const int64_t x0 = (int64_t)cta * a.c_tot / a.n_cta, x1 = ((int64_t)cta + 1) * a.c_tot / a.n_cta;
 
-  // CTA-resident tables: rotations by delta in [0, 64), dequant tables of this kv-head, the
-  // group's queries in fp32
-  for (int e = tid; e < NP * kChunk; e += kThr) {  // coalesced read of rope rows 0..63, transposed
-    const int d = e / NP, i = e % NP;
-    dtab[i * kChunk + d] = a.rope[(int64_t)min((int64_t)d, a.rope_len - 1) * NP + i];
+  // CTA-resident rotations by delta in [0, 64): coalesced reads of rope rows 0..63, all issued
+  // before the transposed stores
+  {
+    constexpr int NE = (NP * kChunk + kThr - 1) / kThr;
+    float2 v[NE];
+#pragma unroll
+    for (int k = 0; k < NE; ++k) {
+      const int e = tid + k * kThr;
+      const int d = e / NP, i = e % NP;
+      if (e < NP * kChunk) v[k] = __ldg(a.rope + (int64_t)min((int64_t)d, a.rope_len - 1) * NP + i);
+    }
+#pragma unroll
+    for (int k = 0; k < NE; ++k) {
+      const int e = tid + k * kThr;
+      if (e < NP * kChunk) dtab[(e % NP) * kChunk + e / NP] = v[k];
+    }
   }
-  for (int e = tid; e < D * K; e += kThr) {
-    kdq[e] = a.k_dq[(int64_t)kvh * D * K + e];
-    vtb[e] = __half2float(__ushort_as_half(a.v_tbl[(int64_t)kvh * D * K + e]));
-  }
-  for (int e = tid; e < a.G * D; e += kThr)
-    qs[e] = __half2float(a.q[((int64_t)b * a.Hq + (int64_t)kvh * a.G) * D + e]);
   __syncthreads();
 
-  // the four attention warps' (m, l, o) per query row, merged after both roles finish
+  // the four attention warps' (m, l, o) per query row, merged after both roles finish a segment
   float* wm = reinterpret_cast<float*>(stg);                // [4 warps][8 rows]
   float* wl = wm + 32;                                       // [4][8]
   float* wo = wl + 32;                                       // [4][8][D]  natural channel order
+
+  // Both roles run the same segments; these steps take every thread of the CTA.
+  // Start of a segment of unit bh: dequant tables of its kv-head, its group's queries in fp32.
+  auto begin_unit = [&](int64_t bh) {
+    const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
+    constexpr int NT = (D * K + kThr - 1) / kThr;           // all loads in flight, then the stores
+    float kv[NT];
+    uint16_t vv[NT];
+#pragma unroll
+    for (int k = 0; k < NT; ++k) {
+      const int e = tid + k * kThr;
+      if (e < D * K) {
+        kv[k] = __ldg(a.k_dq + (int64_t)kvh * D * K + e);
+        vv[k] = __ldg(a.v_tbl + (int64_t)kvh * D * K + e);
+      }
+    }
+    constexpr int NQ = (8 * D + kThr - 1) / kThr;
+    __half qv[NQ];
+#pragma unroll
+    for (int k = 0; k < NQ; ++k) {
+      const int e = tid + k * kThr;
+      if (e < a.G * D) qv[k] = a.q[((int64_t)b * a.Hq + (int64_t)kvh * a.G) * D + e];
+    }
+#pragma unroll
+    for (int k = 0; k < NT; ++k) {
+      const int e = tid + k * kThr;
+      if (e < D * K) {
+        kdq[e] = kv[k];
+        vtb[e] = __half2float(__ushort_as_half(vv[k]));
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < NQ; ++k) {
+      const int e = tid + k * kThr;
+      if (e < a.G * D) qs[e] = __half2float(qv[k]);
+    }
+    __syncthreads();
+  };
+  // End of a segment: the warps' partials merged into this CTA's partial slot of the unit, and
+  // the unit's last CTA merges all of them.
+  auto end_unit = [&](int64_t bh) {
+    const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
+    const int64_t first = cta_of_chunk(bh * a.cpu, a.c_tot, a.n_cta);
+    const int slot = (int)(cta - first);
+    const int parts = (int)(cta_of_chunk((bh + 1) * a.cpu - 1, a.c_tot, a.n_cta) - first + 1);
+    __syncthreads();
+    for (int e = tid; e < a.G * D; e += kThr) {
+      const int row = e / D, d = e % D;
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < kConsWarps; ++w) M = fmaxf(M, wm[w * 8 + row]);
+      float L = 0.f, O = 0.f;
+      if (M != -INFINITY) {
+#pragma unroll
+        for (int w = 0; w < kConsWarps; ++w) {
+          const float f = exp2f(wm[w * 8 + row] - M);
+          L += wl[w * 8 + row] * f;
+          O += wo[(w * 8 + row) * D + d] * f;
+        }
+      }
+      const int64_t hq = (int64_t)b * a.Hq + (int64_t)kvh * a.G + row;
+      const int64_t pi = hq * a.n_split + slot;
+      a.part_o[pi * D + d] = O;
+      if (d == 0) {
+        a.part_m[pi] = M;
+        a.part_l[pi] = L;
+      }
+    }
+    __syncthreads();                   // the stage buffers now serve as the merge's scratch
+    merge_if_last<D, kThr>(a.merge, bh, b, kvh, reinterpret_cast<float*>(stg), Lay::NS * Lay::STAGE / 4, parts);
+    __syncthreads();                   // before the next segment's copies into the stages
+  };
 
   if (warp < kProdWarps) {
     // ======================= producers: stage, dequantize, rotate =======================
@@ -259,6 +333,15 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     const int ptid = tid;
     const int tok = (warp & 1) * 32 + lane;   // this thread's token row in every chunk
     const int grp = warp >> 1;                // its pairs: grp * QP .. grp * QP + QP - 1
+    for (int64_t x = x0; x < x1;) {
+      const int64_t bh = x / a.cpu;                           // this segment's unit
+      const int64_t xe = min(x1, (bh + 1) * a.cpu);
+      begin_unit(bh);
+      const int b = (int)(bh / a.Hkv);
+      const int n_len = (int)min((int64_t)a.T_len[b], a.T_cap);
+      const int64_t v_begin = (x - bh * a.cpu) * kChunk;
+      const int64_t v_end = min((xe - bh * a.cpu) * kChunk, (int64_t)n_len);
+      const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
     const uint32_t* kc_base = reinterpret_cast<const uint32_t*>(a.k_codes) + bh * a.T_cap * ROWW;
     const uint32_t* vc_base = reinterpret_cast<const uint32_t*>(a.v_codes) + bh * a.T_cap * ROWW;
     const uint32_t* gents = a.k_out + bh * a.k_out_cap;
@@ -471,6 +554,9 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       bar_arrive(kBarFull + buf, kThr);       // chunk c's tiles are ready
     }
     cp_async_wait<0>();
+    end_unit(bh);
+    x = xe;
+    }
   } else {
     // ======================= consumers: tensor-core attention =======================
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegCons) : "memory");
@@ -480,6 +566,15 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     const int t0w = cw * 16;
     const int tokA = t0w + (mi & 1) * 8 + rowi, chA = mi >> 1;   // K slab as the A operand
     const int tokV = t0w + (mi >> 1) * 8 + rowi, chV = mi & 1;   // V^T slab as the A operand
+    for (int64_t x = x0; x < x1;) {
+      const int64_t bh = x / a.cpu;                           // this segment's unit
+      const int64_t xe = min(x1, (bh + 1) * a.cpu);
+      begin_unit(bh);
+      const int b = (int)(bh / a.Hkv);
+      const int n_len = (int)min((int64_t)a.T_len[b], a.T_cap);
+      const int64_t v_begin = (x - bh * a.cpu) * kChunk;
+      const int64_t v_end = min((xe - bh * a.cpu) * kChunk, (int64_t)n_len);
+      const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
     // o[j] = O^T rows (tile columns) 16j + g and 16j + g + 8, heads 2r and 2r + 1
     float o[D / 16][4];
 #pragma unroll
@@ -634,36 +729,14 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
         }
       }
     }
-  }
-  __syncthreads();
-  for (int e = tid; e < a.G * D; e += kThr) {
-    const int row = e / D, d = e % D;
-    float M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < kConsWarps; ++w) M = fmaxf(M, wm[w * 8 + row]);
-    float L = 0.f, O = 0.f;
-    if (M != -INFINITY) {
-#pragma unroll
-      for (int w = 0; w < kConsWarps; ++w) {
-        const float f = exp2f(wm[w * 8 + row] - M);
-        L += wl[w * 8 + row] * f;
-        O += wo[(w * 8 + row) * D + d] * f;
-      }
-    }
-    const int64_t hq = (int64_t)b * a.Hq + (int64_t)kvh * a.G + row;
-    const int64_t pi = hq * a.n_split + split;
-    a.part_o[pi * D + d] = O;
-    if (d == 0) {
-      a.part_m[pi] = M;
-      a.part_l[pi] = L;
+    end_unit(bh);
+    x = xe;
     }
   }
-  __syncthreads();                     // the stage buffers now serve as the merge's scratch
-  merge_if_last<D, kThr>(a.merge, bh, b, kvh, reinterpret_cast<float*>(stg), Lay::NS * Lay::STAGE / 4);
 }
 
 template <int D, int BITS>
-cudaError_t launch_kvq_t(const KvqArgs& a, int units, int n_split, cudaStream_t st) {
+cudaError_t launch_kvq_t(const KvqArgs& a, cudaStream_t st) {
   using Lay = KvqLayout<D, BITS>;
   static_assert(Lay::BYTES <= 227 * 1024, "one CTA per SM");
   static int checked = 0;                 // 1: attributes set and register count verified
@@ -677,7 +750,7 @@ cudaError_t launch_kvq_t(const KvqArgs& a, int units, int n_split, cudaStream_t 
     if (e != cudaSuccess) return e;
     checked = 1;
   }
-  decode_kvq_kernel<D, BITS><<<dim3(n_split, units), kThr, Lay::BYTES, st>>>(a);
+  decode_kvq_kernel<D, BITS><<<a.n_cta, kThr, Lay::BYTES, st>>>(a);
   return cudaPeekAtLastError();
 }
 
@@ -705,23 +778,24 @@ cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_
   a.Hkv = c.Hkv;
   a.G = c.Hq / c.Hkv;
     a.n_v = std::min(c.D, (int)ceil((double)c.outlier_frac * c.D));
-  a.chunks_per_split = sp.chunks_per_split;
   a.n_split = sp.n_split;
+  a.n_cta = sp.n_cta;
+  a.cpu = sp.chunks_per_unit;
+  a.c_tot = sp.chunks_per_unit * c.B * c.Hkv;
   const float scale = c.softmax_scale > 0.f ? c.softmax_scale : 1.0f / sqrtf((float)c.D);
   a.scale_log2 = scale * kLog2e;
   a.part_m = ws.part_m;
   a.part_l = ws.part_l;
   a.part_o = ws.part_o;
   a.merge = merge_args(c, ws, sp, out, false);
-  const int units = c.B * c.Hkv;
   if (c.D == 128) {
-    if (c.bits == 4) return launch_kvq_t<128, 4>(a, units, sp.n_split, st);
-    if (c.bits == 3) return launch_kvq_t<128, 3>(a, units, sp.n_split, st);
-    return launch_kvq_t<128, 2>(a, units, sp.n_split, st);
+    if (c.bits == 4) return launch_kvq_t<128, 4>(a, st);
+    if (c.bits == 3) return launch_kvq_t<128, 3>(a, st);
+    return launch_kvq_t<128, 2>(a, st);
   }
-  if (c.bits == 4) return launch_kvq_t<64, 4>(a, units, sp.n_split, st);
-  if (c.bits == 3) return launch_kvq_t<64, 3>(a, units, sp.n_split, st);
-  return launch_kvq_t<64, 2>(a, units, sp.n_split, st);
+  if (c.bits == 4) return launch_kvq_t<64, 4>(a, st);
+  if (c.bits == 3) return launch_kvq_t<64, 3>(a, st);
+  return launch_kvq_t<64, 2>(a, st);
 }
 
 }  // namespace mkv

@@ -47,6 +47,20 @@ Split decode_split(const mkv_config& c, int64_t T_cap) {
   }
   s.chunks_per_split = (int)ceil_div(chunks, best_n);
   s.n_split = (int)ceil_div(chunks, s.chunks_per_split);
+  if (c.method == MKV_KVQUANT) {
+    // one CTA per SM, each over an equal range of all units' chunks (at most a few units per
+    // CTA); a unit's partial slots are the CTAs that cover part of it
+    const int64_t c_tot = units * chunks;
+    s.chunks_per_unit = chunks;
+    s.n_cta = (int)std::min<int64_t>(kNumSMs, c_tot);
+    int64_t slots_max = 1;
+    for (int64_t u = 0; u < units; ++u) {
+      const int64_t n = cta_of_chunk((u + 1) * chunks - 1, c_tot, s.n_cta) - cta_of_chunk(u * chunks, c_tot, s.n_cta) + 1;
+      slots_max = std::max(slots_max, n);
+    }
+    s.n_split = (int)slots_max;
+    s.chunks_per_split = (int)chunks;
+  }
   return s;
 }
 

@@ -25,13 +25,22 @@ constexpr int kMaxUnits = (int)(kCounterBytes / 4);
 inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 // Work split of a decode call: `n_split` CTAs per (batch, kv-head), each over
-// `chunks_per_split` chunks of kChunk virtual tokens.
+// `chunks_per_split` chunks of kChunk virtual tokens (KVQuant: a balanced range per CTA).
 struct Split {
-  int n_split;
+  int n_split;           // partial slots per (batch, kv-head)
   int chunks_per_split;
-  int64_t v_tokens;  // virtual tokens per (batch, kv-head)
+  int64_t v_tokens;      // virtual tokens per (batch, kv-head)
+  // KVQuant: one CTA per SM over the concatenated chunks of all (batch, kv-head) units; CTA i
+  // takes chunks [i * c_tot / n_cta, (i + 1) * c_tot / n_cta)
+  int n_cta;
+  int64_t chunks_per_unit;
 };
 Split decode_split(const mkv_config& c, int64_t T_cap);
+// The balanced KVQuant split: CTA of virtual chunk x, first and last CTA of unit u.
+#ifdef __CUDACC__
+__host__ __device__
+#endif
+inline int64_t cta_of_chunk(int64_t x, int64_t c_tot, int64_t n_cta) { return ((x + 1) * n_cta - 1) / c_tot; }
 
 // Workspace carve-up (all float32).  Offsets are 256-byte aligned.
 struct DecodeWs {

@@ -20,28 +20,29 @@ struct MergeArgs {
   int Hq, G, n_split;
 };
 
-// `scratch`: shared memory the caller no longer needs, `cap` floats of it.
+// `scratch`: shared memory the caller no longer needs, `cap` floats of it.  `n_parts`: the
+// partials of this group (slots 0 .. n_parts-1 of a.n_split; default all).
 template <int D, int NT>
 __device__ __forceinline__ void merge_if_last(const MergeArgs& a, int64_t bh, int b, int kvh, float* scratch,
-                                              int cap) {
+                                              int cap, int n_parts = -1) {
   __shared__ int s_last;
   __threadfence();
   __syncthreads();
   if (threadIdx.x == 0) {
     const int t = atomicAdd(&a.counters[bh], 1);
-    s_last = (t == a.n_split - 1);
+    s_last = (t == (n_parts > 0 ? n_parts : a.n_split) - 1);
     if (s_last) a.counters[bh] = 0;
   }
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  const int ns = a.n_split, G = a.G;
+  const int ns = n_parts > 0 ? n_parts : a.n_split, stride = a.n_split, G = a.G;
   const int64_t hq0 = (int64_t)b * a.Hq + (int64_t)kvh * G;
   if (2 * G * ns + 2 * G <= cap) {
     // weights f[row][s] = 2^(m_s - M) and totals, then independent loads of the o partials
     float* f = scratch;                 // [G][ns]
     float* tot = scratch + G * ns;      // [G] M, [G] L
-    for (int e = threadIdx.x; e < G * ns; e += NT) f[e] = __ldcg(a.part_m + hq0 * ns + e);
+    for (int e = threadIdx.x; e < G * ns; e += NT) f[e] = __ldcg(a.part_m + (hq0 + e / ns) * stride + e % ns);
     __syncthreads();
     if (threadIdx.x < G) {
       const int row = threadIdx.x;
@@ -52,7 +53,7 @@ __device__ __forceinline__ void merge_if_last(const MergeArgs& a, int64_t bh, in
         const float ms = f[row * ns + s];
         const float w = (M == -INFINITY || ms == -INFINITY) ? 0.f : exp2f(ms - M);
         f[row * ns + s] = w;
-        L += __ldcg(a.part_l + (hq0 + row) * ns + s) * w;
+        L += __ldcg(a.part_l + (hq0 + row) * stride + s) * w;
       }
       tot[row] = M;
       tot[G + row] = L;
@@ -60,7 +61,7 @@ __device__ __forceinline__ void merge_if_last(const MergeArgs& a, int64_t bh, in
     __syncthreads();
     for (int e = threadIdx.x; e < G * D; e += NT) {
       const int row = e / D, d = e % D;
-      const float* po = a.part_o + ((hq0 + row) * ns) * D + d;
+      const float* po = a.part_o + ((hq0 + row) * stride) * D + d;
       const float* fw = f + row * ns;
       float O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
       int s = 0;
@@ -84,8 +85,8 @@ __device__ __forceinline__ void merge_if_last(const MergeArgs& a, int64_t bh, in
   for (int e = threadIdx.x; e < G * D; e += NT) {      // many splits: direct loop
     const int row = e / D, d = e % D;
     const int64_t hq = hq0 + row;
-    const float* pm = a.part_m + hq * ns;
-    const float* pl = a.part_l + hq * ns;
+    const float* pm = a.part_m + hq * stride;
+    const float* pl = a.part_l + hq * stride;
     float M = -INFINITY;
     for (int s = 0; s < ns; ++s) M = fmaxf(M, __ldcg(pm + s));
     float L = 0.f, O = 0.f;
@@ -95,7 +96,7 @@ __device__ __forceinline__ void merge_if_last(const MergeArgs& a, int64_t bh, in
         if (ms == -INFINITY) continue;
         const float w = exp2f(ms - M);
         L += __ldcg(pl + s) * w;
-        O += __ldcg(a.part_o + (hq * ns + s) * D + d) * w;
+        O += __ldcg(a.part_o + (hq * stride + s) * D + d) * w;
       }
     }
     a.out[hq * D + d] = __float2half_rn(L > 0.f ? O / L : 0.f);
