@@ -246,7 +246,9 @@ mkv_status mkv_append_kv(const mkv_config* cfg, const void* k_new, const void* v
  *                  token (Section 2.1, RocketKV paragraph, second stage).
  * out fp16 [B][Hq][D].  For H2O the call also leaves, in ws, the per-slot
  * logits and per-head softmax statistics that mkv_h2o_update reads.
- * qparams: KVQUANT only (else NULL).  ws/ws_bytes: workspace. */
+ * qparams: KVQUANT only (else NULL).  ws/ws_bytes: workspace.
+ * KVQUANT also requires k_out_cap <= INT32_MAX and T_cap < INT32_MAX
+ * (MKV_ERR_UNSUPPORTED otherwise). */
 mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_cache* cache,
                                 const mkv_quant_params* qparams, const int32_t* page_idx,
                                 void* out, void* ws, size_t ws_bytes, void* stream);

@@ -425,7 +425,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     // ahead of that iteration's chunk copies; those of chunk 0 with chunk 0.
     auto load_entries = [&](int stage, int64_t e0, int64_t e1) {
       const int64_t e = e0 + ptid;
-      const bool ok = e < e1;
+      const bool ok = e >= 0 && e < e1;       // offsets of a corrupted cache stay harmless
       if (ptid < kEnt)
         cp_async4s(stg_s + stage * Lay::STAGE + Lay::S_ENT + ptid * 4, gents + (ok ? e : 0), ok ? 4 : 0);
     };
@@ -600,7 +600,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
         const int E0 = ko[0];
         const int e_lo = ko[t0w], e_hi = (int)min((int64_t)ko[t0w + 16], a.k_out_cap);
         auto fetch = [&](int e) -> uint32_t {
-          if (e >= e_hi) return 0xffff0000u;  // no entry: not a channel
+          if (e < 0 || e >= e_hi) return 0xffff0000u;  // no entry: not a channel
           if (e - E0 < kEnt) return ents[e - E0];
           return __ldg(gents + e);            // beyond the staged entries
         };

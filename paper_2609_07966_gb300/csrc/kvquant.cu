@@ -100,9 +100,20 @@ __global__ void quantize_kernel(const QuantArgs a) {
   if (a.nuq) {
     const uint16_t* kc = a.k_cb + ((int64_t)h * D + c) * K;
     const uint16_t* vc = a.v_cb + ((int64_t)h * D + c) * K;
-    for (int j = 0; j < L; ++j) {
-      kmu[j] = fl32_mid(h2f(kc[j]), h2f(kc[j + 1]));
-      vmu[j] = fl32_mid(h2f(vc[j]), h2f(vc[j + 1]));
+    uint16_t kr[16], vr[16];                 // all codebook loads in flight at once (K <= 16)
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      if (j < K) {
+        kr[j] = __ldg(kc + j);
+        vr[j] = __ldg(vc + j);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 15; ++j) {
+      if (j < L) {
+        kmu[j] = fl32_mid(h2f(kr[j]), h2f(kr[j + 1]));
+        vmu[j] = fl32_mid(h2f(vr[j]), h2f(vr[j + 1]));
+      }
     }
   }
   int32_t* off_row = a.k_out_off + (int64_t)bh * (a.T_cap + 1);
@@ -119,7 +130,8 @@ __global__ void quantize_kernel(const QuantArgs a) {
     int code;
     if (a.nuq) {
       code = 0;
-      for (int j = 0; j < L; ++j) code += (x > kmu[j]) ? 1 : 0;
+#pragma unroll
+      for (int j = 0; j < 15; ++j) code += (j < L && x > kmu[j]) ? 1 : 0;   // registers, no local array
     } else {
       code = uniform_code(x, klo, ksc, L);
     }
@@ -177,7 +189,8 @@ __global__ void quantize_kernel(const QuantArgs a) {
       scale = __fsub_rn(hi, lo);
       const float u = scale == 0.f ? 0.f : __fdiv_rn(__fsub_rn(vx, lo), scale);
       vc = 0;
-      for (int j = 0; j < L; ++j) vc += (u > vmu[j]) ? 1 : 0;
+#pragma unroll
+      for (int j = 0; j < 15; ++j) vc += (j < L && u > vmu[j]) ? 1 : 0;
     } else {
       scale = __fdiv_rn(__fsub_rn(hi, lo), (float)L);
       vc = uniform_code(vx, lo, scale, L);

@@ -344,6 +344,9 @@ mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_
     MKV_TRY(check_qparams(cfg, qparams, true));
     MKV_REQUIRE(qparams->rope && qparams->rope_len >= std::max<int64_t>(cache->T_cap, 64), MKV_ERR_INVALID_ARG,
                 "KVQUANT decode needs a rope table with rope_len >= max(T_cap, 64)");
+    MKV_REQUIRE(cache->k_out_cap <= INT32_MAX && cache->T_cap < INT32_MAX, MKV_ERR_UNSUPPORTED,
+                "KVQUANT decode indexes key outliers and tokens with 32 bits (k_out_cap %lld, T_cap %lld)",
+                (long long)cache->k_out_cap, (long long)cache->T_cap);
   }
   const DecodeWs need = decode_ws(*cfg, cache->T_cap, nullptr);
   MKV_REQUIRE(ws != nullptr && ws_bytes >= need.bytes, MKV_ERR_WORKSPACE,

@@ -237,3 +237,37 @@ def test_quantize_capacity_flag():
 def test_decode_full_size_sampled():
     """B=8, T=8192, 32/8/128, NUQ 4-bit: one layer, every kv-head of batch entries 0 and 7."""
     _decode_vs_oracle(B=8, Hq=32, Hkv=8, D=128, bits=4, mode="nuq", T=8192, steps=1, seed=99, check=(0, 7))
+
+
+def test_decode_many_units_ragged_lengths():
+    """More (batch, kv-head) units than SMs and a different length per batch entry (0 .. T): the
+    CTAs' equal runs of chunks cross unit boundaries, units are merged from several CTAs, and a
+    batch entry with no tokens gets a zero output."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    B, Hq, Hkv, D, bits, T = 40, 8, 4, 64, 3, 150
+    k, v = _data(B, Hkv, T, D, seed=5)
+    plist = _oracle_params(k, v, T, bits, "uniform", 0.01)
+    cfg = make_cfg(B, Hq, Hkv, D, bits, "uniform", 0.01)
+    cache, qp = _quantized_cache(cfg, k, v, plist, T, 0, dev, T_cap=T + 8)
+    lens = [(37 * b) % (T + 1) for b in range(B)]
+    assert 0 in lens and max(lens) > 128
+    cache.t["T_len"].copy_(torch.tensor(lens, dtype=cache.t["T_len"].dtype, device=dev))
+    ws, nws = caches.workspace(cfg, cache.T_cap, device=dev)
+    q = np.random.default_rng(6).standard_normal((B, Hq, D)).astype(np.float16)
+    qt = to_dev(q, dev)
+    out = torch.empty_like(qt)
+    G = Hq // Hkv
+    for rep in range(2):                      # the ticket counters return to zero after a call
+        mkv.mkv_decode_attention(cfg, qt.data_ptr(), cache.c, qp.c, 0, out.data_ptr(), ws.data_ptr(), nws)
+        got = out.float().cpu().numpy()
+        for b in range(B):
+            n = lens[b]
+            for h in range(Hkv):
+                rows = got[b, h * G:(h + 1) * G]
+                if n == 0:
+                    assert np.all(rows == 0.0), f"empty b{b} h{h}"
+                    continue
+                qh = kvquant.quantize_head(k[b, h, :n], v[b, h, :n], plist[h])
+                ref = kvquant.decode_head(q[b, h * G:(h + 1) * G], qh, plist[h], cfg.rope_theta)
+                assert_close(rows, ref, f"call {rep} b{b} h{h} n{n}")
