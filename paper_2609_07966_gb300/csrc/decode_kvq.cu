@@ -465,10 +465,12 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       const int32_t my_ko = ptid <= kChunk ? koff[ptid] : 0;
       const float2 qcs = reinterpret_cast<const float2*>(st + Lay::S_RT)[qi];
       uint32_t vo[Lay::NVS];
+      const int n_vs = stage_vout ? a.n_v : 0;  // staged value outliers of a token
 #pragma unroll
-      for (int k = 0; k < Lay::NVS; ++k)
-        vo[k] = (stage_vout && k < a.n_v) ? reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[k * kChunk + tok]
-                                          : 0xffff0000u;
+      for (int k = 0; k < Lay::NVS; ++k) {
+        if (k >= n_vs) break;
+        vo[k] = reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[k * kChunk + tok];
+      }
       if (c >= 2) bar_sync(kBarEmpty + buf, kThr);   // attention on chunk c-2 released the buffer
       uint8_t* B_ = bufs + buf * Lay::BUF;
       uint8_t* khi_t = B_ + Lay::B_KHI;
@@ -539,14 +541,17 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
         auto put = [&](uint32_t ev) {
           const int chn = (int)(ev >> 16);
           const int i = chn < NP ? chn : chn - NP;
-          if (chn < D && i / QP == grp) {
+          if ((unsigned)(i - grp * QP) < (unsigned)QP && chn < D) {
             const int col = 2 * i + (chn >= NP ? 1 : 0);
             *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(tok, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
           }
         };
         if (stage_vout) {
 #pragma unroll
-          for (int k = 0; k < Lay::NVS; ++k) put(vo[k]);
+          for (int k = 0; k < Lay::NVS; ++k) {
+            if (k >= n_vs) break;
+            put(vo[k]);
+          }
         } else {
           for (int k = 0; k < a.n_v; ++k) put(__ldg(a.v_out + (bh * a.T_cap + t0 + tok) * a.n_v + k));
         }
