@@ -67,7 +67,7 @@ __host__ __device__ constexpr int a16(int x) { return (x + 15) & ~15; }
 
 // Shared-memory layout (bytes); every region 16-byte aligned.  `rs` = halves per bounds row.
 struct RfLayout {
-  int qs, sc, kf, part, sel, bounds, pages, wpart, cpart, bytes;
+  int qs, sc, kf, part, sel, bounds, pages, wpart, cpart, tail, bytes;
   __host__ __device__ RfLayout(int D, int G, int64_t npc, int kp, int rs) {
     qs = 0;                                              // float [G][D]
     sc = a16(qs + G * D * 4);                            // float [npc rounded to 4] page scores
@@ -81,6 +81,8 @@ struct RfLayout {
     cpart = bounds;
     bytes = pages + kRfWarps * 2 * kPage * D * 2;        // per warp: K and V tiles of one page
     if (wpart + kRfWarps * G * (D + 2) * 4 > bytes) bytes = wpart + kRfWarps * G * (D + 2) * 4;
+    tail = a16(bytes);                                   // K and V tiles of the newest token's page
+    bytes = tail + 2 * kPage * D * 2;
   }
 };
 
@@ -125,6 +127,16 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
   const int sp = (int)((a.npc + kCl - 1) / kCl);        // pages per CTA
   const int p0 = min((int)a.npc, rank * sp), npf = min((int)a.npc, p0 + sp) - p0;
 
+  // the group's query (fp16) and the cache length, loaded before the prefetch is issued
+  constexpr int kQW = (8 * D / 2 + kRfThreads - 1) / kRfThreads;   // query words per thread (G <= 8)
+  const uint32_t* qg = reinterpret_cast<const uint32_t*>(a.q + ((int64_t)b * a.Hq + (int64_t)kvh * G) * D);
+  uint32_t qw[kQW];
+#pragma unroll
+  for (int k = 0; k < kQW; ++k) {
+    const int e = tid + k * kRfThreads;
+    qw[k] = e < G * (D / 2) ? __ldg(qg + e) : 0u;
+  }
+  const int n = (int)min((int64_t)__ldg(a.T_len + b), a.T_cap);
   // ---- 1. prefetch every dim's bounds of this CTA's pages (16-byte copies from the row start
   // rounded down to 16 bytes, the last one cut at the end of the pages)
   if (npf > 0) {
@@ -142,15 +154,35 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
       }
     }
   }
+  // the newest token's page, always attended, is staged now by the warp that attends to it
+  const int ns = n > 0 ? (n - 1) / kPage : 0;          // candidate (full) pages; page ns is the newest
+  const bool tail_warp = rank == kCl - 1 && warp == kRfWarps - 1 && n > 0;
+  const int tail_valid = n - ns * kPage;               // 1 .. 16 rows
+  uint8_t* tk = smem + L.tail;
+  uint8_t* tv = tk + kPage * D * 2;
+  if (tail_warp) {
+    const __half* kb = a.k + (bh * a.T_cap + (int64_t)ns * kPage) * D;
+    const __half* vb = a.v + (bh * a.T_cap + (int64_t)ns * kPage) * D;
+    for (int e = lane; e < 2 * kPage * (D / 8); e += 32) {
+      const int kv = e / (kPage * (D / 8)), rem = e % (kPage * (D / 8));
+      const int row = rem / (D / 8), ch = rem % (D / 8);
+      const bool ok = row < tail_valid;
+      cp_async16((kv ? tv : tk) + tile_off<D>(row, ch), (kv ? vb : kb) + (ok ? row : 0) * D + ch * 8, ok ? 16 : 0);
+    }
+  }
   cp_async_commit();
-  const int n = (int)min((int64_t)a.T_len[b], a.T_cap);
-  const int ns = n > 0 ? (n - 1) / kPage : 0;          // candidate (full) pages
   const int np = max(0, min(ns, p0 + sp) - p0);        // of them, this CTA's
-  for (int e = tid; e < G * D; e += kRfThreads)
-    qs[e] = __half2float(a.q[((int64_t)b * a.Hq + (int64_t)kvh * G) * D + e]);
-  for (int e = tid; e < G * (D / 2); e += kRfThreads)
-    qh2[e / (D / 2)][e % (D / 2)] =
-        reinterpret_cast<const uint32_t*>(a.q + ((int64_t)b * a.Hq + (int64_t)kvh * G) * D)[e];
+#pragma unroll
+  for (int k = 0; k < kQW; ++k) {
+    const int e = tid + k * kRfThreads;
+    if (e < G * (D / 2)) {
+      const int row = e / (D / 2), w = e % (D / 2);
+      qh2[row][w] = qw[k];
+      const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&qw[k]));
+      qs[row * D + 2 * w] = f.x;
+      qs[row * D + 2 * w + 1] = f.y;
+    }
+  }
   __syncthreads();
   if (tid < D) {
     float s = 0.f;
@@ -211,18 +243,20 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
   for (int p = ns + tid; p < ((ns + 3) & ~3); p += kRfThreads) sc[p] = -INFINITY;   // local pads
   cluster_sync();
 
-  // ---- 3. each CTA ranks its own pages against all scores under (score desc, page asc),
-  // eight threads per page each counting over an eighth of the pages, and stores the kept flags
-  // into every CTA; then thread t takes a contiguous run of pages so that the kept pages come
-  // out in ascending order from one block scan
+  // ---- 3. CTA r ranks the r-th run of ceil(ns / kCl) candidate pages against all scores under
+  // (score desc, page asc), eight threads per page each counting over an eighth of the pages,
+  // and stores the kept flags into every CTA; then thread t takes a contiguous run of pages so
+  // that the kept pages come out in ascending order from one block scan
   const int k = min(a.kp, ns);
   const int seg = ((ns + 7) / 8 + 3) & ~3;              // pages per counting segment (multiple of 4)
-  for (int base = 0; base < np * 8; base += kRfThreads) {   // uniform trip count: shuffles below
+  const int rp = (ns + kCl - 1) / kCl;                 // pages ranked per CTA
+  const int r0 = rank * rp, nr = max(0, min(ns, r0 + rp) - r0);
+  for (int base = 0; base < nr * 8; base += kRfThreads) {   // uniform trip count: shuffles below
     const int task = base + tid;
     const int pl = task >> 3, sg = task & 7;
     int rk = 0;
-    if (pl < np) {
-      const int p = p0 + pl;
+    if (pl < nr) {
+      const int p = r0 + pl;
       const float s = sc[p];
       const int j1 = min(ns, (sg + 1) * seg);
       for (int j = sg * seg; j < j1; j += 4) {        // scores are padded to a multiple of four
@@ -234,7 +268,7 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
     rk += __shfl_xor_sync(0xffffffffu, rk, 1);
     rk += __shfl_xor_sync(0xffffffffu, rk, 2);
     rk += __shfl_xor_sync(0xffffffffu, rk, 4);
-    if (pl < np && sg < kCl) st_cluster_u8(cluster_addr(kf + p0 + pl, sg), rk < k ? 1u : 0u);
+    if (pl < nr && sg < kCl) st_cluster_u8(cluster_addr(kf + r0 + pl, sg), rk < k ? 1u : 0u);
   }
   cluster_sync();
   const int ppt = (ns + kRfThreads - 1) / kRfThreads;
@@ -251,11 +285,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
   int pos = block_exclusive_scan(cnt, warp_sums, &total);
   for (int u = 0; u < ppt; ++u)
     if (keep_bits & (1u << u)) sel[pos++] = tid * ppt + u;
-  if (tid == 0) sel[total] = ns;                       // the newest token's page, always attended
   __syncthreads();
   if (rank == 0 && a.page_idx != nullptr)
     for (int i = tid; i < a.kp; i += kRfThreads) a.page_idx[bh * a.kp + i] = i < total ? sel[i] : -1;
-  const int n_att = n > 0 ? total + 1 : 0;             // pages attended
+  const int n_att = n > 0 ? total : 0;                 // chosen pages attended (and the newest one)
 
   // ---- 4. attention: page i goes to CTA i % kCl, warp (i / kCl) % kRfWarps
   const int g = lane >> 2, r = lane & 3;
@@ -271,69 +304,87 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
   const int tokk = (mi >> 1) * 8 + rowi, tokv = (mi & 1) * 8 + rowi;
   const __half* kbase = a.k + bh * a.T_cap * D;
   const __half* vbase = a.v + bh * a.T_cap * D;
-  for (int i = rank + kCl * warp; i < n_att; i += kCl * kRfWarps) {
-    const int page = sel[i];
-    const int valid = min(kPage, n - page * kPage);    // 16, or the newest page's length
+  // QK^T, online softmax and PV of the group's heads on one page's K and V tiles (16 rows)
+  auto attend = [&](const uint8_t* kt_, const uint8_t* vt_, int valid) {
+      float s[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+#pragma unroll
+      for (int kc = 0; kc < KC; ++kc) {
+        uint32_t bk[4];
+        ldsm_x4(bk, kt_ + tile_off<D>(tokk, kc * 2 + (mi & 1)));
+        const uint32_t a0 = real ? qrow[kc * 8 + r] : 0u, a2 = real ? qrow[kc * 8 + 4 + r] : 0u;
+        mma16816(s[0], a0, 0u, a2, 0u, bk[0], bk[1]);
+        mma16816(s[1], a0, 0u, a2, 0u, bk[2], bk[3]);
+      }
+      const int tk[4] = {2 * r, 2 * r + 1, 8 + 2 * r, 9 + 2 * r};
+      float x[4] = {s[0][0], s[0][1], s[1][0], s[1][1]};
+      float mx = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        x[j] = tk[j] < valid ? x[j] * a.scale_log2 : -INFINITY;
+        mx = fmaxf(mx, x[j]);
+      }
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+      const float m_new = fmaxf(m_run, mx);
+      float p[4] = {0.f, 0.f, 0.f, 0.f};
+      float alpha = 1.f;
+      if (m_new != -INFINITY) {
+        alpha = exp2f(m_run - m_new);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) p[j] = exp2f(x[j] - m_new);
+      }
+      l_part = l_part * alpha + (p[0] + p[1]) + (p[2] + p[3]);
+      m_run = m_new;
+#pragma unroll
+      for (int j = 0; j < D / 8; ++j) {
+        o[j][0] *= alpha;
+        o[j][1] *= alpha;
+      }
+      const uint32_t pa0 = pack_half2(p[0], p[1]);
+      const uint32_t pa2 = pack_half2(p[2], p[3]);
+#pragma unroll
+      for (int j = 0; j < D / 16; ++j) {
+        uint32_t bv[4];
+        ldsm_x4_t(bv, vt_ + tile_off<D>(tokv, 2 * j + (mi >> 1)));
+        float d0[4] = {o[2 * j][0], o[2 * j][1], 0.f, 0.f};
+        float d1[4] = {o[2 * j + 1][0], o[2 * j + 1][1], 0.f, 0.f};
+        mma16816(d0, pa0, 0u, pa2, 0u, bv[0], bv[1]);
+        mma16816(d1, pa0, 0u, pa2, 0u, bv[2], bv[3]);
+        o[2 * j][0] = d0[0];
+        o[2 * j][1] = d0[1];
+        o[2 * j + 1][0] = d1[0];
+        o[2 * j + 1][1] = d1[1];
+      }
+  };
+  // This warp's pages: chosen page i = rank + kCl * warp (+ kCl * kRfWarps ...), and for the
+  // designated warp first the newest page, staged at the start, attended while the copies of its
+  // first chosen page are in flight.  One call site of attend().
+  auto load_page = [&](int i) {
+    const int page = sel[i];                           // a full page
     for (int e = lane; e < 2 * kPage * (D / 8); e += 32) {
       const int kv = e / (kPage * (D / 8)), rem = e % (kPage * (D / 8));
       const int row = rem / (D / 8), ch = rem % (D / 8);
-      const bool ok = row < valid;
-      const int64_t src = ((int64_t)page * kPage + (ok ? row : 0)) * D + ch * 8;
-      cp_async16((kv ? vt : kt) + tile_off<D>(row, ch), (kv ? vbase : kbase) + src, ok ? 16 : 0);
+      cp_async16((kv ? vt : kt) + tile_off<D>(row, ch), (kv ? vbase : kbase) + ((int64_t)page * kPage + row) * D + ch * 8, 16);
     }
     cp_async_commit();
-    cp_async_wait<0>();
-    __syncwarp();
-    float s[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
-#pragma unroll
-    for (int kc = 0; kc < KC; ++kc) {
-      uint32_t bk[4];
-      ldsm_x4(bk, kt + tile_off<D>(tokk, kc * 2 + (mi & 1)));
-      const uint32_t a0 = real ? qrow[kc * 8 + r] : 0u, a2 = real ? qrow[kc * 8 + 4 + r] : 0u;
-      mma16816(s[0], a0, 0u, a2, 0u, bk[0], bk[1]);
-      mma16816(s[1], a0, 0u, a2, 0u, bk[2], bk[3]);
+  };
+  int i = rank + kCl * warp;
+  if (i < n_att) load_page(i);
+  bool tail_left = tail_warp;
+  while (tail_left || i < n_att) {
+    const bool tail_now = tail_left;
+    if (!tail_now) {
+      cp_async_wait<0>();
+      __syncwarp();
     }
-    const int tk[4] = {2 * r, 2 * r + 1, 8 + 2 * r, 9 + 2 * r};
-    float x[4] = {s[0][0], s[0][1], s[1][0], s[1][1]};
-    float mx = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      x[j] = tk[j] < valid ? x[j] * a.scale_log2 : -INFINITY;
-      mx = fmaxf(mx, x[j]);
+    attend(tail_now ? tk : kt, tail_now ? tv : vt, tail_now ? tail_valid : kPage);
+    if (tail_now) {
+      tail_left = false;
+    } else {
+      __syncwarp();                                    // the tiles are reloaded next page
+      i += kCl * kRfWarps;
+      if (i < n_att) load_page(i);
     }
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-    const float m_new = fmaxf(m_run, mx);
-    float p[4] = {0.f, 0.f, 0.f, 0.f};
-    float alpha = 1.f;
-    if (m_new != -INFINITY) {
-      alpha = exp2f(m_run - m_new);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) p[j] = exp2f(x[j] - m_new);
-    }
-    l_part = l_part * alpha + (p[0] + p[1]) + (p[2] + p[3]);
-    m_run = m_new;
-#pragma unroll
-    for (int j = 0; j < D / 8; ++j) {
-      o[j][0] *= alpha;
-      o[j][1] *= alpha;
-    }
-    const uint32_t pa0 = pack_half2(p[0], p[1]);
-    const uint32_t pa2 = pack_half2(p[2], p[3]);
-#pragma unroll
-    for (int j = 0; j < D / 16; ++j) {
-      uint32_t bv[4];
-      ldsm_x4_t(bv, vt + tile_off<D>(tokv, 2 * j + (mi >> 1)));
-      float d0[4] = {o[2 * j][0], o[2 * j][1], 0.f, 0.f};
-      float d1[4] = {o[2 * j + 1][0], o[2 * j + 1][1], 0.f, 0.f};
-      mma16816(d0, pa0, 0u, pa2, 0u, bv[0], bv[1]);
-      mma16816(d1, pa0, 0u, pa2, 0u, bv[2], bv[3]);
-      o[2 * j][0] = d0[0];
-      o[2 * j][1] = d0[1];
-      o[2 * j + 1][0] = d1[0];
-      o[2 * j + 1][1] = d1[1];
-    }
-    __syncwarp();                                      // the tiles are reloaded next page
   }
   __syncthreads();                                     // every warp is done with its tiles
 
