@@ -20,12 +20,17 @@ __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits
                                                 int32_t* __restrict__ slot_out, int64_t bh) {
   const int b = (int)(bh / Hkv), kvh = (int)(bh % Hkv);
   const int64_t newest = (int64_t)T_len[b] - 1;
-  float m[8], il[8];
-  for (int h = 0; h < G; ++h) {
-    const int64_t hq = (int64_t)b * Hkv * G + (int64_t)kvh * G + h;
-    m[h] = __ldcg(m_tot + hq);
-    const float l = __ldcg(l_tot + hq);
-    il[h] = l > 0.f ? 1.f / l : 0.f;
+  float m[8], il[8];                  // G <= 8; unrolled so both stay in registers
+#pragma unroll
+  for (int h = 0; h < 8; ++h) {
+    m[h] = 0.f;
+    il[h] = 0.f;
+    if (h < G) {
+      const int64_t hq = (int64_t)b * Hkv * G + (int64_t)kvh * G + h;
+      m[h] = __ldcg(m_tot + hq);
+      const float l = __ldcg(l_tot + hq);
+      il[h] = l > 0.f ? 1.f / l : 0.f;
+    }
   }
   int held = 0;
   uint64_t best = ~0ull;          // minimum key among candidates -> evicted
@@ -51,7 +56,9 @@ __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits
           add[u] = exp2f(x.x - m[0]) * il[0] + exp2f(x.y - m[1]) * il[1] + exp2f(x.z - m[2]) * il[2] +
                    exp2f(x.w - m[3]) * il[3];
         } else {
-          for (int h = 0; h < G; ++h) add[u] += exp2f(__ldcg(lg + h) - m[h]) * il[h];
+#pragma unroll
+          for (int h = 0; h < 8; ++h)
+            if (h < G) add[u] += exp2f(__ldcg(lg + h) - m[h]) * il[h];
         }
       }
     }
@@ -96,17 +103,22 @@ __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits
     s_slot[warp] = best_slot;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    int hsum = 0, ff = INT32_MAX, bs = -1;
-    uint64_t bk = ~0ull;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
-      hsum += s_held[w];
-      ff = min(ff, s_free[w]);
-      if (s_key[w] < bk) {
-        bk = s_key[w];
-        bs = s_slot[w];
+  if (warp == 0) {                    // the warps' results, reduced by warp 0
+    const int nw = (int)(blockDim.x >> 5);
+    int hsum = lane < nw ? s_held[lane] : 0, ff = lane < nw ? s_free[lane] : INT32_MAX;
+    uint64_t bk = lane < nw ? s_key[lane] : ~0ull;
+    int bs = lane < nw ? s_slot[lane] : -1;
+    for (int o = 16; o > 0; o >>= 1) {
+      hsum += __shfl_xor_sync(0xffffffffu, hsum, o);
+      ff = min(ff, __shfl_xor_sync(0xffffffffu, ff, o));
+      const uint64_t ok = __shfl_xor_sync(0xffffffffu, bk, o);
+      const int os = __shfl_xor_sync(0xffffffffu, bs, o);
+      if (ok < bk) {
+        bk = ok;
+        bs = os;
       }
     }
+    if (lane != 0) return;
     if (hsum > H + R && bs >= 0) {
       pos[bh * T_cap + bs] = -1;
       slot_out[bh] = bs;
