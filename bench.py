@@ -204,6 +204,13 @@ class Runner:
         (update scores)."""
         mkv = self.mkv
         cache, _ = self.layers[l]
+        if self.method == "rocket":           # append, page choice and attention in one launch
+            kn = self.kn[l] if kn is None else kn
+            vn = self.vn[l] if vn is None else vn
+            q = self.q[l] if q is None else q
+            out = self.out[l] if out is None else out
+            mkv.mkv_rocket_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, 0, out.data_ptr())
+            return
         self.append(l, kn, vn)
         self.decode(l, q, out)
         if self.method == "h2o":
@@ -233,9 +240,9 @@ class Runner:
             self.step()
 
     def launches_per_step(self):
-        # per layer: append (KVQuant: quantize + length advance), decode (RocketKV: page choice
-        # and attention fused), (H2O: score update)
-        per = {"fp16": 2, "kvquant": 3, "h2o": 3, "rocket": 2}[self.method]
+        # per layer: append (KVQuant: quantize + length advance), decode, (H2O: score update);
+        # RocketKV: append, page choice and attention in one launch
+        per = {"fp16": 2, "kvquant": 3, "h2o": 3, "rocket": 1}[self.method]
         return per * self.w.L
 
     def decode_bytes(self):

@@ -362,6 +362,19 @@ mkv_status mkv_rocket_select(const mkv_config* cfg, const void* q, const mkv_cac
 mkv_status mkv_rocket_decode(const mkv_config* cfg, const void* q, const mkv_cache* cache,
                              int32_t* page_idx_out, void* out, void* stream);
 
+/* A whole RocketKV decode step in one launch: mkv_append_kv of the step's
+ * token followed by mkv_rocket_decode, with the same cache contents, page
+ * choice and output.  k_new, v_new fp16 [B][Hkv][D] (post-rotation keys),
+ * 16-byte aligned (MKV_ERR_INVALID_ARG otherwise).
+ * While the launch runs, the top 8 bits of T_len[b] count its finished CTAs
+ * (the last one stores the new length), so nothing else may read or write
+ * T_len of this cache during the call.  A batch entry whose cache is full is
+ * not appended (MKV_FLAG_CACHE_FULL, read by mkv_get_status) and attends to
+ * its existing tokens.  MKV_ERR_UNSUPPORTED as mkv_rocket_decode, and when
+ * T_cap >= 2^24 or 8 * Hkv > 256. */
+mkv_status mkv_rocket_step(const mkv_config* cfg, const void* q, const void* k_new, const void* v_new,
+                           mkv_cache* cache, int32_t* page_idx_out, void* out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

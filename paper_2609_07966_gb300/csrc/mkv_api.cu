@@ -315,6 +315,7 @@ mkv_status mkv_get_status(void* stream, uint32_t* flags) {
   *flags = 0;
   MKV_CUDA(take_status_append(flags, as_stream(stream)));
   MKV_CUDA(take_status_kvquant(flags, as_stream(stream)));
+  MKV_CUDA(take_status_rocket(flags, as_stream(stream)));
   if (*flags != 0) {
     set_error("device status flags 0x%x", *flags);
     return MKV_ERR_CAPACITY;
@@ -467,7 +468,25 @@ mkv_status mkv_rocket_decode(const mkv_config* cfg, const void* q, const mkv_cac
   MKV_REQUIRE(rocket_fused_smem(*cfg, cache->T_cap) <= 227 * 1024, MKV_ERR_UNSUPPORTED,
               "T_cap = %lld is too long for the fused step; use mkv_rocket_select + mkv_decode_attention",
               (long long)cache->T_cap);
-  MKV_CUDA(launch_rocket_fused(*cfg, q, *cache, page_idx_out, out, as_stream(stream)));
+  MKV_CUDA(launch_rocket_fused(*cfg, q, *cache, page_idx_out, out, nullptr, nullptr, as_stream(stream)));
+  return MKV_OK;
+}
+
+mkv_status mkv_rocket_step(const mkv_config* cfg, const void* q, const void* k_new, const void* v_new,
+                           mkv_cache* cache, int32_t* page_idx_out, void* out, void* stream) {
+  MKV_TRY(check_config(cfg));
+  MKV_REQUIRE(cfg->method == MKV_ROCKET, MKV_ERR_INVALID_ARG, "rocket_step is for ROCKET");
+  MKV_TRY(check_cache(cfg, cache));
+  MKV_REQUIRE(q && out && k_new && v_new, MKV_ERR_INVALID_ARG, "q/out/k_new/v_new NULL");
+  MKV_REQUIRE(((uintptr_t)k_new | (uintptr_t)v_new) % 16 == 0, MKV_ERR_INVALID_ARG,
+              "k_new/v_new must be 16-byte aligned (the step reads them in 16-byte pieces)");
+  MKV_REQUIRE(rocket_fused_smem(*cfg, cache->T_cap) <= 227 * 1024, MKV_ERR_UNSUPPORTED,
+              "T_cap = %lld is too long for the fused step; use the separate calls", (long long)cache->T_cap);
+  // the launch counts its finished CTAs per batch entry in the top 8 bits of T_len[b]
+  MKV_REQUIRE(cache->T_cap < (1 << 24) && (int64_t)kRocketCluster * cfg->Hkv <= 256, MKV_ERR_UNSUPPORTED,
+              "rocket_step needs T_cap < 2^24 and 8 * Hkv <= 256 (T_cap %lld, Hkv %d)", (long long)cache->T_cap,
+              cfg->Hkv);
+  MKV_CUDA(launch_rocket_fused(*cfg, q, *cache, page_idx_out, out, k_new, v_new, as_stream(stream)));
   return MKV_OK;
 }
 

@@ -108,8 +108,10 @@ cudaError_t launch_rocket_select(const mkv_config& c, const void* q, const mkv_c
                                  int32_t* page_idx, cudaStream_t st);
 // Fused RocketKV step (page choice + sparse attention, one cluster per (batch, kv-head)).
 size_t rocket_fused_smem(const mkv_config& c, int64_t T_cap);
+// k_new / v_new: the step's token, appended by the same launch (null: no append).
 cudaError_t launch_rocket_fused(const mkv_config& c, const void* q, const mkv_cache& cache, int32_t* page_idx,
-                                void* out, cudaStream_t st);
+                                void* out, const void* k_new, const void* v_new, cudaStream_t st);
+constexpr int kRocketCluster = 8;   // CTAs of the fused step per (batch, kv-head)
 
 // Host-side argument checks of an FP16 decode call (config, cache, q/out pointers).
 mkv_status check_fp16_decode_args(const mkv_config* cfg, const mkv_cache* cache, const void* q, const void* out);
@@ -117,5 +119,6 @@ mkv_status check_fp16_decode_args(const mkv_config* cfg, const mkv_cache* cache,
 // Status word accessors (one per translation unit that can set a flag).
 cudaError_t take_status_kvquant(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_append(uint32_t* flags, cudaStream_t st);
+cudaError_t take_status_rocket(uint32_t* flags, cudaStream_t st);
 
 }  // namespace mkv

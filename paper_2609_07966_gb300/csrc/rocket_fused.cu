@@ -20,6 +20,13 @@
 //     shared memory), and after a cluster barrier CTA 0 merges the kCl partials and writes
 //     the output.
 // No workspace, no global round trip of scores, page ids or partials.
+//
+// With k_new / v_new (mkv_rocket_step) the launch also appends the step's token first, as
+// mkv_append_kv does: every CTA takes the length as T_len + 1, the warp that stages the newest
+// page takes the new row from the input and writes it into the cache, completes the page's
+// per-dim min/max when the row fills it, and the last CTA of the batch entry to finish stores
+// the new length.  During the launch the top 8 bits of T_len[b] count the finished CTAs of
+// batch entry b (every reader masks them off); the last one writes the clean length.
 #include <math.h>
 
 #include "mkv_common.cuh"
@@ -28,9 +35,11 @@
 
 namespace mkv {
 
+__device__ uint32_t g_status_rocket;   // MKV_FLAG_* bits raised by this unit
+
 namespace {
 
-constexpr int kCl = 8;              // CTAs per (batch, kv-head)
+constexpr int kCl = kRocketCluster;  // CTAs per (batch, kv-head)
 constexpr int kRfWarps = 8;
 constexpr int kRfThreads = kRfWarps * 32;
 constexpr int kRfSlices = 8;        // dim slices of the page scoring
@@ -88,11 +97,13 @@ struct RfLayout {
 
 struct RfArgs {
   const __half* q;          // [B][Hq][D]
-  const __half* k;          // [B][Hkv][T_cap][D]
-  const __half* v;
-  const __half* kmin;       // [B][Hkv][D][npc]
-  const __half* kmax;
-  const int32_t* T_len;
+  __half* k;                // [B][Hkv][T_cap][D]
+  __half* v;
+  __half* kmin;             // [B][Hkv][D][npc]
+  __half* kmax;
+  int32_t* T_len;           // low 24 bits: length; top 8: finished CTAs during an appending launch
+  const __half* k_new;      // [B][Hkv][D], or null: no append
+  const __half* v_new;
   int64_t T_cap, npc;
   int Hq, Hkv, G, kp, rd, rs;
   float scale_log2;
@@ -136,7 +147,10 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
     const int e = tid + k * kRfThreads;
     qw[k] = e < G * (D / 2) ? __ldg(qg + e) : 0u;
   }
-  const int n = (int)min((int64_t)__ldg(a.T_len + b), a.T_cap);
+  const bool append = a.k_new != nullptr;
+  const int n_old = (int)min((int64_t)(a.T_len[b] & 0xffffff), a.T_cap);
+  const bool room = append && (int64_t)n_old + 1 <= a.T_cap;
+  const int n = room ? n_old + 1 : n_old;              // the step's token included
   // ---- 1. prefetch every dim's bounds of this CTA's pages (16-byte copies from the row start
   // rounded down to 16 bytes, the last one cut at the end of the pages)
   if (npf > 0) {
@@ -163,11 +177,21 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
   if (tail_warp) {
     const __half* kb = a.k + (bh * a.T_cap + (int64_t)ns * kPage) * D;
     const __half* vb = a.v + (bh * a.T_cap + (int64_t)ns * kPage) * D;
+    const int new_row = room ? tail_valid - 1 : kPage;  // the appended token's row (from the input)
     for (int e = lane; e < 2 * kPage * (D / 8); e += 32) {
       const int kv = e / (kPage * (D / 8)), rem = e % (kPage * (D / 8));
       const int row = rem / (D / 8), ch = rem % (D / 8);
       const bool ok = row < tail_valid;
-      cp_async16((kv ? tv : tk) + tile_off<D>(row, ch), (kv ? vb : kb) + (ok ? row : 0) * D + ch * 8, ok ? 16 : 0);
+      const __half* src = row == new_row ? (kv ? a.v_new : a.k_new) + bh * D + ch * 8
+                                         : (kv ? vb : kb) + (ok ? row : 0) * D + ch * 8;
+      cp_async16((kv ? tv : tk) + tile_off<D>(row, ch), src, ok ? 16 : 0);
+    }
+    if (room) {                                        // the new row into the cache
+      for (int e = lane; e < 2 * (D / 8); e += 32) {
+        const int kv = e / (D / 8), ch = e % (D / 8);
+        const uint4 x = __ldg(reinterpret_cast<const uint4*>((kv ? a.v_new : a.k_new) + bh * D) + ch);
+        reinterpret_cast<uint4*>((kv ? a.v : a.k) + (bh * a.T_cap + (int64_t)n_old) * D)[ch] = x;
+      }
     }
   }
   cp_async_commit();
@@ -445,6 +469,29 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
       a.out[((int64_t)b * a.Hq + (int64_t)kvh * G + row) * D + d] = __float2half_rn(Lsum > 0.f ? O / Lsum : 0.f);
     }
   }
+  if (!append) return;
+  // the appended token filled its page: the page's per-dim min and max, from the staged tiles
+  if (tail_warp && room && n % kPage == 0) {
+    for (int d = lane; d < D; d += 32) {
+      const int off = tile_off<D>(0, d / 8) + (d % 8) * 2;
+      __half lo = *reinterpret_cast<const __half*>(tk + off), hi = lo;
+      for (int row = 1; row < kPage; ++row) {
+        const __half x = *reinterpret_cast<const __half*>(tk + tile_off<D>(row, d / 8) + (d % 8) * 2);
+        lo = __hlt(x, lo) ? x : lo;
+        hi = __hgt(x, hi) ? x : hi;
+      }
+      a.kmin[(bh * D + d) * a.npc + ns] = lo;
+      a.kmax[(bh * D + d) * a.npc + ns] = hi;
+    }
+  }
+  // every thread of this CTA read T_len before this point; the last CTA of batch entry b (all
+  // kCl CTAs of its Hkv clusters) stores the new length and clears the count
+  __syncthreads();
+  if (tid == 0) {
+    const unsigned old = atomicAdd(reinterpret_cast<unsigned*>(a.T_len) + b, 1u << 24);
+    if ((int)(old >> 24) == kCl * a.Hkv - 1) a.T_len[b] = n;
+    if (!room && rank == 0 && kvh == 0) atomicOr(&g_status_rocket, MKV_FLAG_CACHE_FULL);
+  }
 }
 
 template <int D>
@@ -465,14 +512,16 @@ size_t rocket_fused_smem(const mkv_config& c, int64_t T_cap) {
 }
 
 cudaError_t launch_rocket_fused(const mkv_config& c, const void* q, const mkv_cache& cache, int32_t* page_idx,
-                                void* out, cudaStream_t st) {
+                                void* out, const void* k_new, const void* v_new, cudaStream_t st) {
   RfArgs a{};
   a.q = static_cast<const __half*>(q);
-  a.k = static_cast<const __half*>(cache.k);
-  a.v = static_cast<const __half*>(cache.v);
-  a.kmin = static_cast<const __half*>(cache.kmin);
-  a.kmax = static_cast<const __half*>(cache.kmax);
+  a.k = static_cast<__half*>(cache.k);
+  a.v = static_cast<__half*>(cache.v);
+  a.kmin = static_cast<__half*>(cache.kmin);
+  a.kmax = static_cast<__half*>(cache.kmax);
   a.T_len = cache.T_len;
+  a.k_new = static_cast<const __half*>(k_new);
+  a.v_new = static_cast<const __half*>(v_new);
   a.T_cap = cache.T_cap;
   a.npc = cache.T_cap / kPage;
   a.Hq = c.Hq;
@@ -489,6 +538,15 @@ cudaError_t launch_rocket_fused(const mkv_config& c, const void* q, const mkv_ca
   const size_t smem = rocket_fused_smem(c, cache.T_cap);
   const int units = c.B * c.Hkv;
   return c.D == 128 ? launch_rf_t<128>(a, units, smem, st) : launch_rf_t<64>(a, units, smem, st);
+}
+
+cudaError_t take_status_rocket(uint32_t* flags, cudaStream_t st) {
+  uint32_t zero = 0, v = 0;
+  cudaError_t e = cudaMemcpyFromSymbolAsync(&v, g_status_rocket, sizeof(v), 0, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemcpyToSymbolAsync(g_status_rocket, &zero, sizeof(zero), 0, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  *flags |= v;
+  return e;
 }
 
 }  // namespace mkv

@@ -121,3 +121,21 @@ def test_rocket_fused_step_checks(L):
     cache.T_cap = 1 << 20                              # 65536 pages: beyond the fused step
     st = L.mkv_rocket_decode(ctypes.byref(rc), 64, ctypes.byref(cache), None, 128, None)
     assert st == mkv.MKV_ERR_UNSUPPORTED and "mkv_rocket_select" in mkv.mkv_last_error()
+
+
+def test_rocket_step_checks(L):
+    """The one-launch RocketKV step also needs the token's rows, and counts its CTAs in the top
+    8 bits of T_len: 8 * Hkv <= 256; every rejection happens on the host."""
+    rc = mkv.config(mkv.MKV_ROCKET, 1, 32, 8, 128, snap_window=32, snap_pool=7, snap_keep=4096, page_size=16,
+                    topk_pages=64, topq_dims=32)
+    cache = mkv.mkv_cache()
+    cache.T_cap, cache.T_len, cache.k, cache.v, cache.kmin, cache.kmax = 4208, 8, 256, 512, 768, 1024
+    st = L.mkv_rocket_step(ctypes.byref(rc), 64, None, 96, ctypes.byref(cache), None, 128, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG
+    st = L.mkv_rocket_step(ctypes.byref(rc), 64, 88, 96, ctypes.byref(cache), None, 128, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG and "aligned" in mkv.mkv_last_error()
+    wide = mkv.config(mkv.MKV_ROCKET, 1, 40, 40, 64, snap_window=32, snap_pool=7, snap_keep=256, page_size=16,
+                      topk_pages=4, topq_dims=16)
+    cache.T_cap = 256
+    st = L.mkv_rocket_step(ctypes.byref(wide), 64, 80, 96, ctypes.byref(cache), None, 128, None)
+    assert st == mkv.MKV_ERR_UNSUPPORTED and "8 * Hkv" in mkv.mkv_last_error()

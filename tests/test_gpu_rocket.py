@@ -1,6 +1,6 @@
 """GPU parity: SnapKV prefill compression, page metadata, page selection and sparse decode,
-both as two calls (mkv_rocket_select + mkv_decode_attention) and as the fused step
-(mkv_rocket_decode)."""
+both as two calls (mkv_rocket_select + mkv_decode_attention), as the fused step
+(mkv_rocket_decode) and as the whole step with the token's append (mkv_rocket_step)."""
 import numpy as np
 import pytest
 
@@ -16,7 +16,8 @@ pytestmark = pytest.mark.gpu
 
 
 def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev, exact, units, tag, fused=False):
-    """K, V [B,Hkv,T+steps,D]; QW [B,Hq,W,D] window queries; Q [steps,B,Hq,D] (device tensors)."""
+    """K, V [B,Hkv,T+steps,D]; QW [B,Hq,W,D] window queries; Q [steps,B,Hq,D] (device tensors).
+    fused: False (two calls), True (append + mkv_rocket_decode), "step" (mkv_rocket_step)."""
     torch = torch_cuda()
     G = Hq // Hkv
     cfg = mkv.config(mkv.MKV_ROCKET, B, Hq, Hkv, D, snap_window=W, snap_pool=pool, snap_keep=keep,
@@ -61,11 +62,16 @@ def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev,
         vn = V[:, :, T + s].contiguous()
         q = Q[s].contiguous()
         out = torch.empty_like(q)
-        mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
-        if fused:
+        if fused == "step":
+            page_idx.fill_(-7)
+            mkv.mkv_rocket_step(cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, page_idx.data_ptr(),
+                                out.data_ptr())
+        elif fused:
+            mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
             page_idx.fill_(-7)
             mkv.mkv_rocket_decode(cfg, q.data_ptr(), cache.c, page_idx.data_ptr(), out.data_ptr())
         else:
+            mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
             mkv.mkv_rocket_select(cfg, q.data_ptr(), cache.c, page_idx.data_ptr())
             mkv.mkv_decode_attention(cfg, q.data_ptr(), cache.c, None, page_idx.data_ptr(), out.data_ptr(),
                                      ws.data_ptr(), nws)
@@ -89,7 +95,7 @@ def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev,
     return near
 
 
-@pytest.mark.parametrize("fused", [False, True])
+@pytest.mark.parametrize("fused", [False, True, "step"])
 def test_tiny_exact(fused):
     torch = torch_cuda()
     dev = torch.device("cuda")
@@ -103,7 +109,7 @@ def test_tiny_exact(fused):
     assert near == 0
 
 
-@pytest.mark.parametrize("fused", [False, True])
+@pytest.mark.parametrize("fused", [False, True, "step"])
 def test_keep_everything_is_full_attention(fused):
     """keep >= T and k_p >= pages: every step attends the whole cache."""
     torch = torch_cuda()
@@ -119,7 +125,7 @@ def test_keep_everything_is_full_attention(fused):
 
 
 @pytest.mark.parametrize("G,D,fused", [(1, 128, False), (8, 64, False), (1, 128, True), (8, 64, True),
-                                       (4, 128, True), (2, 64, True)])
+                                       (4, 128, True), (2, 64, True), (4, 128, "step"), (8, 64, "step")])
 def test_shapes_lockstep(G, D, fused):
     torch = torch_cuda()
     dev = torch.device("cuda")
@@ -134,7 +140,7 @@ def test_shapes_lockstep(G, D, fused):
                to_dev(Q, dev), dev, False, [(0, 1), (1, 0)], f"G{G}D{D}", fused)
 
 
-@pytest.mark.parametrize("fused", [False, True])
+@pytest.mark.parametrize("fused", [False, True, "step"])
 def test_full_size_lockstep(fused):
     """B=4, T=32768 -> keep 4096, W=32, pool 7, top-64 pages over top-32 dims: one layer,
     16 steps, two (batch, kv-head) units in lockstep with the oracle."""
@@ -189,3 +195,55 @@ def test_fused_short_contexts():
             assert np.all(pidx[b, h][len(sel):] == -1)
             ref, _, _ = rocket.decode(qh, K[b, h, :n], V[b, h, :n], n, 16, kp, rd)
             assert_close(got[b, h * G:(h + 1) * G], ref, f"n={n} h{h}")
+
+
+def test_step_equals_append_then_decode():
+    """mkv_rocket_step against mkv_append_kv + mkv_rocket_decode on twin caches, over 40 steps that
+    complete pages and then fill the cache: identical outputs, page lists, K/V rows, page bounds and
+    lengths; a full cache is not appended, keeps its length, raises MKV_FLAG_CACHE_FULL and
+    attends to its tokens."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(44)
+    B, Hq, Hkv, D, kp, rd = 3, 8, 2, 128, 4, 32
+    T0, T_cap, steps = [20, 47, 64], 96, 40           # entry 2 is full from step 32 on
+    cfg = mkv.config(mkv.MKV_ROCKET, B, Hq, Hkv, D, snap_window=8, snap_pool=7, snap_keep=64, page_size=16,
+                     topk_pages=kp, topq_dims=rd)
+    K = rng.standard_normal((B, Hkv, T_cap + steps, D)).astype(np.float16)
+    V = rng.standard_normal((B, Hkv, T_cap + steps, D)).astype(np.float16)
+    twins = []
+    for _ in range(2):
+        cache = caches.alloc_cache(cfg, T_cap, device=dev)
+        cache.t["k"].copy_(to_dev(K[:, :, :T_cap], dev))
+        cache.t["v"].copy_(to_dev(V[:, :, :T_cap], dev))
+        for b in range(B):
+            for h in range(Hkv):
+                npg = T0[b] // 16
+                kmin, kmax = rocket.page_minmax(K[b, h, :T0[b]], 16, npg)
+                cache.t["kmin"][b, h, :, :npg] = to_dev(kmin.T.astype(np.float16), dev)
+                cache.t["kmax"][b, h, :, :npg] = to_dev(kmax.T.astype(np.float16), dev)
+        cache.t["T_len"].copy_(torch.tensor(T0, dtype=torch.int32))
+        twins.append(cache)
+    a, c = twins
+    full_seen = False
+    for s in range(steps):
+        kn = to_dev(K[:, :, T_cap + s], dev)          # rows the caches do not hold yet
+        vn = to_dev(V[:, :, T_cap + s], dev)
+        q = to_dev(rng.standard_normal((B, Hq, D)).astype(np.float16), dev)
+        oa, oc = torch.empty_like(q), torch.empty_like(q)
+        pa = torch.full((B, Hkv, kp), -7, dtype=torch.int32, device=dev)
+        pc = torch.full_like(pa, -7)
+        will_fill = [int(a.t["T_len"][b]) >= T_cap for b in range(B)]
+        mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), a.c)
+        fa = mkv.mkv_get_status()
+        mkv.mkv_rocket_decode(cfg, q.data_ptr(), a.c, pa.data_ptr(), oa.data_ptr())
+        mkv.mkv_rocket_step(cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), c.c, pc.data_ptr(), oc.data_ptr())
+        fc = mkv.mkv_get_status()
+        assert fa == fc == (mkv.MKV_FLAG_CACHE_FULL if any(will_fill) else 0), f"step {s}: flags {fa} {fc}"
+        full_seen |= any(will_fill)
+        assert torch.equal(oa.view(torch.int16), oc.view(torch.int16)), f"step {s}: outputs differ"
+        assert torch.equal(pa, pc), f"step {s}: page lists differ"
+        for key in ("T_len", "k", "v", "kmin", "kmax"):
+            assert torch.equal(a.t[key].view(torch.int16) if key != "T_len" else a.t[key],
+                               c.t[key].view(torch.int16) if key != "T_len" else c.t[key]), f"step {s}: {key}"
+    assert full_seen
