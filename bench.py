@@ -240,9 +240,9 @@ class Runner:
             self.step()
 
     def launches_per_step(self):
-        # per layer: append (KVQuant: quantize + length advance), decode, (H2O: score update);
-        # RocketKV: append, page choice and attention in one launch
-        per = {"fp16": 2, "kvquant": 3, "h2o": 3, "rocket": 1}[self.method]
+        # per layer: append (KVQuant: quantize, which also stores the new length), decode,
+        # (H2O: score update); RocketKV: append, page choice and attention in one launch
+        per = {"fp16": 2, "kvquant": 2, "h2o": 3, "rocket": 1}[self.method]
         return per * self.w.L
 
     def decode_bytes(self):

@@ -298,9 +298,13 @@ mkv_status mkv_quant_prepare(const mkv_config* cfg, mkv_quant_params* qparams, v
  * at slots T_len[b]..T_len[b]+n_tokens-1 (n_tokens = T at prefill, 1 per
  * decode step): key outliers by the per-channel range, value outliers as the
  * n_v largest |x| per token, codes by correctly rounded fp32 arithmetic.
- * k_pre (keys before rotation), v fp16 [B][Hkv][n_tokens][D].  T_len += n.
- * A full key-outlier region sets MKV_FLAG_K_OUTLIER_OVERFLOW (entries past
- * k_out_cap are dropped). */
+ * k_pre (keys before rotation), v fp16 [B][Hkv][n_tokens][D].  T_len += n,
+ * stored by the launch's last CTA of each batch entry: while it runs, the
+ * top 8 bits of T_len[b] count its finished CTAs, so nothing else may read
+ * or write T_len of this cache during the call (MKV_ERR_UNSUPPORTED when
+ * T_cap >= 2^24 or Hkv > 256).  A full cache sets MKV_FLAG_CACHE_FULL and
+ * keeps T_len.  A full key-outlier region sets MKV_FLAG_K_OUTLIER_OVERFLOW
+ * (entries past k_out_cap are dropped). */
 mkv_status mkv_quantize_kv(const mkv_config* cfg, const mkv_quant_params* qparams,
                            const void* k_pre, const void* v, int64_t n_tokens,
                            mkv_cache* cache, void* stream);

@@ -71,8 +71,9 @@ __device__ __forceinline__ int uniform_code(float x, float lo, float scale, int 
 }
 
 // One CTA per (batch, kv-head), one thread per channel; tokens in order so the
-// key-outlier CSR is appended sequentially.  Blocks of this kernel run alone
-// per (b, h), so T_len is read once by every CTA and advanced by kv-head 0.
+// key-outlier CSR is appended sequentially.  Every CTA reads T_len[b] once; the
+// last CTA of batch entry b to finish stores the new length: during the launch
+// the top 8 bits of T_len[b] count the finished CTAs (readers mask them off).
 __global__ void quantize_kernel(const QuantArgs a) {
   extern __shared__ uint8_t sm[];
   const int D = a.D, K = 1 << a.bits, L = K - 1, NP = D / 2;
@@ -86,9 +87,18 @@ __global__ void quantize_kernel(const QuantArgs a) {
   __shared__ int s_cnt[32];
   __shared__ float s_lo[32], s_hi[32];
 
-  const int64_t t_base = a.T_len[b];
-  if (t_base < 0 || t_base + a.n_tokens > a.T_cap) {   // no room: drop, flag, keep T_len
+  const int64_t t_base = a.T_len[b] & 0xffffff;
+  // the last CTA of batch entry b stores its new length (after every thread of this CTA read it)
+  auto finish = [&](int64_t len) {
+    __syncthreads();
+    if (c == 0) {
+      const unsigned old = atomicAdd(reinterpret_cast<unsigned*>(a.T_len) + b, 1u << 24);
+      if ((int)(old >> 24) == a.Hkv - 1) a.T_len[b] = (int32_t)len;
+    }
+  };
+  if (t_base + a.n_tokens > a.T_cap) {   // no room: drop, flag, keep T_len
     if (c == 0 && h == 0) atomicOr(&g_status_kvquant, MKV_FLAG_CACHE_FULL);
+    finish(t_base);
     return;
   }
   const int rowb = D * a.bits / 8;
@@ -223,14 +233,9 @@ __global__ void quantize_kernel(const QuantArgs a) {
     if (c == 0) off_row[t + 1] = off;
     __syncthreads();
   }
+  finish(t_base + a.n_tokens);
 }
 
-// T_len[b] += n after every (b, h) CTA of quantize_kernel finished (stream order);
-// a batch entry without room was left unwritten and keeps its length.
-__global__ void advance_kernel(int32_t* T_len, int B, int64_t n, int64_t T_cap) {
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b < B && T_len[b] >= 0 && T_len[b] + n <= T_cap) T_len[b] += (int32_t)n;
-}
 
 // ----------------------------------------------------------------- calibrate
 
@@ -479,9 +484,6 @@ cudaError_t launch_quantize(const mkv_config& c, const mkv_quant_params& qp, con
   const int nwords = (c.D * c.bits / 8 + 3) / 4;
   const size_t smem = 2 * c.D + 4 * c.D + 2 * nwords * 4 + 16;
   quantize_kernel<<<c.B * c.Hkv, c.D, smem, st>>>(a);
-  cudaError_t e = cudaPeekAtLastError();
-  if (e != cudaSuccess) return e;
-  advance_kernel<<<(c.B + 127) / 128, 128, 0, st>>>(cache.T_len, c.B, n_tokens, cache.T_cap);
   return cudaPeekAtLastError();
 }
 

@@ -398,6 +398,9 @@ mkv_status mkv_quantize_kv(const mkv_config* cfg, const mkv_quant_params* qparam
   MKV_TRY(check_qparams(cfg, qparams, false));
   MKV_REQUIRE(k_pre && v && n_tokens >= 1 && n_tokens <= cache->T_cap, MKV_ERR_INVALID_ARG,
               "k_pre/v NULL or n_tokens outside [1, T_cap]");
+  // the launch counts its finished CTAs per batch entry in the top 8 bits of T_len[b]
+  MKV_REQUIRE(cache->T_cap < (1 << 24) && cfg->Hkv <= 256, MKV_ERR_UNSUPPORTED,
+              "quantize needs T_cap < 2^24 and Hkv <= 256 (T_cap %lld, Hkv %d)", (long long)cache->T_cap, cfg->Hkv);
   MKV_CUDA(launch_quantize(*cfg, *qparams, k_pre, v, n_tokens, *cache, as_stream(stream)));
   return MKV_OK;
 }
