@@ -314,25 +314,29 @@ def time_decode_launches(runner, reps):
 
 
 def time_e2e(runner, steps, warmup):
-    """Through the public API with host buffers: per step, H2D of every layer's q and
-    new k/v from pinned memory, the step, and D2H of every layer's output."""
+    """Through the public API with host buffers: per step, one H2D copy of every layer's q and
+    new k/v from pinned memory (packed in one buffer), the step's API calls, and one D2H copy of
+    every layer's output."""
     torch = runner.torch
     w = runner.w
-    hq = [t.cpu().pin_memory() for t in runner.q]
-    hk = [t.cpu().pin_memory() for t in runner.kn]
-    hv = [t.cpu().pin_memory() for t in runner.vn]
-    ho = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in runner.out]
-    dq = [torch.empty_like(t) for t in runner.q]
-    dk = [torch.empty_like(t) for t in runner.kn]
-    dv = [torch.empty_like(t) for t in runner.vn]
+    ins = [t for l in range(w.L) for t in (runner.q[l], runner.kn[l], runner.vn[l])]
+    sizes = [t.numel() for t in ins]
+    h_in = torch.cat([t.reshape(-1).cpu() for t in ins]).pin_memory()
+    d_in = torch.empty_like(h_in, device=runner.q[0].device)
+    views, off = [], 0
+    for t, n in zip(ins, sizes):
+        views.append(d_in[off:off + n].view(t.shape))
+        off += n
+    o_shape, o_n = runner.out[0].shape, runner.out[0].numel()
+    d_out = torch.empty(w.L * o_n, dtype=runner.out[0].dtype, device=runner.out[0].device)
+    h_out = torch.empty(d_out.shape, dtype=d_out.dtype).pin_memory()
+    outs = [d_out[l * o_n:(l + 1) * o_n].view(o_shape) for l in range(w.L)]
 
     def one():
+        d_in.copy_(h_in, non_blocking=True)
         for l in range(w.L):
-            dq[l].copy_(hq[l], non_blocking=True)
-            dk[l].copy_(hk[l], non_blocking=True)
-            dv[l].copy_(hv[l], non_blocking=True)
-            runner.layer_step(l, dq[l], dk[l], dv[l], runner.out[l])
-            ho[l].copy_(runner.out[l], non_blocking=True)
+            runner.layer_step(l, views[3 * l], views[3 * l + 1], views[3 * l + 2], outs[l])
+        h_out.copy_(d_out, non_blocking=True)
 
     for _ in range(warmup):
         one()
@@ -342,8 +346,8 @@ def time_e2e(runner, steps, warmup):
         one()
     torch.cuda.synchronize()
     dt = (time.perf_counter() - t0) / steps
-    h2d = sum(t.numel() * t.element_size() for t in hq + hk + hv)
-    d2h = sum(t.numel() * t.element_size() for t in ho)
+    h2d = h_in.numel() * h_in.element_size()
+    d2h = h_out.numel() * h_out.element_size()
     return dt, h2d, d2h
 
 
