@@ -21,14 +21,14 @@
 // a rotation held in registers for the whole kernel (the chunk start's own
 // rotation R(t0) is applied to the query instead:
 // q . R(t0 + d) k = (R(t0)^T q) . (R(d) k)) and written as fp16 hi plus the
-// fp16 remainder lo, so the tensor-core product keeps fp32 accuracy.  The same
-// thread restores its token's value outliers in its pairs (exact fp16 values).
-// Consumers: each of the four attention warps owns 16 token rows of a chunk.  It
-// first restores the key outliers of its rows in the key tiles (an outlier x at
-// channel ch adds (x - k_dense[ch]) R(d) e_ch to the rotated pair, which is split
-// again; x-channels before y-channels so the two entries of a pair never write
-// one word at once; __syncwarp orders it, as only this warp reads those rows),
-// then computes S^T (tokens x heads) = K_hi q_hi + K_lo q_hi + K_hi q_lo, the
+// fp16 remainder lo, so the tensor-core product keeps fp32 accuracy.
+// Consumers: each of the four attention warps owns 16 token rows of a chunk and
+// first restores their outliers (only this warp reads those rows, so __syncwarp
+// orders it): a key outlier x at channel ch adds (x - k_dense[ch]) R(d) e_ch to
+// the rotated pair, which is split again (x-channels before y-channels, so the
+// two entries of a pair never write one word at once); a value outlier
+// overwrites its value tile entry with the exact fp16 value.  The warp then
+// computes S^T (tokens x heads) = K_hi q_hi + K_lo q_hi + K_hi q_lo, the
 // online softmax, and O^T (dims x heads) += V^T P^T with P^T transposed in
 // registers (movmatrix).  Tile columns hold pair i at columns (2i, 2i+1) =
 // channels (i, i + D/2); the output is un-permuted at the end.
@@ -126,7 +126,8 @@ struct KvqLayout {
   static constexpr int B_QL = B_QH + 8 * QROW * 4;           // q_lo
   static constexpr int B_ENT = B_QL + 8 * QROW * 4;          // [kEnt] u32 first key-outlier entries
   static constexpr int B_KO = B_ENT + kEnt * 4;              // [68] int32 CSR offsets of the chunk
-  static constexpr int BUF = B_KO + 68 * 4;
+  static constexpr int B_VO = B_KO + 68 * 4;                 // [NVS][64] u32 value outliers
+  static constexpr int BUF = B_VO + NVS * kChunk * 4;
   // CTA layout
   static constexpr int DTAB = 0;                             // [NP][64] float2 rotation by delta
   static constexpr int KDQ = DTAB + NP * kChunk * 8;         // [D][K] float
@@ -464,13 +465,8 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       const uint32_t my_ent = ptid < kEnt ? reinterpret_cast<const uint32_t*>(st + Lay::S_ENT)[ptid] : 0u;
       const int32_t my_ko = ptid <= kChunk ? koff[ptid] : 0;
       const float2 qcs = reinterpret_cast<const float2*>(st + Lay::S_RT)[qi];
-      uint32_t vo[Lay::NVS];
-      const int n_vs = stage_vout ? a.n_v : 0;  // staged value outliers of a token
-#pragma unroll
-      for (int k = 0; k < Lay::NVS; ++k) {
-        if (k >= n_vs) break;
-        vo[k] = reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[k * kChunk + tok];
-      }
+      const bool my_vo_in = stage_vout && ptid < kChunk * a.n_v;
+      const uint32_t my_vo = my_vo_in ? reinterpret_cast<const uint32_t*>(st + Lay::S_VO)[ptid] : 0u;
       if (c >= 2) bar_sync(kBarEmpty + buf, kThr);   // attention on chunk c-2 released the buffer
       uint8_t* B_ = bufs + buf * Lay::BUF;
       uint8_t* khi_t = B_ + Lay::B_KHI;
@@ -487,9 +483,10 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
         reinterpret_cast<uint32_t*>(B_ + Lay::B_QL)[qpos] = pack_half2(xr - hf.x, yr - hf.y);
       }
 
-      // the chunk's key-outlier entries for the consumers, who restore them
+      // the chunk's outlier entries for the consumers, who restore them
       if (ptid < kEnt) reinterpret_cast<uint32_t*>(B_ + Lay::B_ENT)[ptid] = my_ent;
       if (ptid <= kChunk) reinterpret_cast<int32_t*>(B_ + Lay::B_KO)[ptid] = my_ko;
+      if (my_vo_in) reinterpret_cast<uint32_t*>(B_ + Lay::B_VO)[ptid] = my_vo;
 
       // keys: dequantize, rotate by R(tok), split; rows past the cache end were zero-filled
       // (finite keys, masked in the attention)
@@ -534,26 +531,6 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
           }
           const int ch = (grp * QP + jj) / 4;
           *reinterpret_cast<uint4*>(v_t + tile_off<D>(tok, ch)) = make_uint4(pv[0], pv[1], pv[2], pv[3]);
-        }
-      }
-      // value outliers of this thread's token in its pairs: the exact fp16 value over the dense one
-      if (t0 + tok < n_len) {
-        auto put = [&](uint32_t ev) {
-          const int chn = (int)(ev >> 16);
-          const int i = chn < NP ? chn : chn - NP;
-          if ((unsigned)(i - grp * QP) < (unsigned)QP && chn < D) {
-            const int col = 2 * i + (chn >= NP ? 1 : 0);
-            *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(tok, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
-          }
-        };
-        if (stage_vout) {
-#pragma unroll
-          for (int k = 0; k < Lay::NVS; ++k) {
-            if (k >= n_vs) break;
-            put(vo[k]);
-          }
-        } else {
-          for (int k = 0; k < a.n_v; ++k) put(__ldg(a.v_out + (bh * a.T_cap + t0 + tok) * a.n_v + k));
         }
       }
       bar_arrive(kBarFull + buf, kThr);       // chunk c's tiles are ready
@@ -642,6 +619,17 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
         fix(ea, 1);
         fix(eb, 1);
         for (int e = e_lo + 64 + lane; e < e_hi; e += 32) fix(fetch(e), 1);
+        // value outliers of the warp's rows: the exact fp16 value over the dense one, one lane per entry
+        for (int e = lane; e < 16 * a.n_v; e += 32) {
+          const int t = t0w + (e & 15), k = e >> 4;
+          if (t0 + t >= n_len) continue;
+          const uint32_t ev = a.n_v <= Lay::NVS ? reinterpret_cast<const uint32_t*>(B_ + Lay::B_VO)[k * kChunk + t]
+                                                : __ldg(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
+          const int chn = (int)(ev >> 16);
+          if (chn >= D) continue;
+          const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
+          *reinterpret_cast<uint16_t*>(v_t + tile_off<D>(t, col / 8) + (col % 8) * 2) = (uint16_t)(ev & 0xffffu);
+        }
         __syncwarp();
       }
       const int qrow = (real ? g : 0) * (QROW / 2);
