@@ -424,20 +424,19 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     // The first kEnt key-outlier entries of a chunk are staged by cp.async one chunk ahead
     // (once the chunk's offsets have landed), one per thread, in a commit group of their own
     // ahead of that iteration's chunk copies; those of chunk 0 with chunk 0.
-    auto load_entries = [&](int stage, int64_t e0, int64_t e1) {
-      const int64_t e = e0 + ptid;
+    // (threads ptid < kEnt, whole warps; entry indices fit in 32 bits, checked by the host)
+    auto load_entries = [&](int stage, int e0, int e1) {
+      const int e = e0 + ptid;
       const bool ok = e >= 0 && e < e1;       // offsets of a corrupted cache stay harmless
-      if (ptid < kEnt)
-        cp_async4s(stg_s + stage * Lay::STAGE + Lay::S_ENT + ptid * 4, gents + (ok ? e : 0), ok ? 4 : 0);
+      cp_async4s(stg_s + stage * Lay::STAGE + Lay::S_ENT + ptid * 4, gents + (ok ? e : 0), ok ? 4 : 0);
     };
 #pragma unroll
     for (int s = 0; s < NS - 1; ++s) {
       if (s < nchunks) {
         load_chunk(s, s);
-        if (s == 0) {
-          const int64_t e0 = __ldg(a.k_out_off + off_base + v_begin);
-          const int64_t e1 = min((int64_t)__ldg(a.k_out_off + off_base + min(v_begin + kChunk, (int64_t)n_len)),
-                                 a.k_out_cap);
+        if (s == 0 && ptid < kEnt) {
+          const int e0 = __ldg(a.k_out_off + off_base + v_begin);
+          const int e1 = min(__ldg(a.k_out_off + off_base + min(v_begin + kChunk, (int64_t)n_len)), (int)a.k_out_cap);
           load_entries(0, e0, e1);
         }
       }
@@ -446,9 +445,9 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     for (int c = 0; c < nchunks; ++c) {
       cp_async_wait<NS - 3>();                // this thread's copies of chunks c, c+1 and entries of c landed
       bar_sync(kBarProd, kProdThr);           // everyone's landed; the stage of chunk c-1 is free
-      if (c + 1 < nchunks) {                  // chunk c+1's offsets landed with the wait above
+      if (c + 1 < nchunks && ptid < kEnt) {   // chunk c+1's offsets landed with the wait above
         const int32_t* ko1 = reinterpret_cast<const int32_t*>(stg + ((c + 1) % NS) * Lay::STAGE + Lay::S_KO);
-        load_entries((c + 1) % NS, ko1[0], min((int64_t)ko1[kChunk], a.k_out_cap));
+        load_entries((c + 1) % NS, ko1[0], min(ko1[kChunk], (int)a.k_out_cap));
       }
       cp_async_commit();
       if (c + NS - 1 < nchunks) load_chunk(c + NS - 1, (c + NS - 1) % NS);
