@@ -7,12 +7,15 @@
 //   v_t = lo_t + scale_t * tbl[code] with outliers restored,
 //   out_h = softmax_t(scale q_h . k_t) v_t.
 //
-// GB300 design: one CTA of 20 warps per (batch, kv-head, split), one CTA per
-// SM, warp-specialised.  Sixteen producer warps stage packed codes by cp.async
-// (three 64-token chunks in flight) and dequantize chunk c into one of two
-// fp16 tile buffers while four consumer warps run the tensor-core attention on
-// the previous chunk from the other; named barriers (FULL / EMPTY per buffer)
-// hand the buffers over.
+// GB300 design: one CTA of 20 warps per SM (at most 152), warp-specialised.
+// The 64-token chunks of all (batch, kv-head) units, laid end to end, are cut
+// into equal ranges, one per CTA; a CTA runs its range unit by unit, writes one
+// partial (m, l, o) per unit into its slot, and the last CTA of a unit merges
+// the unit's partials.  Sixteen producer warps stage packed codes by cp.async
+// (three chunks in flight) and dequantize chunk c into one of two fp16 tile
+// buffers while four consumer warps run the tensor-core attention on the
+// previous chunk from the other; named barriers (FULL / EMPTY per buffer) hand
+// the buffers over.
 //
 // Producers: thread (token row tok, pair group g) dequantizes QP = D/16 pairs
 // (i, i + D/2) of its token's key and value rows from shared per-channel tables
@@ -20,7 +23,8 @@
 // key pair is rotated by the token's offset d = tok from the chunk start with
 // a rotation held in registers for the whole kernel (the chunk start's own
 // rotation R(t0) is applied to the query instead:
-// q . R(t0 + d) k = (R(t0)^T q) . (R(d) k)) and written as fp16 hi plus the
+// q . R(t0 + d) k = (R(t0)^T q) . (R(d) k)), computed on the paired fp32 pipe
+// from key tables stored as (v, v) pairs, and written as fp16 hi plus the
 // fp16 remainder lo, so the tensor-core product keeps fp32 accuracy.
 // Consumers: each of the four attention warps owns 16 token rows of a chunk and
 // first restores their outliers (only this warp reads those rows, so __syncwarp
@@ -130,8 +134,8 @@ struct KvqLayout {
   static constexpr int BUF = B_VO + NVS * kChunk * 4;
   // CTA layout
   static constexpr int DTAB = 0;                             // [NP][64] float2 rotation by delta
-  static constexpr int KDQ = DTAB + NP * kChunk * 8;         // [D][K] float
-  static constexpr int VTB = KDQ + D * K * 4;                // [D][K] float
+  static constexpr int KDQ = DTAB + NP * kChunk * 8;         // [D][K] float pairs (v, v)
+  static constexpr int VTB = KDQ + D * K * 8;                // [D][K] float
   static constexpr int QS = VTB + D * K * 4;                 // [8][D] f32 query (as given, rotated)
   static constexpr int STG = QS + 8 * D * 4;                 // [NS][STAGE]
   static constexpr int BUFS = STG + NS * STAGE;              // [2][BUF]
@@ -174,6 +178,26 @@ __device__ __forceinline__ void group_words(const uint32_t* row, int g, uint32_t
 #pragma unroll
     for (int k = 0; k < NW; ++k) w[k] = __funnelshift_r(raw[k], raw[k + 1], sh);
   }
+}
+
+// packed fp32 pairs (two lanes of one 64-bit register; Blackwell's paired fp32 pipe)
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
 }
 
 // (a, b) as fp16 hi and the fp16 remainder lo = x - hi (exact in fp32 before its rounding)
@@ -220,7 +244,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   constexpr int KC = D / 16;
   extern __shared__ __align__(128) uint8_t smem[];
   float2* dtab = reinterpret_cast<float2*>(smem + Lay::DTAB);
-  float* kdq = reinterpret_cast<float*>(smem + Lay::KDQ);
+  uint64_t* kdq = reinterpret_cast<uint64_t*>(smem + Lay::KDQ);
   float* vtb = reinterpret_cast<float*>(smem + Lay::VTB);
   float* qs = reinterpret_cast<float*>(smem + Lay::QS);
   uint8_t* stg = smem + Lay::STG;
@@ -282,7 +306,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     for (int k = 0; k < NT; ++k) {
       const int e = tid + k * kThr;
       if (e < D * K) {
-        kdq[e] = kv[k];
+        kdq[e] = f2_pack(kv[k], kv[k]);
         vtb[e] = __half2float(__ushort_as_half(vv[k]));
       }
     }
@@ -406,10 +430,15 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
         }
       }
     };
-    // this thread's key rotations R(tok) for its pairs: the same in every chunk
-    float2 rot[QP];
+    // this thread's key rotations R(tok) = [c -s; s c] for its pairs, the same in every chunk, as
+    // the packed columns (c, s) and (-s, c)
+    uint64_t rc0[QP], rc1[QP];
 #pragma unroll
-    for (int j = 0; j < QP; ++j) rot[j] = dtab[(grp * QP + j) * kChunk + tok];
+    for (int j = 0; j < QP; ++j) {
+      const float2 cs = dtab[(grp * QP + j) * kChunk + tok];
+      rc0[j] = f2_pack(cs.x, cs.y);
+      rc1[j] = f2_pack(-cs.y, cs.x);
+    }
 
     // this thread's element of the rotated-query table (head qg, pair qi)
     const int nq = a.G * NP;
@@ -457,7 +486,6 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       const int32_t* koff = reinterpret_cast<const int32_t*>(st + Lay::S_KO);
       const uint32_t* kcodes = reinterpret_cast<const uint32_t*>(st + Lay::S_KC);
       const int buf = c & 1;
-      const int64_t t0 = v_begin + (int64_t)c * kChunk;
       // staged words this thread hands on or uses late, read before the wait for the buffer: its
       // key-outlier entry and offset for the consumers, its part of the chunk-start rotation, and
       // its token's value outliers
@@ -493,7 +521,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       {
         uint32_t w[NWG];
         group_words<BITS, QP, NWG>(krow, grp, w);
-        const float* kq = kdq + grp * QP * K;
+        const uint64_t* kq = kdq + grp * QP * K;
 #pragma unroll
         for (int jj = 0; jj < QP; jj += 4) {
           uint32_t ph[4], pl[4];
@@ -502,9 +530,20 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
             const int j = jj + u;
             int clo, chi;
             pair_codes<BITS, NWG>(w, j, clo, chi);
-            const float x = kq[j * K + clo];
-            const float y = kq[(j + NP) * K + chi];
-            split_hi_lo(x * rot[j].x - y * rot[j].y, y * rot[j].x + x * rot[j].y, ph[u], pl[u]);
+            // (x, x) (c, s) + (y, y) (-s, c) = R(tok) (x, y); as scalars for 3-bit codes, whose
+            // word-straddling extraction schedules worse around the paired ops (measured)
+            float xr, yr;
+            if constexpr (BITS != 3) {
+              f2_unpack(f2_fma(kq[(j + NP) * K + chi], rc1[j], f2_mul(kq[j * K + clo], rc0[j])), xr, yr);
+            } else {
+              float x, y, c, sn, unused0, unused1;
+              f2_unpack(kq[j * K + clo], x, unused0);
+              f2_unpack(kq[(j + NP) * K + chi], y, unused1);
+              f2_unpack(rc0[j], c, sn);
+              xr = x * c - y * sn;
+              yr = y * c + x * sn;
+            }
+            split_hi_lo(xr, yr, ph[u], pl[u]);
           }
           const int ch = (grp * QP + jj) / 4;
           *reinterpret_cast<uint4*>(khi_t + tile_off<D>(tok, ch)) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
@@ -769,7 +808,7 @@ cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_
   a.Hq = c.Hq;
   a.Hkv = c.Hkv;
   a.G = c.Hq / c.Hkv;
-    a.n_v = std::min(c.D, (int)ceil((double)c.outlier_frac * c.D));
+  a.n_v = std::min(c.D, (int)ceil((double)c.outlier_frac * c.D));
   a.n_split = sp.n_split;
   a.n_cta = sp.n_cta;
   a.cpu = sp.chunks_per_unit;

@@ -218,6 +218,13 @@ def test_decode_all_outliers_equals_fp16_path():
     _decode_vs_oracle(B=1, Hq=8, Hkv=2, D=64, bits=2, mode="uniform", T=130, steps=1, seed=77, frac=1.0)
 
 
+def test_decode_dense_outliers():
+    """outlier_frac = 0.1 at the Llama shape: ~13 key outliers per token, so each attention warp
+    restores several rounds of entries, many beyond the staged ones, and pairs with outliers in
+    both channels (i and i + D/2) of a token are common."""
+    _decode_vs_oracle(B=2, Hq=32, Hkv=8, D=128, bits=4, mode="nuq", T=700, steps=1, seed=12, frac=0.1)
+
+
 def test_quantize_capacity_flag():
     """An append past T_cap writes nothing, keeps T_len and raises MKV_FLAG_CACHE_FULL."""
     torch = torch_cuda()
