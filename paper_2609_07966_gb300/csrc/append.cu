@@ -29,6 +29,7 @@ struct AppendArgs {
 // One CTA per batch entry: every kv-head's row, then (ROCKET) the metadata of a
 // page the token completes, then T_len[b] += 1.
 __global__ void append_kernel(const AppendArgs a) {
+  pdl_wait_and_trigger();
   const int b = blockIdx.x;
   const int t = a.T_len[b];
   const int nc = a.D / 8;
@@ -111,8 +112,7 @@ cudaError_t launch_append(const mkv_config& c, const void* k_new, const void* v_
   a.Hkv = c.Hkv;
   a.D = c.D;
   a.mode = c.method == MKV_H2O ? 1 : (c.method == MKV_ROCKET ? 2 : 0);
-  append_kernel<<<c.B, 256, 0, st>>>(a);
-  return cudaPeekAtLastError();
+  return launch_pdl(append_kernel, dim3(c.B), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_rope_table(int D, float theta, int64_t T_max, float* table, cudaStream_t st) {

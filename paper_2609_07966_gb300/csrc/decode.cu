@@ -73,6 +73,7 @@ __device__ __forceinline__ int64_t slot_of(const Fp16Args& a, int64_t v, int n_l
 
 template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args a) {
+  pdl_wait_and_trigger();
   constexpr int ROWB = D * 2;           // bytes per token row
   constexpr int NC = D / 8;             // 16-byte chunks per row
   constexpr int TILE = kChunk * ROWB;   // one K (or V) tile
@@ -307,8 +308,7 @@ cudaError_t launch_fp16_t(const Fp16Args& a, int n_units, int n_split, cudaStrea
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   dim3 grid(n_split, n_units);
-  decode_fp16_kernel<D, MODE><<<grid, kThreads, smem, st>>>(a);
-  return cudaPeekAtLastError();
+  return launch_pdl(decode_fp16_kernel<D, MODE>, grid, dim3(kThreads), smem, st, a);
 }
 
 }  // namespace

@@ -87,6 +87,7 @@ __global__ void __launch_bounds__(1024) h2o_update_kernel(const float* __restric
                                                          int H, int R, const int32_t* __restrict__ T_len,
                                                          int32_t* __restrict__ pos, float* __restrict__ acc,
                                                          int32_t* __restrict__ slot_out) {
+  pdl_wait_and_trigger();
   h2o_update_unit(logits, m_tot, l_tot, Hkv, G, T_cap, H, R, T_len, pos, acc, slot_out, blockIdx.x);
 }
 
@@ -109,10 +110,9 @@ cudaError_t launch_h2o_keep(const mkv_config& c, const void* full_k, const void*
 }
 
 cudaError_t launch_h2o_update(const mkv_config& c, const mkv_cache& cache, const DecodeWs& ws, cudaStream_t st) {
-  h2o_update_kernel<<<c.B * c.Hkv, 1024, 0, st>>>(ws.logits, ws.m_tot, ws.l_tot, c.Hkv, c.Hq / c.Hkv, cache.T_cap,
-                                                 c.h2o_heavy, c.h2o_recent, cache.T_len, cache.pos, cache.acc,
-                                                 cache.slot);
-  return cudaPeekAtLastError();
+  return launch_pdl(h2o_update_kernel, dim3(c.B * c.Hkv), dim3(1024), 0, st, (const float*)ws.logits,
+                    (const float*)ws.m_tot, (const float*)ws.l_tot, c.Hkv, c.Hq / c.Hkv, cache.T_cap, c.h2o_heavy,
+                    c.h2o_recent, (const int32_t*)cache.T_len, cache.pos, cache.acc, cache.slot);
 }
 
 }  // namespace mkv

@@ -16,6 +16,18 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 __host__ __device__ __forceinline__ int64_t ceil_div_dev(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// Programmatic dependent launch: the FP16-family kernels of a decode step (append, FP16 / H2O /
+// page-list decode, H2O update) are launched with the programmatic stream-serialization attribute,
+// so a kernel may be scheduled while its predecessor in the stream is still running.  It waits here
+// for that grid's completion and memory before its first global access, then lets its own
+// successor be scheduled (which waits the same way); a successor can only be scheduled once every
+// CTA of this grid has passed this point, so it never holds resources a CTA of this grid is waiting
+// for.  (The KVQuant and fused RocketKV kernels launch plainly: there it measured slower.)
+__device__ __forceinline__ void pdl_wait_and_trigger() {
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
+
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

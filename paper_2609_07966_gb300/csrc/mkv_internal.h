@@ -6,6 +6,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "mkv.h"
 
 namespace mkv {
@@ -76,6 +78,25 @@ CalibWs calib_ws(const mkv_config& c, int64_t N, void* base);
 
 struct MergeArgs;
 MergeArgs merge_args(const mkv_config& c, const DecodeWs& ws, const Split& sp, void* out, bool h2o_stats);
+
+// Launch of a decode-step kernel with the programmatic stream-serialization attribute (the kernel
+// calls pdl_wait_and_trigger() before its first global access).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              Args&&... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+  return e != cudaSuccess ? e : cudaPeekAtLastError();
+}
 
 // ---- launchers (return the launch status; arguments already validated) ----
 cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const mkv_cache& cache,
