@@ -86,8 +86,31 @@ __global__ void quantize_kernel(const QuantArgs a) {
   uint32_t* words = reinterpret_cast<uint32_t*>(absx + D);   // [2][D*bits/32] packed rows
   __shared__ int s_cnt[32];
   __shared__ float s_lo[32], s_hi[32];
+  __shared__ uint32_t s_max[2][32];
 
+  // Every load that does not depend on the length is issued before it: the channel's parameters and
+  // codebooks, and the first token's key and value; then the length and the CSR offset it selects.
+  const float tlo = a.t_lo[h * D + c], thi = a.t_hi[h * D + c];
+  const float klo = a.k_lo ? a.k_lo[h * D + c] : 0.f, ksc = a.k_scale ? a.k_scale[h * D + c] : 0.f;
+  uint16_t kr[16], vr[16];                   // all codebook loads in flight at once (K <= 16)
+  if (a.nuq) {
+    const uint16_t* kc = a.k_cb + ((int64_t)h * D + c) * K;
+    const uint16_t* vc = a.v_cb + ((int64_t)h * D + c) * K;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      if (j < K) {
+        kr[j] = __ldg(kc + j);
+        vr[j] = __ldg(vc + j);
+      }
+    }
+  }
+  const int64_t src0 = (int64_t)bh * a.n_tokens * D + c;
+  __half xk_next = a.n_tokens > 0 ? a.k_pre[src0] : __ushort_as_half(0);
+  __half xv_next = a.n_tokens > 0 ? a.v[src0] : __ushort_as_half(0);
   const int64_t t_base = a.T_len[b] & 0xffffff;
+  int32_t* off_row = a.k_out_off + (int64_t)bh * (a.T_cap + 1);
+  const bool room = t_base + a.n_tokens <= a.T_cap;
+  int32_t off = (t_base == 0 || !room) ? 0 : off_row[t_base];
   // the last CTA of batch entry b stores its new length (after every thread of this CTA read it)
   auto finish = [&](int64_t len) {
     __syncthreads();
@@ -96,28 +119,15 @@ __global__ void quantize_kernel(const QuantArgs a) {
       if ((int)(old >> 24) == a.Hkv - 1) a.T_len[b] = (int32_t)len;
     }
   };
-  if (t_base + a.n_tokens > a.T_cap) {   // no room: drop, flag, keep T_len
+  if (!room) {                            // no room: drop, flag, keep T_len
     if (c == 0 && h == 0) atomicOr(&g_status_kvquant, MKV_FLAG_CACHE_FULL);
     finish(t_base);
     return;
   }
   const int rowb = D * a.bits / 8;
   const int nwords = (rowb + 3) / 4;
-  // per-channel parameters
-  const float tlo = a.t_lo[h * D + c], thi = a.t_hi[h * D + c];
-  const float klo = a.k_lo ? a.k_lo[h * D + c] : 0.f, ksc = a.k_scale ? a.k_scale[h * D + c] : 0.f;
   float kmu[15], vmu[15];
   if (a.nuq) {
-    const uint16_t* kc = a.k_cb + ((int64_t)h * D + c) * K;
-    const uint16_t* vc = a.v_cb + ((int64_t)h * D + c) * K;
-    uint16_t kr[16], vr[16];                 // all codebook loads in flight at once (K <= 16)
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      if (j < K) {
-        kr[j] = __ldg(kc + j);
-        vr[j] = __ldg(vc + j);
-      }
-    }
 #pragma unroll
     for (int j = 0; j < 15; ++j) {
       if (j < L) {
@@ -126,16 +136,18 @@ __global__ void quantize_kernel(const QuantArgs a) {
       }
     }
   }
-  int32_t* off_row = a.k_out_off + (int64_t)bh * (a.T_cap + 1);
-  int32_t off = (t_base == 0) ? 0 : off_row[t_base];
   if (t_base == 0 && c == 0) off_row[0] = 0;
   const int warp = c >> 5, lane = c & 31, nwarp = D >> 5;
 
   for (int64_t i = 0; i < a.n_tokens; ++i) {
     const int64_t t = t_base + i;
-    const int64_t src = ((int64_t)bh * a.n_tokens + i) * D + c;
+    const __half xk = xk_next, xv = xv_next;     // this token's key and value; the next one's in flight
+    if (i + 1 < a.n_tokens) {
+      xk_next = a.k_pre[src0 + (i + 1) * D];
+      xv_next = a.v[src0 + (i + 1) * D];
+    }
     // ---- keys
-    const float x = __half2float(a.k_pre[src]);
+    const float x = __half2float(xk);
     const bool kout = (x < tlo) || (x > thi);
     int code;
     if (a.nuq) {
@@ -149,9 +161,19 @@ __global__ void quantize_kernel(const QuantArgs a) {
     // rank of this outlier among the token's outliers (channel order)
     const unsigned bal = __ballot_sync(0xffffffffu, kout);
     if (lane == 0) s_cnt[warp] = __popc(bal);
-    // ---- values: rank by (|x| desc, channel asc)
-    const float vx = __half2float(a.v[src]);
-    absx[c] = fabsf(vx);
+    // ---- values: rank by (|x| desc, channel asc).  With few value outliers the ranks 0..n_v-1 are
+    // taken by block-wide maxima of key = (|x| as fp16 magnitude bits << 8) | (255 - c), which orders
+    // like (|x| desc, channel asc) for finite values and is unique; the first round shares this
+    // barrier.  Otherwise each thread counts the channels ahead of it.
+    const float vx = __half2float(xv);
+    const bool few = a.n_v <= 8;
+    uint32_t vkey = ((uint32_t)(__half_as_ushort(xv) & 0x7fffu) << 8) | (uint32_t)(255 - c);
+    if (few) {
+      const uint32_t wmax = __reduce_max_sync(0xffffffffu, vkey);
+      if (lane == 0 && a.n_v > 0) s_max[0][warp] = wmax;
+    } else {
+      absx[c] = fabsf(vx);
+    }
     __syncthreads();
     int before = 0, total = 0;
     for (int w = 0; w < nwarp; ++w) {
@@ -163,16 +185,33 @@ __global__ void quantize_kernel(const QuantArgs a) {
       if (e < a.k_out_cap) {
         // (token position within its 64-token block << 24) | (channel << 16) | fp16 bits
         a.k_out[(int64_t)bh * a.k_out_cap + e] =
-            ((uint32_t)(t & 63) << 24) | ((uint32_t)c << 16) | __half_as_ushort(a.k_pre[src]);
+            ((uint32_t)(t & 63) << 24) | ((uint32_t)c << 16) | __half_as_ushort(xk);
       } else {
         atomicOr(&g_status_kvquant, MKV_FLAG_K_OUTLIER_OVERFLOW);
       }
     }
-    const float ax = absx[c];
     int rank = 0;
-    for (int j = 0; j < D; ++j) {
-      const float o = absx[j];
-      rank += (o > ax || (o == ax && j < c)) ? 1 : 0;
+    if (few) {
+      rank = a.n_v;                      // not among the n_v largest unless a round picks it
+      for (int r = 0; r < a.n_v; ++r) {
+        if (r > 0) {
+          const uint32_t wmax = __reduce_max_sync(0xffffffffu, vkey);
+          if (lane == 0) s_max[r & 1][warp] = wmax;
+          __syncthreads();
+        }
+        uint32_t m = s_max[r & 1][0];
+        for (int w = 1; w < nwarp; ++w) m = max(m, s_max[r & 1][w]);
+        if (vkey == m) {
+          rank = r;
+          vkey = 0u;                       // out of the later rounds (every live key is >= 128)
+        }
+      }
+    } else {
+      const float ax = absx[c];
+      for (int j = 0; j < D; ++j) {
+        const float o = absx[j];
+        rank += (o > ax || (o == ax && j < c)) ? 1 : 0;
+      }
     }
     const bool vout = rank < a.n_v;
     // inlier range of the token's values
@@ -207,7 +246,7 @@ __global__ void quantize_kernel(const QuantArgs a) {
     }
     vcode[c] = (uint8_t)vc;
     const int64_t slot = (int64_t)bh * a.T_cap + t;
-    if (vout) a.v_out[slot * a.n_v + rank] = ((uint32_t)c << 16) | __half_as_ushort(a.v[src]);
+    if (vout) a.v_out[slot * a.n_v + rank] = ((uint32_t)c << 16) | __half_as_ushort(xv);
     if (c == 0) a.v_params[slot] = make_float2(lo, scale);
     for (int wi = c; wi < 2 * nwords; wi += D) words[wi] = 0u;
     __syncthreads();
