@@ -211,6 +211,16 @@ class Runner:
             out = self.out[l] if out is None else out
             mkv.mkv_rocket_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, 0, out.data_ptr())
             return
+        if self.method in ("fp16", "h2o"):    # append and attention in one launch, then (H2O) the update
+            kn = self.kn[l] if kn is None else kn
+            vn = self.vn[l] if vn is None else vn
+            q = self.q[l] if q is None else q
+            out = self.out[l] if out is None else out
+            mkv.mkv_decode_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, out.data_ptr(),
+                                self.ws.data_ptr(), self.nws)
+            if self.method == "h2o":
+                mkv.mkv_h2o_update(self.cfg, cache.c, self.ws.data_ptr(), self.nws)
+            return
         self.append(l, kn, vn)
         self.decode(l, q, out)
         if self.method == "h2o":
@@ -240,9 +250,10 @@ class Runner:
             self.step()
 
     def launches_per_step(self):
-        # per layer: append (KVQuant: quantize, which also stores the new length), decode,
-        # (H2O: score update); RocketKV: append, page choice and attention in one launch
-        per = {"fp16": 2, "kvquant": 2, "h2o": 3, "rocket": 1}[self.method]
+        # per layer: FP16 / H2O append and attention in one launch (H2O: + score update); KVQuant
+        # quantize (which also stores the new length) + decode; RocketKV append, page choice and
+        # attention in one launch
+        per = {"fp16": 1, "kvquant": 2, "h2o": 2, "rocket": 1}[self.method]
         return per * self.w.L
 
     def decode_bytes(self):

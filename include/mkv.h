@@ -366,6 +366,23 @@ mkv_status mkv_rocket_select(const mkv_config* cfg, const void* q, const mkv_cac
 mkv_status mkv_rocket_decode(const mkv_config* cfg, const void* q, const mkv_cache* cache,
                              int32_t* page_idx_out, void* out, void* stream);
 
+/* A whole FP16 or H2O decode step's attention in one launch: mkv_append_kv of
+ * the step's token followed by mkv_decode_attention, with the same cache
+ * contents and output (Section 2.1; H2O's score update stays a separate
+ * mkv_h2o_update).  k_new, v_new fp16 [B][Hkv][D], 16-byte aligned
+ * (MKV_ERR_INVALID_ARG otherwise); q, out, ws as mkv_decode_attention.
+ * The split of the decode whose range holds the token's slot (FP16: T_len,
+ * H2O: slot[b][kv-head]) stages the row from k_new / v_new and writes it
+ * (H2O: with position T_len and a zero score).  While the launch runs, the
+ * top 8 bits of T_len[b] count its finished CTAs (the last one stores the new
+ * length), so nothing else may read or write T_len of this cache during the
+ * call.  A batch entry with no room is not appended (MKV_FLAG_CACHE_FULL, read
+ * by mkv_get_status) and attends to its existing tokens.  MKV_ERR_UNSUPPORTED
+ * when T_cap >= 2^24 or Hkv x (the decode's splits) > 255: use the two calls
+ * then. */
+mkv_status mkv_decode_step(const mkv_config* cfg, const void* q, const void* k_new, const void* v_new,
+                           mkv_cache* cache, void* out, void* ws, size_t ws_bytes, void* stream);
+
 /* A whole RocketKV decode step in one launch: mkv_append_kv of the step's
  * token followed by mkv_rocket_decode, with the same cache contents, page
  * choice and output.  k_new, v_new fp16 [B][Hkv][D] (post-rotation keys),

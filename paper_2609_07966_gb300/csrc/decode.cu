@@ -11,6 +11,7 @@
 // ~5 warp instructions per token, leaving the issue slots to the copies.
 // Online softmax runs in the log2 domain on the accumulator fragments; splits
 // are merged by the last CTA of each (batch, kv-head) (mkv_merge.cuh).
+// mkv_decode_step appends the step's token in the same launch (FP16, H2O).
 #include <math.h>
 
 #include <mutex>
@@ -22,6 +23,8 @@
 namespace mkv {
 
 namespace {
+
+__device__ uint32_t g_status_decode;   // MKV_FLAG_* bits raised by the step's append
 
 constexpr int kStages = 3;
 constexpr int kThreads = 128;   // 4 warps x 16 tokens = one 64-token chunk
@@ -44,6 +47,15 @@ struct Fp16Args {
   float* logits;          // H2O [B][Hkv][T_cap][G]
   int n_split;
   MergeArgs merge;
+  // mkv_decode_step (FP16, H2O): the step's token, appended by this launch (k_new NULL: no append)
+  const __half* k_new;    // [B][Hkv][D]
+  const __half* v_new;
+  __half* k_w;            // the cache rows it is written into
+  __half* v_w;
+  int32_t* T_len_w;
+  int32_t* pos_w;         // H2O: its position and a zero score go to its slot
+  float* acc_w;
+  const int32_t* slot;    // H2O [B][Hkv]: the slot the token takes
 };
 
 constexpr int kMaxSplitPages = 1024;   // ROCKET: page ids of one split, staged in shared memory
@@ -89,10 +101,35 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, r = lane & 3;
 
+  // The step's token (mkv_decode_step).  Every CTA takes the cache as holding it: FP16 T_len + 1
+  // tokens, H2O the token at position T_len in slot[bh].  The CTA whose range holds its slot writes
+  // the row from k_new / v_new (H2O: with its position and a zero score) into the cache before it
+  // stages anything; the last CTA of the batch entry stores the new length (meanwhile the top 8 bits of
+  // T_len count the finished CTAs, masked off here).  A batch entry with no room (FP16: a full
+  // cache; H2O: a slot outside the cache) keeps its length, as mkv_append_kv does.
+  const bool step = MODE != 2 && a.k_new != nullptr;
+  int t_old = 0;
+  bool ok_b = true;
+  int64_t s_new = -1;                  // this unit's slot of the new token (-1: none)
+  if (step) {
+    t_old = a.T_len[b] & 0xffffff;
+    if (MODE == 0) {
+      ok_b = t_old < a.T_cap;
+      s_new = ok_b ? t_old : -1;
+    } else {
+      for (int h = 0; h < a.Hkv; ++h) {
+        const int sh = a.slot[(int64_t)b * a.Hkv + h];
+        ok_b = ok_b && sh >= 0 && sh < a.T_cap;
+      }
+      const int sh = a.slot[bh];
+      s_new = (sh >= 0 && sh < a.T_cap) ? sh : -1;
+    }
+  }
+
   int n_len = 0, ns = 0;
   int64_t v_total;
   if (MODE == 0) {
-    n_len = min((int64_t)a.T_len[b], a.T_cap);
+    n_len = step ? (int)min((int64_t)t_old + (ok_b ? 1 : 0), a.T_cap) : (int)min((int64_t)a.T_len[b], a.T_cap);
     v_total = n_len;
   } else if (MODE == 1) {
     v_total = a.T_cap;
@@ -109,6 +146,26 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
   const __half* kbase = a.k + bh * a.T_cap * D;
   const __half* vbase = a.v + bh * a.T_cap * D;
   const int unit0 = (int)(v_begin / kPage);
+  // The CTA holding the new token's slot writes its row (H2O: and position) before anything is
+  // staged, fenced, so that the chunk copies below read it like any other row.
+  if (step && s_new >= v_begin && s_new < v_end) {
+    constexpr int NC16 = D / 8;
+    if (tid < NC16) {
+      reinterpret_cast<uint4*>(a.k_w + (bh * a.T_cap + s_new) * D)[tid] =
+          reinterpret_cast<const uint4*>(a.k_new + bh * D)[tid];
+    } else if (tid < 2 * NC16) {
+      reinterpret_cast<uint4*>(a.v_w + (bh * a.T_cap + s_new) * D)[tid - NC16] =
+          reinterpret_cast<const uint4*>(a.v_new + bh * D)[tid - NC16];
+    } else if (MODE == 1 && tid == 2 * NC16) {
+      a.pos_w[bh * a.T_cap + s_new] = t_old;
+      a.acc_w[bh * a.T_cap + s_new] = 0.f;
+    }
+    __threadfence();
+  }
+  if (step) {
+    if (!ok_b && split == 0 && kvh == 0 && tid == 0) atomicOr(&g_status_decode, MKV_FLAG_CACHE_FULL);
+    __syncthreads();
+  }
   if (MODE == 2) {                       // this split's page ids, read once
     int64_t nu64 = ceil_div_dev(v_end, kPage) - unit0;
     if (nu64 > kMaxSplitPages) nu64 = kMaxSplitPages;
@@ -297,6 +354,10 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
     }
   }
   __syncthreads();                     // the stage buffers now serve as the merge's scratch
+  if (step && tid == 0) {              // every thread of this CTA read T_len before this point
+    const unsigned old = atomicAdd(reinterpret_cast<unsigned*>(a.T_len_w) + b, 1u << 24);
+    if ((int)(old >> 24) == a.Hkv * (int)gridDim.x - 1) a.T_len_w[b] = ok_b ? t_old + 1 : t_old;
+  }
   merge_if_last<D, kThreads>(a.merge, bh, b, kvh, reinterpret_cast<float*>(smem), kStages * 2 * TILE / 4);
 }
 
@@ -328,10 +389,27 @@ MergeArgs merge_args(const mkv_config& c, const DecodeWs& ws, const Split& sp, v
   return m;
 }
 
+cudaError_t take_status_decode(uint32_t* flags, cudaStream_t st) {
+  uint32_t v = 0, zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbolAsync(&v, g_status_decode, sizeof(v), 0, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemcpyToSymbolAsync(g_status_decode, &zero, sizeof(zero), 0, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  *flags |= v;
+  return e;
+}
+
 cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const mkv_cache& cache,
                                       const int32_t* page_idx, void* out, const DecodeWs& ws,
-                                      const Split& sp, cudaStream_t st) {
+                                      const Split& sp, cudaStream_t st, const void* k_new, const void* v_new) {
   Fp16Args a{};
+  a.k_new = static_cast<const __half*>(k_new);
+  a.v_new = static_cast<const __half*>(v_new);
+  a.k_w = static_cast<__half*>(cache.k);
+  a.v_w = static_cast<__half*>(cache.v);
+  a.T_len_w = cache.T_len;
+  a.pos_w = cache.pos;
+  a.acc_w = cache.acc;
+  a.slot = cache.slot;
   a.q = static_cast<const __half*>(q);
   a.k = static_cast<const __half*>(cache.k);
   a.v = static_cast<const __half*>(cache.v);

@@ -316,6 +316,7 @@ mkv_status mkv_get_status(void* stream, uint32_t* flags) {
   MKV_CUDA(take_status_append(flags, as_stream(stream)));
   MKV_CUDA(take_status_kvquant(flags, as_stream(stream)));
   MKV_CUDA(take_status_rocket(flags, as_stream(stream)));
+  MKV_CUDA(take_status_decode(flags, as_stream(stream)));
   if (*flags != 0) {
     set_error("device status flags 0x%x", *flags);
     return MKV_ERR_CAPACITY;
@@ -362,6 +363,30 @@ mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_
   } else {
     MKV_CUDA(launch_decode_fp16_family(*cfg, q, *cache, page_idx, out, w, sp, st));
   }
+  return MKV_OK;
+}
+
+mkv_status mkv_decode_step(const mkv_config* cfg, const void* q, const void* k_new, const void* v_new,
+                           mkv_cache* cache, void* out, void* ws, size_t ws_bytes, void* stream) {
+  MKV_TRY(check_config(cfg));
+  MKV_REQUIRE(cfg->method == MKV_FP16 || cfg->method == MKV_H2O, MKV_ERR_INVALID_ARG,
+              "decode_step is for FP16 and H2O (KVQUANT: mkv_quantize_kv + mkv_decode_attention; ROCKET: "
+              "mkv_rocket_step)");
+  MKV_TRY(check_cache(cfg, cache));
+  MKV_REQUIRE(q && out && k_new && v_new, MKV_ERR_INVALID_ARG, "q/out/k_new/v_new NULL");
+  MKV_REQUIRE(((uintptr_t)k_new | (uintptr_t)v_new) % 16 == 0, MKV_ERR_INVALID_ARG,
+              "k_new/v_new must be 16-byte aligned (the step reads them in 16-byte pieces)");
+  const DecodeWs need = decode_ws(*cfg, cache->T_cap, nullptr);
+  MKV_REQUIRE(ws != nullptr && ws_bytes >= need.bytes, MKV_ERR_WORKSPACE,
+              "workspace %zu bytes < %zu needed", ws_bytes, need.bytes);
+  const Split sp = decode_split(*cfg, cache->T_cap);
+  // the launch counts its finished CTAs per batch entry (Hkv x splits) in the top 8 bits of T_len[b]
+  MKV_REQUIRE(cache->T_cap < (1 << 24) && (int64_t)cfg->Hkv * sp.n_split <= 255, MKV_ERR_UNSUPPORTED,
+              "decode_step needs T_cap < 2^24 and Hkv * splits <= 255 (T_cap %lld, Hkv %d, splits %d); use "
+              "mkv_append_kv + mkv_decode_attention",
+              (long long)cache->T_cap, cfg->Hkv, sp.n_split);
+  MKV_CUDA(launch_decode_fp16_family(*cfg, q, *cache, nullptr, out, decode_ws(*cfg, cache->T_cap, ws), sp,
+                                     as_stream(stream), k_new, v_new));
   return MKV_OK;
 }
 

@@ -99,9 +99,11 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
 }
 
 // ---- launchers (return the launch status; arguments already validated) ----
+// k_new / v_new (FP16, H2O): the step's token, appended by the same launch (null: no append).
 cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const mkv_cache& cache,
                                       const int32_t* page_idx, void* out, const DecodeWs& ws,
-                                      const Split& sp, cudaStream_t st);
+                                      const Split& sp, cudaStream_t st, const void* k_new = nullptr,
+                                      const void* v_new = nullptr);
 cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_cache& cache,
                                   const mkv_quant_params& qp, void* out,
                                   const DecodeWs& ws, const Split& sp, cudaStream_t st);
@@ -141,5 +143,6 @@ mkv_status check_fp16_decode_args(const mkv_config* cfg, const mkv_cache* cache,
 cudaError_t take_status_kvquant(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_append(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_rocket(uint32_t* flags, cudaStream_t st);
+cudaError_t take_status_decode(uint32_t* flags, cudaStream_t st);
 
 }  // namespace mkv

@@ -139,3 +139,28 @@ def test_rocket_step_checks(L):
     cache.T_cap = 256
     st = L.mkv_rocket_step(ctypes.byref(wide), 64, 80, 96, ctypes.byref(cache), None, 128, None)
     assert st == mkv.MKV_ERR_UNSUPPORTED and "8 * Hkv" in mkv.mkv_last_error()
+
+
+def test_decode_step_checks(L):
+    """mkv_decode_step is for FP16 and H2O, needs the token's rows 16-byte aligned and counts its
+    CTAs in the top 8 bits of T_len: Hkv x splits <= 255; every rejection happens on the host."""
+    fc = mkv.config(mkv.MKV_FP16, 1, 32, 8, 128)
+    cache = mkv.mkv_cache()
+    cache.T_cap, cache.T_len, cache.k, cache.v = 8192, 8, 256, 512
+    big = ctypes.c_size_t(1 << 40)
+    st = L.mkv_decode_step(ctypes.byref(fc), 64, None, 96, ctypes.byref(cache), 128, 4096, big, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG
+    st = L.mkv_decode_step(ctypes.byref(fc), 64, 88, 96, ctypes.byref(cache), 128, 4096, big, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG and "aligned" in mkv.mkv_last_error()
+    st = L.mkv_decode_step(ctypes.byref(fc), 64, 80, 96, ctypes.byref(cache), 128, 4096, ctypes.c_size_t(16),
+                           None)
+    assert st == mkv.MKV_ERR_WORKSPACE
+    kq = mkv.config(mkv.MKV_KVQUANT, 1, 32, 8, 128, bits=4)
+    st = L.mkv_decode_step(ctypes.byref(kq), 64, 80, 96, ctypes.byref(cache), 128, 4096, big, None)
+    assert st == mkv.MKV_ERR_INVALID_ARG and "FP16 and H2O" in mkv.mkv_last_error()
+    cache.T_cap = 1 << 20                      # 38 splits per unit x 8 kv-heads > 255 CTAs per entry
+    st = L.mkv_decode_step(ctypes.byref(fc), 64, 80, 96, ctypes.byref(cache), 128, 4096, big, None)
+    assert st == mkv.MKV_ERR_UNSUPPORTED and "splits" in mkv.mkv_last_error()
+    cache.T_cap = 1 << 24
+    st = L.mkv_decode_step(ctypes.byref(fc), 64, 80, 96, ctypes.byref(cache), 128, 4096, big, None)
+    assert st == mkv.MKV_ERR_UNSUPPORTED

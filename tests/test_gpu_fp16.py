@@ -110,3 +110,47 @@ def test_capacity_flag():
     assert mkv.mkv_get_status() == mkv.MKV_FLAG_CACHE_FULL
     assert int(cache.t["T_len"][0]) == 4
     assert mkv.mkv_get_status() == 0      # reading clears the word
+
+
+def test_step_equals_append_then_decode():
+    """mkv_decode_step against mkv_append_kv + mkv_decode_attention on twin caches, over steps whose
+    tokens cross chunk and split boundaries and fill one batch entry: identical outputs, K/V rows and
+    lengths; a full cache is not appended, keeps its length, raises MKV_FLAG_CACHE_FULL and attends
+    to its tokens."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(45)
+    B, Hq, Hkv, D = 3, 8, 2, 128
+    T0, T_cap, steps = [1, 126, 250], 256, 12          # entry 2 is full from step 6 on
+    cfg = mkv.config(mkv.MKV_FP16, B, Hq, Hkv, D)
+    K = rng.standard_normal((B, Hkv, T_cap + steps, D)).astype(np.float16)
+    V = rng.standard_normal((B, Hkv, T_cap + steps, D)).astype(np.float16)
+    twins = []
+    for _ in range(2):
+        cache = caches.alloc_cache(cfg, T_cap, device=dev)
+        cache.t["k"].copy_(to_dev(K[:, :, :T_cap], dev))
+        cache.t["v"].copy_(to_dev(V[:, :, :T_cap], dev))
+        cache.t["T_len"].copy_(torch.tensor(T0, dtype=torch.int32))
+        ws, nws = caches.workspace(cfg, T_cap, device=dev)
+        twins.append((cache, ws, nws))
+    (a, wa, na), (c, wc, nc) = twins
+    full_seen = False
+    for s in range(steps):
+        kn = to_dev(K[:, :, T_cap + s], dev)           # rows the caches do not hold yet
+        vn = to_dev(V[:, :, T_cap + s], dev)
+        q = to_dev(rng.standard_normal((B, Hq, D)).astype(np.float16), dev)
+        oa, oc = torch.empty_like(q), torch.empty_like(q)
+        will_fill = [int(a.t["T_len"][b]) >= T_cap for b in range(B)]
+        mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), a.c)
+        fa = mkv.mkv_get_status()
+        mkv.mkv_decode_attention(cfg, q.data_ptr(), a.c, None, 0, oa.data_ptr(), wa.data_ptr(), na)
+        mkv.mkv_decode_step(cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), c.c, oc.data_ptr(), wc.data_ptr(), nc)
+        fc = mkv.mkv_get_status()
+        assert fa == fc == (mkv.MKV_FLAG_CACHE_FULL if any(will_fill) else 0), f"step {s}: flags {fa} {fc}"
+        full_seen |= any(will_fill)
+        assert torch.equal(oa.view(torch.int16), oc.view(torch.int16)), f"step {s}: outputs differ"
+        assert torch.equal(a.t["T_len"], c.t["T_len"]), f"step {s}: T_len"
+        for key in ("k", "v"):
+            assert torch.equal(a.t[key].view(torch.int16), c.t[key].view(torch.int16)), f"step {s}: {key}"
+    assert full_seen
+    assert [int(x) for x in c.t["T_len"]] == [1 + steps, 126 + steps, T_cap]

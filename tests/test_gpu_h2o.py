@@ -137,3 +137,50 @@ def test_full_size_lockstep():
     near = run_h2o(w.B, w.Hq, w.Hkv, w.D, w.T, 24, w.h2o_heavy, w.h2o_recent, x["k"], x["v"], x["q_prompt"],
                    x["q"][:24], dev, False, [(0, 0), (15, 7)], "h2o16k")
     print(f"near-ties adopted: {near}")
+
+
+def test_step_equals_append_then_decode():
+    """mkv_decode_step against mkv_append_kv + mkv_decode_attention on twin H2O caches, each step
+    followed by mkv_h2o_update, over steps that evict and reuse slots: identical outputs, rows,
+    positions, scores, chosen slots and lengths."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(46)
+    B, Hq, Hkv, D, T, H, R, steps = 2, 8, 2, 64, 300, 64, 64, 10
+    cfg = mkv.config(mkv.MKV_H2O, B, Hq, Hkv, D, h2o_heavy=H, h2o_recent=R)
+    T_cap = H + R + 1
+    K = to_dev(rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16), dev)
+    V = to_dev(rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16), dev)
+    QP = to_dev(rng.standard_normal((B, Hq, T, D)).astype(np.float16), dev)
+    Kp, Vp = K[:, :, :T].contiguous(), V[:, :, :T].contiguous()
+    twins = []
+    for _ in range(2):
+        cache = caches.alloc_cache(cfg, T_cap, device=dev)
+        ws, nws = caches.workspace(cfg, max(T, T_cap), device=dev)
+        mkv.mkv_h2o_prefill(cfg, QP.data_ptr(), Kp.data_ptr(), Vp.data_ptr(), T, cache.c, ws.data_ptr(), nws)
+        twins.append((cache, ws, nws))
+    (a, wa, na), (c, wc, nc) = twins
+    keys = ("k", "v", "pos", "acc", "slot", "T_len")
+
+    def same(x, y):
+        if x.dtype == torch.float16:
+            return torch.equal(x.view(torch.int16), y.view(torch.int16))
+        return torch.equal(x, y)
+
+    for key in keys:
+        assert same(a.t[key], c.t[key]), f"prefill: {key}"
+    for s in range(steps):
+        kn = K[:, :, T + s].contiguous()
+        vn = V[:, :, T + s].contiguous()
+        q = to_dev(rng.standard_normal((B, Hq, D)).astype(np.float16), dev)
+        oa, oc = torch.empty_like(q), torch.empty_like(q)
+        mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), a.c)
+        mkv.mkv_decode_attention(cfg, q.data_ptr(), a.c, None, 0, oa.data_ptr(), wa.data_ptr(), na)
+        mkv.mkv_h2o_update(cfg, a.c, wa.data_ptr(), na)
+        mkv.mkv_decode_step(cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), c.c, oc.data_ptr(), wc.data_ptr(), nc)
+        mkv.mkv_h2o_update(cfg, c.c, wc.data_ptr(), nc)
+        assert mkv.mkv_get_status() == 0
+        assert torch.equal(oa.view(torch.int16), oc.view(torch.int16)), f"step {s}: outputs differ"
+        for key in keys:
+            assert same(a.t[key], c.t[key]), f"step {s}: {key}"
+    assert int(c.t["T_len"][0]) == T + steps
