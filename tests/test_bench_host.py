@@ -1,0 +1,33 @@
+"""Host logic of bench.py (no GPU): the committed DRAM-traffic record of a kernel is reported only
+while the kernel source it was captured from is unchanged."""
+import hashlib
+import json
+import os
+
+import bench
+
+
+def test_captured_traffic_follows_the_kernel_source(tmp_path, monkeypatch):
+    src = tmp_path / "k.cu"
+    src.write_text("kernel v1")
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    rec = {"w": {"source": "k.cu", "source_sha256": hashlib.sha256(b"kernel v1").hexdigest(),
+                 "dram_bytes_read": 100, "dram_bytes_write": 20, "summary": "profiles/w.md"}}
+    (prof / "traffic.json").write_text(json.dumps(rec))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.captured_traffic("w") == 120
+    assert bench.captured_traffic("other") is None
+    src.write_text("kernel v2")                  # the kernel changed since the capture
+    assert bench.captured_traffic("w") is None
+
+
+def test_committed_traffic_record_is_well_formed():
+    rec = json.load(open(os.path.join(bench.ROOT, "profiles", "traffic.json")))
+    assert rec
+    for workload, e in rec.items():
+        assert workload in bench.WORKLOADS
+        assert os.path.exists(os.path.join(bench.ROOT, e["source"]))
+        assert os.path.exists(os.path.join(bench.ROOT, e["summary"]))
+        assert e["dram_bytes_read"] > 0 and e["dram_bytes_write"] >= 0
+        assert len(e["source_sha256"]) == 64
