@@ -380,10 +380,29 @@ def whole_job_tokens_per_s(batch: int, world: int, ms: float) -> float:
     return batch * world / (ms * 1e-3)
 
 
+def source_digest(path: str) -> str:
+    """SHA-256 over a kernel source and every header it includes from its own directory, followed
+    recursively (each file once, in the order first reached), so the digest changes whenever any
+    code compiled into the kernel's translation unit from this repository changes."""
+    import hashlib
+    import re
+    h = hashlib.sha256()
+    seen, todo = set(), [os.path.abspath(path)]
+    while todo:
+        f = todo.pop(0)
+        if f in seen or not os.path.exists(f):
+            continue
+        seen.add(f)
+        text = open(f, "rb").read()
+        h.update(os.path.basename(f).encode() + b"\0" + text)
+        for inc in re.findall(rb'#include\s+"([^"]+)"', text):
+            todo.append(os.path.join(os.path.dirname(f), inc.decode()))
+    return h.hexdigest()
+
+
 def captured_traffic(workload: str):
     """DRAM bytes (read + write) of one decode launch from the committed ncu capture of this workload,
-    or None when there is none or the kernel source changed since it was taken."""
-    import hashlib
+    or None when there is none or the kernel source (with its included headers) changed since."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
@@ -391,7 +410,7 @@ def captured_traffic(workload: str):
     if ent is None:
         return None
     src = os.path.join(ROOT, ent["source"])
-    if not os.path.exists(src) or hashlib.sha256(open(src, "rb").read()).hexdigest() != ent["source_sha256"]:
+    if not os.path.exists(src) or source_digest(src) != ent["source_sha256"]:
         return None
     return ent["dram_bytes_read"] + ent["dram_bytes_write"]
 

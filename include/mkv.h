@@ -226,8 +226,11 @@ const char* mkv_last_error(void);
 
 /* ---------------------------------------------------------------- FP16 */
 
-/* Append one token per (batch entry, kv-head) to an FP16, H2O or ROCKET cache.
- * k_new, v_new fp16 [B][Hkv][D] (keys already rotated).  FP16/ROCKET write
+/* Append one token per (batch entry, kv-head) to an FP16, H2O or ROCKET cache:
+ * the decode step's new key and value join the cache before attention (the
+ * per-step cache growth of every configuration of Table 1, Section 2.1; the
+ * H2O slot reuse follows the H2O paragraph, the page bounds the RocketKV
+ * paragraph's second stage).  k_new, v_new fp16 [B][Hkv][D] (keys already rotated).  FP16/ROCKET write
  * slot T_len[b]; H2O writes slot[b][h] and sets pos = T_len[b], acc = 0.
  * ROCKET also fills kmin/kmax of a page the token completes.  T_len[b] += 1.
  * Errors: MKV_ERR_INVALID_ARG for a null field the method needs. */
@@ -236,7 +239,8 @@ mkv_status mkv_append_kv(const mkv_config* cfg, const void* k_new, const void* v
 
 /* Decode attention (every method).  Each query head h of q attends, with a
  * softmax over the attended set, to the cached tokens of kv-head h / G
- * (O1 of the oracle):
+ * (the decode step of every configuration of Table 1; the attended set of
+ * each method is Section 2.1's):
  *   FP16, KVQUANT: slots 0..T_len[b]-1 (KVQUANT dequantizes keys, restores
  *                  outliers, rotates keys by their position, dequantizes
  *                  values -- all fused; Section 2.1 KVQuant paragraph);
@@ -263,12 +267,17 @@ mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_
  * compiled into the library, which every GPU that loads the library keeps
  * until the process exits.
  *  - cfg->method must be MKV_FP16 (else MKV_ERR_UNSUPPORTED).
- *  - The partials of B*Hq*n_split*(D+2) floats (what mkv_workspace_size
- *    reports for this config and T_cap) must fit in 8 MiB, else
+ *  - The call needs exactly the bytes mkv_workspace_size reports for this
+ *    config and T_cap (16 KiB of merge tickets, then the partials m, l and o
+ *    of B*Hq*n_split, B*Hq*n_split and B*Hq*n_split*D floats, each part
+ *    rounded up to 256 bytes); that must be at most 8 MiB, else
  *    MKV_ERR_WORKSPACE and nothing is launched.
  *  - The first call on each device looks up the array's device address
- *    (cudaGetSymbolAddress) and caches it; make that first call before any
- *    stream capture.
+ *    (cudaGetSymbolAddress) and caches it for the process; make that first
+ *    call before any stream capture.  A cudaDeviceReset (or anything else
+ *    that destroys and recreates the device's primary context) invalidates
+ *    the cached address, and the library does not notice: do not call this
+ *    entry point on a device after resetting it.
  *  - All calls share the one array per device: calls whose kernels overlap on
  *    the GPU (different streams, or a second call before the first finished
  *    on another stream) race and corrupt each other's result.  Calls in order
@@ -294,7 +303,9 @@ mkv_status mkv_kvquant_calibrate(const mkv_config* cfg, const void* k_cal, const
  * calibrations computed elsewhere). */
 mkv_status mkv_quant_prepare(const mkv_config* cfg, mkv_quant_params* qparams, void* stream);
 
-/* Quantize n_tokens tokens per (batch entry, kv-head) into the KVQUANT cache
+/* KVQuant quantization (Section 2.1, KVQuant paragraph: keys per channel,
+ * values per token, outliers kept in fp16; Table 1's 2/3/4-bit settings).
+ * Quantize n_tokens tokens per (batch entry, kv-head) into the KVQUANT cache
  * at slots T_len[b]..T_len[b]+n_tokens-1 (n_tokens = T at prefill, 1 per
  * decode step): key outliers by the per-channel range, value outliers as the
  * n_v largest |x| per token, codes by correctly rounded fp32 arithmetic.
@@ -322,7 +333,11 @@ mkv_status mkv_h2o_prefill(const mkv_config* cfg, const void* q_prompt, const vo
                            const void* full_v, int64_t T, mkv_cache* cache, void* ws,
                            size_t ws_bytes, void* stream);
 
-/* After mkv_decode_attention on an H2O cache: add each slot's softmax
+/* H2O's per-step score update and eviction (Section 2.1, H2O paragraph: tokens
+ * are scored by the attention they receive, and the lowest-scored are evicted
+ * to keep the budget).  The softmax probabilities it adds are the logits and
+ * per-head (m, l) that mkv_decode_attention left in `ws` (so they are not
+ * arguments).  After mkv_decode_attention on an H2O cache: add each slot's softmax
  * probability summed over the group's heads to acc, then, if the cache holds
  * more than heavy + recent tokens, evict among all but the `recent` newest
  * positions the lowest-acc token (exact tie: the higher position) and make
@@ -344,7 +359,9 @@ mkv_status mkv_snap_compress(const mkv_config* cfg, const void* q_window, const 
                              const void* full_v, int64_t T, mkv_cache* cache, int32_t* kept_pos,
                              void* ws, size_t ws_bytes, void* stream);
 
-/* RocketKV second-stage page choice for the current query: dims = the
+/* RocketKV second stage, page choice (Section 2.1, RocketKV paragraph: at each
+ * decode step attention reads a subset of the earlier tokens chosen by an
+ * approximate score).  For the current query: dims = the
  * topq_dims largest sum_h |q_h,i| (ties: lower dim); page score = sum_h
  * sum_{i in dims} max(q_h,i * kmin_i, q_h,i * kmax_i) over the full pages
  * before the newest token's page; page_idx_out int32 [B][Hkv][topk_pages]

@@ -5,7 +5,7 @@ The paper: H2O tracks, for every cached token, an accumulated attention score
 exceeds its budget, evicts older tokens with the lowest accumulated score; a
 setting p% keeps p percent of the prompt's tokens.
 
-Readings (listed in DESIGN.md):
+Readings where the paper is silent:
 * budget = H heavy + R recent tokens, H = R = floor(p/200 * T_prompt)
   (or as given); it stays fixed during decode;
 * grouped-query attention: one kept set per kv-head, scored by the sum over

@@ -3,7 +3,7 @@
 The paper states the method's intent: keys are quantized per channel, because
 outliers concentrate in consistent channels, and outlier values are kept in
 uncompressed FP16; a setting is named by its bit width b in {2, 3, 4}.  The
-remaining choices are readings (each listed in the design doc):
+remaining choices are readings of what the paper leaves open:
 
 * keys are quantized before the rotary embedding, per (layer, kv-head,
   channel); values per (token, kv-head);

@@ -1,7 +1,7 @@
 """O6: RocketKV stage 2, hybrid sparse attention at decode (Section 2.1, RocketKV paragraph).
 
 The paper: at each decoding step attention reads only a subset of the earlier
-tokens.  Readings (listed in the design doc), in the spirit of a page-level upper
+tokens.  Readings where the paper is silent, in the spirit of a page-level upper
 bound on q.k:
 
 * the compressed cache is cut into pages of P consecutive slots; page p's

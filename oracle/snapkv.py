@@ -4,7 +4,7 @@ The paper: the first stage uses aggregated attention scores between the input
 context and an observation window at the end of the prompt to find and keep
 the most relevant tokens.
 
-Readings (listed in DESIGN.md):
+Readings where the paper is silent:
 * the window is the last W prompt positions; window query i (position T-W+i)
   attends causally to keys 0..T-W+i;
 * s[j] = sum over the group's G heads and the W window queries of the softmax

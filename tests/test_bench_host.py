@@ -1,6 +1,5 @@
 """Host logic of bench.py (no GPU): the committed DRAM-traffic record of a kernel is reported only
-while the kernel source it was captured from is unchanged."""
-import hashlib
+while the kernel source it was captured from, and every header that source includes, is unchanged."""
 import json
 import os
 
@@ -9,16 +8,22 @@ import bench
 
 def test_captured_traffic_follows_the_kernel_source(tmp_path, monkeypatch):
     src = tmp_path / "k.cu"
-    src.write_text("kernel v1")
+    src.write_text('#include "a.cuh"\nkernel v1')
+    (tmp_path / "a.cuh").write_text('#include "b.h"\nhelpers v1')
+    (tmp_path / "b.h").write_text("decls v1")
     prof = tmp_path / "profiles"
     prof.mkdir()
-    rec = {"w": {"source": "k.cu", "source_sha256": hashlib.sha256(b"kernel v1").hexdigest(),
+    rec = {"w": {"source": "k.cu", "source_sha256": bench.source_digest(str(src)),
                  "dram_bytes_read": 100, "dram_bytes_write": 20, "summary": "profiles/w.md"}}
     (prof / "traffic.json").write_text(json.dumps(rec))
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
     assert bench.captured_traffic("w") == 120
     assert bench.captured_traffic("other") is None
-    src.write_text("kernel v2")                  # the kernel changed since the capture
+    (tmp_path / "b.h").write_text("decls v2")   # a header two includes deep changed
+    assert bench.captured_traffic("w") is None
+    (tmp_path / "b.h").write_text("decls v1")
+    assert bench.captured_traffic("w") == 120
+    src.write_text('#include "a.cuh"\nkernel v2')   # the kernel itself changed
     assert bench.captured_traffic("w") is None
 
 

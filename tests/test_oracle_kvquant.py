@@ -182,3 +182,77 @@ def test_all_outliers_equals_fp16_exactly():
 def test_calibration_limits():
     assert kvquant.n_cal(512) == 512 and kvquant.n_cal(8192) == 4096
     assert kvquant.n_tail(4096, 0.01) == math.ceil(20.48) == 21
+
+
+def _values_with_planted_outliers(n, D, seed):
+    """N(0,1) values with, per token, two entries pushed far outside the rest (+-40, +-25)."""
+    rng = np.random.default_rng(seed)
+    v = rng.normal(size=(n, D))
+    for t in range(n):
+        a, b = rng.choice(D, size=2, replace=False)
+        v[t, a] = 40.0 * (1 if rng.random() < 0.5 else -1)
+        v[t, b] = 25.0 * (1 if rng.random() < 0.5 else -1)
+    return v.astype(np.float16)
+
+
+def test_value_range_is_the_inlier_range():
+    """(lo, hi) of a token = min / max over its entries that are not value outliers, checked
+    against a plain loop; with the two planted outliers per token a range over all entries
+    would reach +-25..40 and fails here."""
+    D, n = 32, 60
+    v = _values_with_planted_outliers(n, D, 21)
+    mask = kvquant.value_outlier_mask(v, 2)
+    lo, hi = kvquant.value_range(v, mask)
+    for t in range(n):
+        inl = [float(v[t, c]) for c in range(D) if not mask[t, c]]
+        assert lo[t] == np.float32(min(inl)) and hi[t] == np.float32(max(inl)), t
+        assert hi[t] < 5.0 and lo[t] > -5.0            # the planted outliers are excluded
+    # a row whose entries are all outliers has the empty range (0, 0)
+    lo1, hi1 = kvquant.value_range(v[:1], np.ones((1, D), bool))
+    assert lo1[0] == 0 and hi1[0] == 0
+
+
+def test_nuq_values_nearest_level_in_value_space():
+    """Value-side twin of the key pin: every inlier dequantizes to the nearest of the token's
+    levels lo + scale * c_j (up to the fp32 rounding of u and of the decision midpoints), and
+    every outlier to its exact fp16 value.  Dropping lo, skipping the de-normalisation or
+    taking the range over all entries each breaks this."""
+    D, n = 16, 400
+    v = _values_with_planted_outliers(n, D, 22)
+    k = _data(n, D, 23)
+    for bits in (2, 3, 4):
+        p = kvquant.calibrate(k[:300], v[:300], bits, "nuq", 0.02)
+        qh = kvquant.quantize_head(k, v, p)
+        vd = kvquant.dequantize_values(qh.v_codes, qh.v_mask, qh.v_lo, qh.v_scale, v, p)
+        x = v.astype(np.float64)
+        levels = (qh.v_lo.astype(np.float64)[:, None, None]
+                  + qh.v_scale.astype(np.float64)[:, None, None] * p.v_cb.astype(np.float64)[None, :, :])
+        best = np.min(np.abs(x[:, :, None] - levels), axis=2)
+        got = np.abs(x - vd)
+        slack = 1e-6 * (1.0 + qh.v_scale.astype(np.float64))[:, None]
+        inl = ~qh.v_mask
+        assert np.all(got[inl] <= (best + slack)[inl])
+        # the level grid spans the inlier range: no inlier is farther than the widest gap
+        assert np.all(got[inl] <= np.broadcast_to(qh.v_scale.astype(np.float64)[:, None], got.shape)[inl])
+        assert np.all(got[qh.v_mask] == 0)
+        assert qh.v_mask.sum() == kvquant.n_value_outliers(D, 0.02) * n
+
+
+def test_many_centroid_nuq_approaches_fp16():
+    """Many-centroid limit of the NUQ path (oracle only): as the centroids per channel grow from
+    2^4 to 2^6 and 2^8 (keys and values), the fused decode approaches FP16 attention, ending
+    within 5e-3 of it; a value path that skipped the de-normalisation or dropped lo would stay
+    O(1) away at any bit width."""
+    rng = np.random.default_rng(24)
+    D, n = 32, 1024
+    k = _data(n, D, 25, scale_ch=np.geomspace(0.3, 3, D))
+    v = _data(n, D, 26)
+    q = rng.normal(size=(4, D)).astype(np.float16)
+    ref = _fp16_reference(q, k, v, 10000.0)
+    errs = []
+    for bits in (4, 6, 8):
+        p = kvquant.calibrate(k, v, bits, "nuq", 0.01)
+        out = kvquant.decode_head(q, kvquant.quantize_head(k, v, p), p, 10000.0)
+        errs.append(np.abs(out - ref).max())
+    assert errs[0] > errs[1] > errs[2]
+    assert errs[2] < 5e-3 and errs[2] * 5 < errs[0]
