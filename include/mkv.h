@@ -233,6 +233,9 @@ const char* mkv_last_error(void);
  * paragraph's second stage).  k_new, v_new fp16 [B][Hkv][D] (keys already rotated).  FP16/ROCKET write
  * slot T_len[b]; H2O writes slot[b][h] and sets pos = T_len[b], acc = 0.
  * ROCKET also fills kmin/kmax of a page the token completes.  T_len[b] += 1.
+ * A batch entry where any kv-head has no room (FP16/ROCKET: T_len = T_cap;
+ * H2O: a slot outside [0, T_cap)) gets no row in any kv-head, keeps T_len and
+ * sets MKV_FLAG_CACHE_FULL.
  * Errors: MKV_ERR_INVALID_ARG for a null field the method needs. */
 mkv_status mkv_append_kv(const mkv_config* cfg, const void* k_new, const void* v_new,
                          mkv_cache* cache, void* stream);
@@ -393,8 +396,8 @@ mkv_status mkv_rocket_decode(const mkv_config* cfg, const void* q, const mkv_cac
  * (H2O: with position T_len and a zero score).  While the launch runs, the
  * top 8 bits of T_len[b] count its finished CTAs (the last one stores the new
  * length), so nothing else may read or write T_len of this cache during the
- * call.  A batch entry with no room is not appended (MKV_FLAG_CACHE_FULL, read
- * by mkv_get_status) and attends to its existing tokens.  MKV_ERR_UNSUPPORTED
+ * call.  A batch entry with no room in some kv-head is not appended in any
+ * (MKV_FLAG_CACHE_FULL, read by mkv_get_status) and attends to its existing tokens.  MKV_ERR_UNSUPPORTED
  * when T_cap >= 2^24 or Hkv x (the decode's splits) > 255: use the two calls
  * then. */
 mkv_status mkv_decode_step(const mkv_config* cfg, const void* q, const void* k_new, const void* v_new,

@@ -36,14 +36,16 @@ __global__ void append_kernel(const AppendArgs a) {
   __shared__ int ok;
   if (threadIdx.x == 0) ok = 1;
   __syncthreads();
-  for (int e = threadIdx.x; e < a.Hkv * nc; e += blockDim.x) {
+  // all or nothing per batch entry: if any kv-head has no room, no row is written
+  for (int kvh = threadIdx.x; kvh < a.Hkv; kvh += blockDim.x) {
+    const int64_t s = a.mode == 1 ? a.slot[(int64_t)b * a.Hkv + kvh] : t;
+    if (s < 0 || s >= a.T_cap) ok = 0;
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; ok && e < a.Hkv * nc; e += blockDim.x) {
     const int kvh = e / nc, col = e % nc;
     const int64_t bh = (int64_t)b * a.Hkv + kvh;
     const int64_t s = a.mode == 1 ? a.slot[bh] : t;
-    if (s < 0 || s >= a.T_cap) {
-      ok = 0;
-      continue;
-    }
     a.k[(bh * a.T_cap + s) * nc + col] = a.k_new[bh * nc + col];
     a.v[(bh * a.T_cap + s) * nc + col] = a.v_new[bh * nc + col];
     if (a.mode == 1 && col == 0) {

@@ -122,7 +122,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
         ok_b = ok_b && sh >= 0 && sh < a.T_cap;
       }
       const int sh = a.slot[bh];
-      s_new = (sh >= 0 && sh < a.T_cap) ? sh : -1;
+      s_new = ok_b ? sh : -1;          // all or nothing per batch entry, as mkv_append_kv
     }
   }
 

@@ -18,6 +18,16 @@ EPS_REL, EPS_ABS = 1e-5, 1e-7
 HERE = os.path.dirname(os.path.abspath(__file__))
 
 
+def record(tag, near, decisions):
+    """Report a lockstep run's near-tie count: printed, and appended as a JSON line to the file named
+    by MKV_NEAR_TIES_OUT when that is set (the committed summary is made from those lines)."""
+    print(f"NEAR-TIES {tag}: {near} of {decisions} decisions")
+    path = os.environ.get("MKV_NEAR_TIES_OUT")
+    if path:
+        with open(path, "a") as f:
+            f.write(json.dumps({"run": tag, "near_ties": int(near), "decisions": int(decisions)}) + "\n")
+
+
 def tiny_seed():
     with open(os.path.join(HERE, "golden", "tiny_seed.json")) as f:
         return json.load(f)["seed"]

@@ -154,3 +154,33 @@ def test_step_equals_append_then_decode():
             assert torch.equal(a.t[key].view(torch.int16), c.t[key].view(torch.int16)), f"step {s}: {key}"
     assert full_seen
     assert [int(x) for x in c.t["T_len"]] == [1 + steps, 126 + steps, T_cap]
+
+
+def test_step_vs_oracle_bench_shape():
+    """mkv_decode_step at the FP16 bench shape (B=8, T=8192, 32/8/128, the bench's T_cap): two steps
+    against fp64 attention over the T+1 and T+2 tokens, every head of batch entries 0, 4 and 7."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(47)
+    B, Hq, Hkv, D, T, steps = 8, 32, 8, 128, 8192, 2
+    T_cap = T + 4 * 25 + 8 + 64
+    cfg = mkv.config(mkv.MKV_FP16, B, Hq, Hkv, D)
+    K = rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16)
+    V = rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16)
+    Q = rng.standard_normal((steps, B, Hq, D)).astype(np.float16)
+    cache = caches.alloc_cache(cfg, T_cap, device=dev)
+    cache.t["k"][:, :, :T] = to_dev(K[:, :, :T], dev)
+    cache.t["v"][:, :, :T] = to_dev(V[:, :, :T], dev)
+    cache.t["T_len"].fill_(T)
+    ws, nws = caches.workspace(cfg, T_cap, device=dev)
+    for s in range(steps):
+        kn, vn = to_dev(K[:, :, T + s], dev), to_dev(V[:, :, T + s], dev)
+        qt = to_dev(Q[s], dev)
+        out = torch.empty_like(qt)
+        mkv.mkv_decode_step(cfg, qt.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, out.data_ptr(),
+                            ws.data_ptr(), nws)
+        got = out.float().cpu().numpy()
+        for b in (0, 4, 7):
+            assert_close(got[b], _ref(K, V, Q[s], b, T + s + 1), f"step {s} b{b}")
+    assert mkv.mkv_get_status() == 0
+    assert [int(x) for x in cache.t["T_len"]] == [T + steps] * B

@@ -8,7 +8,7 @@ from oracle import attention, h2o
 from paper_2609_07966_gb300 import caches
 
 from gpu_util import assert_close, to_dev, torch_cuda
-from lockstep import check_evict, check_topk, tiny_seed
+from lockstep import check_evict, check_topk, record, tiny_seed
 
 pytestmark = pytest.mark.gpu
 
@@ -20,9 +20,11 @@ def _state(cache, b, h):
     return pos, acc, held
 
 
-def run_h2o(B, Hq, Hkv, D, T, steps, H, R, K, V, QP, Q, dev, exact, units, tag):
+def run_h2o(B, Hq, Hkv, D, T, steps, H, R, K, V, QP, Q, dev, exact, units, tag, step_api=False):
     """K, V [B,Hkv,T+steps,D]; QP [B,Hq,T,D]; Q [steps,B,Hq,D] (device tensors).
-    units: (b, kv-head) pairs checked against the oracle in lockstep."""
+    units: (b, kv-head) pairs checked against the oracle in lockstep.
+    step_api: each step through mkv_decode_step (the token's append and the attention in one
+    launch, as the bench runs it) instead of mkv_append_kv + mkv_decode_attention."""
     torch = torch_cuda()
     G = Hq // Hkv
     cfg = mkv.config(mkv.MKV_H2O, B, Hq, Hkv, D, h2o_heavy=H, h2o_recent=R)
@@ -33,7 +35,7 @@ def run_h2o(B, Hq, Hkv, D, T, steps, H, R, K, V, QP, Q, dev, exact, units, tag):
     mkv.mkv_h2o_prefill(cfg, QP.data_ptr(), Kp.data_ptr(), Vp.data_ptr(), T, cache.c, ws.data_ptr(), nws)
     torch.cuda.synchronize()
     host = {}
-    near = 0
+    near = decisions = 0
     for (b, h) in units:
         k = K[b, h].cpu().numpy()
         v = V[b, h].cpu().numpy()
@@ -44,6 +46,7 @@ def run_h2o(B, Hq, Hkv, D, T, steps, H, R, K, V, QP, Q, dev, exact, units, tag):
         rest = np.arange(max(T - R, 0))
         heavy_got = got_keep[got_keep < T - R]
         near += check_topk(acc0[rest], rest, min(H, rest.shape[0]), heavy_got, exact, f"{tag} keep b{b} h{h}")
+        decisions += 1
         assert set(range(max(T - R, 0), T)) <= set(got_keep.tolist())
         # scores of the kept tokens: fp32 GPU column sums vs fp64
         np.testing.assert_allclose(acc[held], acc0[pos[held]], rtol=2e-4, atol=1e-5)
@@ -54,9 +57,17 @@ def run_h2o(B, Hq, Hkv, D, T, steps, H, R, K, V, QP, Q, dev, exact, units, tag):
         vn = V[:, :, T + s].contiguous()
         q = Q[s].contiguous()
         out = torch.empty_like(q)
-        mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
-        pos_before = cache.t["pos"].clone()
-        mkv.mkv_decode_attention(cfg, q.data_ptr(), cache.c, None, 0, out.data_ptr(), ws.data_ptr(), nws)
+        if step_api:
+            # the cache as the append would leave it: the new position in each (b, kv-head)'s next slot
+            pos_before = cache.t["pos"].clone()
+            sl = cache.t["slot"].long()
+            pos_before.scatter_(2, sl.unsqueeze(2), torch.full_like(sl.unsqueeze(2), T + s, dtype=pos_before.dtype))
+            mkv.mkv_decode_step(cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, out.data_ptr(),
+                                ws.data_ptr(), nws)
+        else:
+            mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), cache.c)
+            pos_before = cache.t["pos"].clone()
+            mkv.mkv_decode_attention(cfg, q.data_ptr(), cache.c, None, 0, out.data_ptr(), ws.data_ptr(), nws)
         mkv.mkv_h2o_update(cfg, cache.c, ws.data_ptr(), nws)
         got = out.float().cpu().numpy()
         for (b, h) in units:
@@ -74,6 +85,7 @@ def run_h2o(B, Hq, Hkv, D, T, steps, H, R, K, V, QP, Q, dev, exact, units, tag):
                 assert len(gone) == 1, f"{tag} step {s}: evicted {gone}"
                 n = check_evict(cand[0], cand[1], gone[0], exact, f"{tag} step {s} b{b} h{h}")
                 near += n
+                decisions += 1
                 if n:
                     _, st2, _, _ = h2o.decode_step(st, qh, k[T + s], v[T + s], T + s, H, R, forced_victim=gone[0])
             ordr = np.argsort(st2.pos)
@@ -82,6 +94,7 @@ def run_h2o(B, Hq, Hkv, D, T, steps, H, R, K, V, QP, Q, dev, exact, units, tag):
             np.testing.assert_allclose([gacc[p] for p in st2.pos[ordr]], st2.acc[ordr], rtol=2e-4, atol=1e-5)
             host[(b, h)] = (k, v, st2)
     assert mkv.mkv_get_status() == 0
+    record(f"h2o {tag}{' (one-launch step)' if step_api else ''}", near, decisions)
     return near
 
 
@@ -92,9 +105,10 @@ def test_tiny_exact():
     x = synth.host_inputs(w, seed=tiny_seed())
     K, V = to_dev(x["k"][0], dev), to_dev(x["v"][0], dev)
     QP, Q = to_dev(x["q_prompt"][0], dev), to_dev(x["q"][:, 0], dev)
-    near = run_h2o(w.B, w.Hq, w.Hkv, w.D, w.T, w.steps, w.h2o_heavy, w.h2o_recent, K, V, QP, Q, dev, True,
-                   [(0, 0), (0, 1)], "tiny")
-    assert near == 0
+    for step_api in (False, True):
+        near = run_h2o(w.B, w.Hq, w.Hkv, w.D, w.T, w.steps, w.h2o_heavy, w.h2o_recent, K, V, QP, Q, dev, True,
+                       [(0, 0), (0, 1)], f"tiny{'-step' if step_api else ''}", step_api)
+        assert near == 0
 
 
 def test_budget_covers_context_is_full_attention():
@@ -128,15 +142,16 @@ def test_shapes_lockstep(G, D):
 
 
 def test_full_size_lockstep():
-    """B=16, T=16384, 32/8/128, 20% budget (1638 heavy + 1638 recent), heavy-hitter inputs:
-    one layer, 24 steps, two (batch, kv-head) units in lockstep with the oracle."""
+    """B=16, T=16384, 32/8/128, 20% budget (1638 heavy + 1638 recent), heavy-hitter inputs, the
+    bench's one-launch step (mkv_decode_step + mkv_h2o_update): one layer, 64 steps, four
+    (batch, kv-head) units in lockstep with the oracle."""
     torch = torch_cuda()
     dev = torch.device("cuda")
     w = synth.h2o_16k(20)
-    x = synth.device_layer_inputs(w, seed=11, layer=0, device=dev, n_tokens=w.T + 24, with_prompt_queries=True)
-    near = run_h2o(w.B, w.Hq, w.Hkv, w.D, w.T, 24, w.h2o_heavy, w.h2o_recent, x["k"], x["v"], x["q_prompt"],
-                   x["q"][:24], dev, False, [(0, 0), (15, 7)], "h2o16k")
-    print(f"near-ties adopted: {near}")
+    n = 64
+    x = synth.device_layer_inputs(w, seed=11, layer=0, device=dev, n_tokens=w.T + n, with_prompt_queries=True)
+    run_h2o(w.B, w.Hq, w.Hkv, w.D, w.T, n, w.h2o_heavy, w.h2o_recent, x["k"], x["v"], x["q_prompt"],
+            x["q"][:n], dev, False, [(0, 0), (5, 3), (10, 6), (15, 7)], "h2o20-b16-t16384", step_api=True)
 
 
 def test_step_equals_append_then_decode():
@@ -174,13 +189,27 @@ def test_step_equals_append_then_decode():
         vn = V[:, :, T + s].contiguous()
         q = to_dev(rng.standard_normal((B, Hq, D)).astype(np.float16), dev)
         oa, oc = torch.empty_like(q), torch.empty_like(q)
+        full = s == 4                       # batch entry 1, kv-head 0 has no free slot at this step
+        if full:
+            len_before = [int(x) for x in a.t["T_len"]]
+            saved = int(a.t["slot"][1, 0])
+            for cc in (a, c):
+                cc.t["slot"][1, 0] = T_cap
         mkv.mkv_append_kv(cfg, kn.data_ptr(), vn.data_ptr(), a.c)
+        fa = mkv.mkv_get_status()
         mkv.mkv_decode_attention(cfg, q.data_ptr(), a.c, None, 0, oa.data_ptr(), wa.data_ptr(), na)
         mkv.mkv_h2o_update(cfg, a.c, wa.data_ptr(), na)
         mkv.mkv_decode_step(cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), c.c, oc.data_ptr(), wc.data_ptr(), nc)
+        fc = mkv.mkv_get_status()
         mkv.mkv_h2o_update(cfg, c.c, wc.data_ptr(), nc)
         assert mkv.mkv_get_status() == 0
+        want = mkv.MKV_FLAG_CACHE_FULL if full else 0
+        assert fa == fc == want, f"step {s}: flags {fa} {fc}"
+        if full:                            # no kv-head of that batch entry was appended; length kept
+            assert int(c.t["T_len"][1]) == len_before[1] and int(c.t["T_len"][0]) == len_before[0] + 1
+            for cc in (a, c):               # nothing was evicted there: give the slot back
+                cc.t["slot"][1, 0] = saved
         assert torch.equal(oa.view(torch.int16), oc.view(torch.int16)), f"step {s}: outputs differ"
         for key in keys:
             assert same(a.t[key], c.t[key]), f"step {s}: {key}"
-    assert int(c.t["T_len"][0]) == T + steps
+    assert int(c.t["T_len"][0]) == T + steps and int(c.t["T_len"][1]) == T + steps - 1

@@ -10,7 +10,7 @@ from oracle import attention, rocket, snapkv
 from paper_2609_07966_gb300 import caches
 
 from gpu_util import assert_close, to_dev, torch_cuda
-from lockstep import check_topk, tiny_seed
+from lockstep import check_topk, record, tiny_seed
 
 pytestmark = pytest.mark.gpu
 
@@ -32,7 +32,7 @@ def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev,
                           ws.data_ptr(), nws)
     torch.cuda.synchronize()
     assert int(cache.t["T_len"][0]) == kept_n
-    near = 0
+    near = decisions = 0
     host = {}
     for (b, h) in units:
         k = K[b, h].cpu().numpy()
@@ -47,6 +47,7 @@ def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev,
             pooled = snapkv.max_pool(s, pool)
             pre = np.arange(T - W)
             near += check_topk(pooled, pre, keep - W, got[got < T - W], exact, f"{tag} snap b{b} h{h}")
+            decisions += 1
             assert np.array_equal(got[got >= T - W], np.arange(T - W, T))
         # the compact cache holds exactly the kept rows, and page min/max match
         gk = cache.t["k"][b, h, :kept_n].cpu().numpy()
@@ -89,9 +90,11 @@ def run_rocket(B, Hq, Hkv, D, T, steps, W, pool, keep, kp, rd, K, V, QW, Q, dev,
             ns = rocket.n_scored_pages(n, 16)
             nn = check_topk(scores, np.arange(ns), min(kp, ns), sel_got, exact, f"{tag} pages step {s} b{b} h{h}")
             near += nn
+            decisions += 1
             ref, _, _ = rocket.decode(qh, np.array(Kc), np.array(Vc), n, 16, kp, rd, forced_pages=sel_got)
             assert_close(got[b, h * G:(h + 1) * G], ref, f"{tag} step {s} b{b} h{h}")
     assert mkv.mkv_get_status() == 0
+    record(f"rocket {tag} ({ {False: 'two calls', True: 'fused decode', 'step': 'one-launch step'}[fused] })", near, decisions)
     return near
 
 
@@ -142,16 +145,18 @@ def test_shapes_lockstep(G, D, fused):
 
 @pytest.mark.parametrize("fused", [False, True, "step"])
 def test_full_size_lockstep(fused):
-    """B=4, T=32768 -> keep 4096, W=32, pool 7, top-64 pages over top-32 dims: one layer,
-    16 steps, two (batch, kv-head) units in lockstep with the oracle."""
+    """B=4, T=32768 -> keep 4096, W=32, pool 7, top-64 pages over top-32 dims: one layer in
+    lockstep with the oracle -- 16 steps on two (batch, kv-head) units for the two-call and fused
+    paths, 48 steps on four units for the one-launch step the bench runs."""
     torch = torch_cuda()
     dev = torch.device("cuda")
     w = synth.rocket_32k(1024)
-    x = synth.device_layer_inputs(w, seed=12, layer=0, device=dev, n_tokens=w.T + 16, with_prompt_queries=True)
+    n, units = (48, [(0, 0), (1, 2), (2, 5), (3, 7)]) if fused == "step" else (16, [(0, 0), (3, 7)])
+    x = synth.device_layer_inputs(w, seed=12, layer=0, device=dev, n_tokens=w.T + n, with_prompt_queries=True)
     QW = x["q_prompt"][:, :, w.T - w.snap_window:].contiguous()
-    near = run_rocket(w.B, w.Hq, w.Hkv, w.D, w.T, 16, w.snap_window, w.snap_pool, w.snap_keep, w.topk_pages,
-                      w.topq_dims, x["k"], x["v"], QW, x["q"][:16], dev, False, [(0, 0), (3, 7)], "rocket32k", fused)
-    print(f"near-ties adopted: {near}")
+    tag = "rocket1024-b4-t32768" + {False: "-two-calls", True: "-fused", "step": "-step"}[fused]
+    run_rocket(w.B, w.Hq, w.Hkv, w.D, w.T, n, w.snap_window, w.snap_pool, w.snap_keep, w.topk_pages,
+               w.topq_dims, x["k"], x["v"], QW, x["q"][:n], dev, False, units, tag, fused)
 
 
 def test_fused_short_contexts():
