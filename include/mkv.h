@@ -254,7 +254,8 @@ mkv_status mkv_append_kv(const mkv_config* cfg, const void* k_new, const void* v
  * out fp16 [B][Hq][D].  For H2O the call also leaves, in ws, the per-slot
  * logits and per-head softmax statistics that mkv_h2o_update reads.
  * qparams: KVQUANT only (else NULL).  ws/ws_bytes: workspace.
- * KVQUANT also requires k_out_cap <= INT32_MAX and T_cap < INT32_MAX
+ * KVQUANT also requires 16-byte aligned k_codes and v_codes (MKV_ERR_INVALID_ARG
+ * otherwise), and k_out_cap <= INT32_MAX and T_cap < INT32_MAX
  * (MKV_ERR_UNSUPPORTED otherwise). */
 mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_cache* cache,
                                 const mkv_quant_params* qparams, const int32_t* page_idx,

@@ -346,6 +346,8 @@ mkv_status mkv_decode_attention(const mkv_config* cfg, const void* q, const mkv_
     MKV_TRY(check_qparams(cfg, qparams, true));
     MKV_REQUIRE(qparams->rope && qparams->rope_len >= std::max<int64_t>(cache->T_cap, 64), MKV_ERR_INVALID_ARG,
                 "KVQUANT decode needs a rope table with rope_len >= max(T_cap, 64)");
+    MKV_REQUIRE(((uintptr_t)cache->k_codes | (uintptr_t)cache->v_codes) % 16 == 0, MKV_ERR_INVALID_ARG,
+                "KVQUANT decode stages k_codes / v_codes in 16-byte pieces: both must be 16-byte aligned");
     MKV_REQUIRE(cache->k_out_cap <= INT32_MAX && cache->T_cap < INT32_MAX, MKV_ERR_UNSUPPORTED,
                 "KVQUANT decode indexes key outliers and tokens with 32 bits (k_out_cap %lld, T_cap %lld)",
                 (long long)cache->k_out_cap, (long long)cache->T_cap);

@@ -94,6 +94,30 @@ def test_calibration_bit_exact(bits, mode, D, N):
             assert bad == 0, f"{key}: {bad} centroids differ"
 
 
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_calibration_bit_exact_bench_size(bits):
+    """The bench's calibration: N_cal = 4096 tokens, D = 128, 2^b NUQ centroids per channel, keys with
+    per-channel scales log-uniform in [0.1, 10]: thresholds and fp16 centroids bit-exact."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    N, D, Hkv = 4096, 128, 1
+    k, v = _data(1, Hkv, N, D, seed=400 + bits)
+    plist = _oracle_params(k, v, N, bits, "nuq", 0.01)
+    cfg = make_cfg(1, 4 * Hkv, Hkv, D, bits, "nuq")
+    qp = caches.alloc_quant_params(cfg, 64, device=dev)
+    ws, nws = caches.workspace(cfg, N, device=dev)
+    kd, vd = to_dev(k[0], dev), to_dev(v[0], dev)
+    mkv.mkv_kvquant_calibrate(cfg, kd.data_ptr(), vd.data_ptr(), N, N, qp.c, ws.data_ptr(), nws)
+    torch.cuda.synchronize()
+    for key in ("t_lo", "t_hi"):
+        ref = np.stack([getattr(p, key) for p in plist]).astype(np.float32)
+        assert np.array_equal(qp.t[key].cpu().numpy().view(np.uint32), ref.view(np.uint32)), key
+    for key in ("k_cb", "v_cb"):
+        ref = np.stack([getattr(p, key) for p in plist])
+        bad = (qp.t[key].cpu().numpy().view(np.uint16) != ref.view(np.uint16)).sum()
+        assert bad == 0, f"{key}: {bad} centroids differ"
+
+
 def _quantized_cache(cfg, k, v, plist, T, steps, dev, T_cap=None):
     """Bulk-quantize T tokens, then append `steps` single tokens; returns cache, qparams."""
     torch = torch_cuda()
