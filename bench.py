@@ -10,6 +10,14 @@ configuration); other workloads via --workload.  Inputs are synthetic and
 seeded (synth), every layer has its own cache buffers, and one step reads
 more than the 129 MB L2 holds, so no flush is needed between steps.
 
+Besides the headline workload the line carries ``per_config`` (the other configurations at their own
+sizes: FP16 8K, KVQuant 3/2-bit, H2O 20 % at 16K, RocketKV 1024 at 32K) and ``sweep``: the ten
+configurations (FP16; KVQuant NUQ 4/3/2-bit; H2O 10/20/40 %; RocketKV budgets 1024/2048/4096) at
+contexts 4K/16K/64K/128K with batch 32/16/4/1, each a 32-layer step.  There the H2O decode cache is
+filled directly with the budget's heavy and recent slots (scoring a 128K prompt is not part of a
+decode step).  Every row gives the step time, tokens/s, the decode launch's algorithmic bytes,
+GB/s and fraction of the measured and of the 8 TB/s peak, and the resident and peak KV bytes.
+
 Under torchrun each rank runs an independent replica on its own GPU (the
 units -- batch entries, heads, layers -- are independent; no collective).
 --impl reference times the fp64 CPU oracle on a bounded sample instead.
@@ -98,12 +106,16 @@ class ClockSampler:
 class Runner:
     """All layers of one workload resident on the device, plus the step."""
 
-    def __init__(self, name: str, w, dev, seed: int, extra_steps: int):
+    def __init__(self, name: str, w, dev, seed: int, extra_steps: int, method: str | None = None,
+                 synthetic_h2o_cache: bool = False):
+        """synthetic_h2o_cache: fill the H2O decode cache (heavy + recent slots, their positions and
+        scores) directly from the seeded inputs instead of scoring the whole prompt (the sweep's long
+        contexts); the decode step then does exactly the same work."""
         import torch
         import paper_2609_07966_gb300 as mkv
         from paper_2609_07966_gb300 import caches
         self.torch, self.mkv, self.name, self.w, self.dev = torch, mkv, name, w, dev
-        self.method = METHOD_OF[name]
+        self.method = method or METHOD_OF[name]
         B, Hq, Hkv, D = w.B, w.Hq, w.Hkv, w.D
         mk = {"fp16": mkv.MKV_FP16, "kvquant": mkv.MKV_KVQUANT, "h2o": mkv.MKV_H2O, "rocket": mkv.MKV_ROCKET}
         kw = {}
@@ -131,8 +143,10 @@ class Runner:
             mkv.mkv_rope_table(D, w.theta, self.T_cap, self.rope.data_ptr())
         t_setup = time.perf_counter()
         for l in range(w.L):
-            x = synth.device_layer_inputs(w, seed, l, device=dev, n_tokens=w.T + 1,
-                                          with_prompt_queries=self.method in ("h2o", "rocket"))
+            syn = self.method == "h2o" and synthetic_h2o_cache
+            n_tok = w.h2o_heavy + w.h2o_recent + 1 if syn else w.T + 1
+            x = synth.device_layer_inputs(w, seed, l, device=dev, n_tokens=n_tok,
+                                          with_prompt_queries=self.method in ("h2o", "rocket") and not syn)
             cache = caches.alloc_cache(self.cfg, self.T_cap, device=dev)
             qp = None
             if self.method == "fp16":
@@ -152,6 +166,20 @@ class Runner:
                 vp = x["v"][:, :, :w.T].contiguous()
                 mkv.mkv_quantize_kv(self.cfg, qp.c, kp.data_ptr(), vp.data_ptr(), w.T, cache.c)
                 del kp, vp
+            elif self.method == "h2o" and syn:
+                n = w.h2o_heavy + w.h2o_recent
+                cache.t["k"][:, :, :n] = x["k"][:, :, :n]
+                cache.t["v"][:, :, :n] = x["v"][:, :, :n]
+                pos = torch.empty(n, dtype=torch.int32, device=dev)
+                hv = torch.arange(w.h2o_heavy, device=dev, dtype=torch.int64)
+                pos[:w.h2o_heavy] = (hv * (w.T - w.h2o_recent) // max(w.h2o_heavy, 1)).to(torch.int32)
+                pos[w.h2o_heavy:] = torch.arange(w.T - w.h2o_recent, w.T, device=dev, dtype=torch.int32)
+                cache.t["pos"][:, :, :n] = pos
+                g = torch.Generator(device=dev)
+                g.manual_seed(seed * 1000 + l)
+                cache.t["acc"][:, :, :n] = torch.rand((B, Hkv, n), generator=g, device=dev)
+                cache.t["slot"].fill_(n)
+                cache.t["T_len"].fill_(w.T)
             elif self.method == "h2o":
                 kp = x["k"][:, :, :w.T].contiguous()
                 vp = x["v"][:, :, :w.T].contiguous()
@@ -168,8 +196,8 @@ class Runner:
                 self.pidx.append(torch.zeros((B, Hkv, w.topk_pages), dtype=torch.int32, device=dev))
             self.layers.append((cache, qp))
             self.q.append(x["q"][0].contiguous())
-            self.kn.append(x["k"][:, :, w.T].contiguous())
-            self.vn.append(x["v"][:, :, w.T].contiguous())
+            self.kn.append(x["k"][:, :, n_tok - 1].contiguous())
+            self.vn.append(x["v"][:, :, n_tok - 1].contiguous())
             self.out.append(torch.empty((B, Hq, D), dtype=torch.float16, device=dev))
             del x
         torch.cuda.synchronize()
@@ -177,6 +205,20 @@ class Runner:
         flags = mkv.mkv_get_status()
         assert flags == 0, f"device status flags {flags:#x} after setup"
         self.graph = None
+        self.step_fused = True
+        # RocketKV: the fused one-launch step unless this shape is too large for it (then append,
+        # page choice and sparse attention as three calls)
+        # (the fused step ranks and attends within one cluster per unit, which suits the 64 pages of
+        # the 1024-token budget; larger page budgets use the split-KV decode over the page list)
+        self.rocket_fused = self.method == "rocket" and w.topk_pages <= 64
+        if self.rocket_fused:
+            try:
+                mkv.mkv_rocket_decode(self.cfg, self.q[0].data_ptr(), self.layers[0][0].c, 0, self.out[0].data_ptr())
+                torch.cuda.synchronize()
+            except mkv.MkvError as e:
+                if e.status != mkv.MKV_ERR_UNSUPPORTED:
+                    raise
+                self.rocket_fused = False
 
     def append(self, l, kn=None, vn=None):
         mkv = self.mkv
@@ -194,7 +236,13 @@ class Runner:
         q = self.q[l] if q is None else q
         out = self.out[l] if out is None else out
         if self.method == "rocket":           # page choice + sparse attention in one launch
-            mkv.mkv_rocket_decode(self.cfg, q.data_ptr(), cache.c, 0, out.data_ptr())
+            if self.rocket_fused:
+                mkv.mkv_rocket_decode(self.cfg, q.data_ptr(), cache.c, 0, out.data_ptr())
+            else:
+                pidx = self.pidx[l]
+                mkv.mkv_rocket_select(self.cfg, q.data_ptr(), cache.c, pidx.data_ptr())
+                mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, None, pidx.data_ptr(), out.data_ptr(),
+                                         self.ws.data_ptr(), self.nws)
             return
         mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, qp.c if qp else None, 0, out.data_ptr(),
                                  self.ws.data_ptr(), self.nws)
@@ -204,6 +252,10 @@ class Runner:
         (update scores)."""
         mkv = self.mkv
         cache, _ = self.layers[l]
+        if self.method == "rocket" and not self.rocket_fused:
+            self.append(l, kn, vn)
+            self.decode(l, q, out)
+            return
         if self.method == "rocket":           # append, page choice and attention in one launch
             kn = self.kn[l] if kn is None else kn
             vn = self.vn[l] if vn is None else vn
@@ -211,13 +263,21 @@ class Runner:
             out = self.out[l] if out is None else out
             mkv.mkv_rocket_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, 0, out.data_ptr())
             return
-        if self.method in ("fp16", "h2o"):    # append and attention in one launch, then (H2O) the update
+        if self.method in ("fp16", "h2o") and self.step_fused:
+            # append and attention in one launch, then (H2O) the update
             kn = self.kn[l] if kn is None else kn
             vn = self.vn[l] if vn is None else vn
             q = self.q[l] if q is None else q
             out = self.out[l] if out is None else out
-            mkv.mkv_decode_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, out.data_ptr(),
-                                self.ws.data_ptr(), self.nws)
+            try:
+                mkv.mkv_decode_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, out.data_ptr(),
+                                    self.ws.data_ptr(), self.nws)
+            except mkv.MkvError as e:
+                # too many splits for the step's ticket counter: nothing was launched; two calls instead
+                if e.status != mkv.MKV_ERR_UNSUPPORTED:
+                    raise
+                self.step_fused = False
+                return self.layer_step(l, q, kn, vn, out)
             if self.method == "h2o":
                 mkv.mkv_h2o_update(self.cfg, cache.c, self.ws.data_ptr(), self.nws)
             return
@@ -253,31 +313,37 @@ class Runner:
         # per layer: FP16 / H2O append and attention in one launch (H2O: + score update); KVQuant
         # quantize (which also stores the new length) + decode; RocketKV append, page choice and
         # attention in one launch
-        per = {"fp16": 1, "kvquant": 2, "h2o": 2, "rocket": 1}[self.method]
+        per = {"fp16": 1 if self.step_fused else 2, "kvquant": 2, "h2o": 2 if self.step_fused else 3,
+               "rocket": 1 if self.rocket_fused else 3}[self.method]
         return per * self.w.L
 
     def decode_bytes(self):
-        """Algorithmic bytes one decode launch reads for one layer now."""
+        """Algorithmic bytes one decode launch reads for one layer now (the per-unit byte models of
+        the compressed KV cache), the attended tokens, and bytes of implementation overhead the
+        launch also moves (reported apart, not in the roofline)."""
         w = self.w
         cache, _ = self.layers[0]
         units = w.B * w.Hkv
         T = int(cache.t["T_len"][0])
         if self.method == "fp16":
-            return units * T * w.D * 2 * 2, T
+            return units * T * w.D * 2 * 2, T, 0
         if self.method == "kvquant":
             nv = self.mkv.n_value_outliers(w.D, w.outlier_frac)
             per_tok = 2 * (w.D * w.bits // 8) + 8 + 4 * nv + 4
             n_kout = int(cache.t["k_out_off"][:, :, T].sum())
-            return units * T * per_tok + 4 * n_kout, T
+            return units * T * per_tok + 4 * n_kout, T, 0
         if self.method == "h2o":
-            slots = self.T_cap
-            # K and V rows, the slot's position (mask) and the G logits written for the update
-            return units * slots * (w.D * 2 * 2 + 4 + 4 * w.G), int(cache.t["pos"][0, 0].ge(0).sum())
+            held = int(cache.t["pos"][0, 0].ge(0).sum())
+            # K and V rows of the held slots; the slot's position (mask) and the G logits written for
+            # the score update are overhead
+            return units * held * w.D * 2 * 2, held, units * self.T_cap * (4 + 4 * w.G)
         n = T
         ns = (n - 1) // 16
         tail = n - 16 * ns
-        # the attended pages' K and V rows, and every dim's min/max of every candidate page
-        return units * ((min(w.topk_pages, ns) * 16 + tail) * w.D * 2 * 2 + ns * w.D * 2 * 2), n
+        # the attended pages' K and V rows, and the chosen dims' min/max of every candidate page
+        alg = units * ((min(w.topk_pages, ns) * 16 + tail) * w.D * 2 * 2 + ns * w.topq_dims * 2 * 2)
+        # the bounds of the other dims, which the fused step reads before the dims are chosen
+        return alg, n, units * ns * (w.D - w.topq_dims) * 2 * 2
 
 
 def time_steps(runner, steps, warmup):
@@ -423,6 +489,35 @@ def peaks():
     return 6800.0, "fallback"
 
 
+def measure_config(name, w, dev, seed, method, steps, warmup, peak, no_graph=False, synthetic_h2o_cache=False):
+    """One configuration: device-timed 32-layer step (graph replays), the decode launch's duration and
+    algorithmic bytes, and the KV bytes; a row of the per-configuration table."""
+    import torch
+    rx = Runner(name, w, dev, seed, extra_steps=4 * (steps + warmup) + 8, method=method,
+                synthetic_h2o_cache=synthetic_h2o_cache)
+    if not no_graph:
+        rx.capture()
+    msx = time_steps(rx, steps, warmup)
+    bx, tx, ox = rx.decode_bytes()
+    dx = time_decode_launches(rx, 10)
+    rres, rpk = rx.mkv.mkv_cache_bytes(rx.cfg, w.T)
+    gbs = bx / (dx * 1e-3) / 1e9
+    row = {"tokens_per_s": w.B / (msx * 1e-3), "ms_per_step": msx, "batch": w.B, "context": w.T,
+           "decode_launch_ms": dx, "decode_alg_bytes": bx, "decode_overhead_bytes": ox, "attended_tokens": tx,
+           "decode_gbs": gbs, "frac_of_measured_peak": gbs / peak, "frac_of_8000": gbs / 8000.0,
+           "kv_bytes_resident": rres * w.L, "kv_bytes_peak": rpk * w.L, "setup_s": rx.setup_s,
+           "gpu_launches_per_step": rx.launches_per_step()}
+    if rx.method == "h2o" and synthetic_h2o_cache:
+        row["note"] = "decode cache filled directly with the budget's heavy + recent slots (no prefill scoring)"
+    if rx.method in ("fp16", "h2o") and not rx.step_fused:
+        row["note"] = "append and attention as two launches (too many splits for the one-launch step)"
+    if rx.method == "rocket" and not rx.rocket_fused:
+        row["note"] = "append, page choice and split-KV attention over the page list as three launches"
+    del rx
+    torch.cuda.empty_cache()
+    return row
+
+
 # --------------------------------------------------------------------------- CPU oracle arm
 
 def oracle_tokens_per_s(name: str, w, budget_s: float, seed: int = 0):
@@ -477,6 +572,22 @@ def oracle_tokens_per_s(name: str, w, budget_s: float, seed: int = 0):
     return w.B / step_s, sample
 
 
+def _oracle_worker(args):
+    name, wd, budget, seed = args
+    return oracle_tokens_per_s(name, synth.Workload(**wd), budget, seed)[0]
+
+
+def oracle_tokens_per_s_all_cores(name: str, w, budget_s: float, seed: int = 0):
+    """The same oracle timing on every host core at once: one single-threaded worker process per core
+    (spawned, so no CUDA state is inherited), each decoding its own units; tokens/s add up."""
+    import dataclasses
+    import multiprocessing as mp
+    n = os.cpu_count() or 1
+    with mp.get_context("spawn").Pool(n) as pool:
+        vals = pool.map(_oracle_worker, [(name, dataclasses.asdict(w), budget_s, seed + i) for i in range(n)])
+    return float(sum(vals)), n
+
+
 # --------------------------------------------------------------------------- main
 
 def main():
@@ -493,6 +604,10 @@ def main():
                     help="profiling only: fewer layers than the workload (the line is then not a bench number)")
     ap.add_argument("--per-config", default="fp16,kvquant3,kvquant2,h2o20,rocket1024",
                     help="other workloads measured after the headline one (comma list, '' for none)")
+    ap.add_argument("--sweep", type=int, default=1,
+                    help="1: also measure the ten configurations at contexts 4K/16K/64K/128K (batch 32/16/4/1)")
+    ap.add_argument("--sweep-steps", type=int, default=5, help="timed steps per sweep configuration")
+    ap.add_argument("--cpu-all-cores", type=int, default=1, help="1: also time the oracle on every host core")
     ap.add_argument("--profile", action="store_true",
                     help="profiling only: run warmup + steps and exit (for ncu), no JSON line")
     args = ap.parse_args()
@@ -522,7 +637,9 @@ def main():
                 "steps": steps, "warmup": args.warmup, "ms_per_step": 1e3 * w.B / value,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
                 "data": "synthetic", "config": config,
-                "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample},
+                "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample,
+                                 "extrapolated": True},
+                "extrapolated": True,
                 "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
         print(json.dumps(line))
         return
@@ -557,7 +674,7 @@ def main():
     if world > 1:
         torch.distributed.barrier()
 
-    alg_bytes, T_now = runner.decode_bytes()
+    alg_bytes, T_now, ovh_bytes = runner.decode_bytes()
     dec_ms = time_decode_launches(runner, 10)
     e2e_s, h2d, d2h = time_e2e(runner, max(1, min(args.steps, 5)), 1)
     peak, peak_kind = peaks()
@@ -575,7 +692,8 @@ def main():
                          "frac": achieved / peak, "traffic": captured_traffic(args.workload),
                          "kernel": "mkv_decode_attention (one fused split-KV decode kernel), one layer",
                          "peak_kind": peak_kind, "frac_of_8000": achieved / 8000.0,
-                         "alg_bytes_per_launch": alg_bytes, "context_at_measure": T_now,
+                         "alg_bytes_per_launch": alg_bytes, "overhead_bytes_per_launch": ovh_bytes,
+                         "context_at_measure": T_now,
                          "avg_launch_ms": dec_ms},
             "kv_bytes": {"resident": res * w.L, "peak": pk * w.L, "unit": "bytes, all layers"},
             "clocks": clk}
@@ -588,26 +706,31 @@ def main():
             if args.layers is not None:
                 import dataclasses
                 wx = dataclasses.replace(wx, L=args.layers)
-            rx = Runner(name, wx, dev, args.seed, extra_steps=4 * total + 8)
-            if not args.no_graph:
-                rx.capture()
-            msx = time_steps(rx, args.steps, args.warmup)
-            bx, tx = rx.decode_bytes()
-            dx = time_decode_launches(rx, 10)
-            rres, rpk = rx.mkv.mkv_cache_bytes(rx.cfg, wx.T)
-            line["per_config"][wx.name] = {
-                "tokens_per_s": wx.B / (msx * 1e-3), "ms_per_step": msx, "batch": wx.B, "context": wx.T,
-                "decode_launch_ms": dx, "decode_alg_bytes": bx, "attended_tokens": tx,
-                "decode_gbs": bx / (dx * 1e-3) / 1e9, "frac_of_measured_peak": bx / (dx * 1e-3) / 1e9 / peak,
-                "frac_of_8000": bx / (dx * 1e-3) / 1e9 / 8000.0,
-                "kv_bytes_resident": rres * wx.L, "kv_bytes_peak": rpk * wx.L,
-                "setup_s": rx.setup_s, "gpu_launches_per_step": rx.launches_per_step()}
-            del rx
-            torch.cuda.empty_cache()
+            line["per_config"][wx.name] = measure_config(name, wx, dev, args.seed, METHOD_OF[name], args.steps,
+                                                         args.warmup, peak, args.no_graph)
+    if world == 1 and args.sweep:
+        # the ten configurations at contexts 4K/16K/64K/128K with batch 32/16/4/1
+        line["sweep"] = {}
+        t_sw = time.perf_counter()
+        for (T, B) in synth.SWEEP_POINTS:
+            for (meth, level) in synth.SWEEP_CONFIGS:
+                wx = synth.sweep(meth, level, T, B)
+                if args.layers is not None:
+                    import dataclasses
+                    wx = dataclasses.replace(wx, L=args.layers)
+                line["sweep"][wx.name] = measure_config(wx.name, wx, dev, args.seed, meth, args.sweep_steps, 3,
+                                                        peak, args.no_graph, synthetic_h2o_cache=True)
+        line["sweep_wall_s"] = time.perf_counter() - t_sw
     if rank == 0:
         if world == 1:
             v, sample = oracle_tokens_per_s(args.workload, w, args.cpu_budget, seed=args.seed)
-            line["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample}
+            line["cpu_baseline"] = {"value": v, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample,
+                                    "extrapolated": True}
+            if args.cpu_all_cores:
+                va, n = oracle_tokens_per_s_all_cores(args.workload, w, args.cpu_budget, seed=args.seed)
+                line["cpu_baseline_all_cores"] = {
+                    "value": va, "unit": "tokens/s", "cores": n, "kind": "oracle", "extrapolated": True,
+                    "sample": f"{n} single-threaded worker processes (nproc = {n}), each as the one-core sample"}
         print(json.dumps(line))
     if world > 1:
         torch.distributed.destroy_process_group()

@@ -208,3 +208,36 @@ def device_layer_inputs(w: Workload, seed: int, layer: int, device="cuda", n_tok
     if qp is not None:
         out["q_prompt"] = qp.half()
     return out
+
+
+# ----------------------------------------------------------------------------
+# the configuration sweep: every method at four (context, batch) points
+# ----------------------------------------------------------------------------
+
+SWEEP_POINTS = ((4096, 32), (16384, 16), (65536, 4), (131072, 1))
+
+
+def sweep(method: str, level: int, T: int, B: int) -> Workload:
+    """One configuration of the sweep at context T and batch B (32/8/128 GQA, 32 layers).
+
+    method "fp16" (level ignored), "kvquant" (level = bits, NUQ, per-channel key scales),
+    "h2o" (level = budget percent, split heavy/recent), "rocket" (level = token budget; keep
+    min(T, 4 * budget) after prefill, budget / 16 pages attended over 32 of 128 dims)."""
+    common = dict(B=B, L=32, Hq=32, Hkv=8, D=128, T=T, steps=64)
+    if method == "fp16":
+        return Workload(name=f"fp16_b{B}_t{T}", **common)
+    if method == "kvquant":
+        return Workload(name=f"kvquant_nuq{level}_b{B}_t{T}", bits=level, quant_mode="nuq", outlier_frac=0.01,
+                        key_scale_loguniform=(0.1, 10.0), **common)
+    if method == "h2o":
+        half = int(math.floor(level / 200.0 * T))
+        return Workload(name=f"h2o{level}_b{B}_t{T}", h2o_heavy=half, h2o_recent=half, heavy_frac=0.05,
+                        heavy_boost=20.0, **common)
+    if method == "rocket":
+        return Workload(name=f"rocket{level}_b{B}_t{T}", snap_window=32, snap_pool=7, snap_keep=min(T, 4 * level),
+                        page=16, topk_pages=level // 16, topq_dims=32, heavy_frac=0.05, heavy_boost=20.0, **common)
+    raise ValueError(method)
+
+
+SWEEP_CONFIGS = (("fp16", 0), ("kvquant", 4), ("kvquant", 3), ("kvquant", 2), ("h2o", 10), ("h2o", 20),
+                 ("h2o", 40), ("rocket", 1024), ("rocket", 2048), ("rocket", 4096))
