@@ -208,9 +208,10 @@ class Runner:
         self.step_fused = True
         # RocketKV: the fused one-launch step unless this shape is too large for it (then append,
         # page choice and sparse attention as three calls)
-        # (the fused step ranks and attends within one cluster per unit, which suits the 64 pages of
-        # the 1024-token budget; larger page budgets use the split-KV decode over the page list)
-        self.rocket_fused = self.method == "rocket" and w.topk_pages <= 64
+        # The fused step ranks and attends within one cluster per unit, which suits the 64 pages of
+        # the 1024-token budget; with more pages and many units the split-KV decode over the page
+        # list (three launches) can be faster.  Above 64 pages both are timed and the faster kept.
+        self.rocket_fused = self.method == "rocket"
         if self.rocket_fused:
             try:
                 mkv.mkv_rocket_decode(self.cfg, self.q[0].data_ptr(), self.layers[0][0].c, 0, self.out[0].data_ptr())
@@ -219,6 +220,11 @@ class Runner:
                 if e.status != mkv.MKV_ERR_UNSUPPORTED:
                     raise
                 self.rocket_fused = False
+            if self.rocket_fused and w.topk_pages > 64:
+                t_fused = time_decode_launches(self, 3)
+                self.rocket_fused = False
+                t_split = time_decode_launches(self, 3)
+                self.rocket_fused = t_fused <= t_split
 
     def append(self, l, kn=None, vn=None):
         mkv = self.mkv

@@ -6,8 +6,8 @@
 //     scores its 1/kCl share of the candidate pages (the full pages before the newest token's
 //     page): score_p = sum_t (kmax_t,p P_t + kmin_t,p N_t) over the chosen dims t, where
 //     P_t / N_t are the group's positive / negative query parts (max(q kmin, q kmax) is q kmax
-//     for q >= 0, q kmin otherwise, since kmin <= kmax).  The bounds of every dim of its
-//     pages are prefetched while the dims are being chosen;
+//     for q >= 0, q kmin otherwise, since kmin <= kmax).  Only the chosen dims' bounds are
+//     read: they are copied once the dims are known, while the newest page is being staged;
 //  2. every score is stored into every CTA of the cluster (distributed shared memory), then a
 //     cluster barrier;
 //  3. each CTA ranks its own pages against all scores (score desc, page asc), stores their
@@ -151,23 +151,6 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
   const int n_old = (int)min((int64_t)(a.T_len[b] & 0xffffff), a.T_cap);
   const bool room = append && (int64_t)n_old + 1 <= a.T_cap;
   const int n = room ? n_old + 1 : n_old;              // the step's token included
-  // ---- 1. prefetch every dim's bounds of this CTA's pages (16-byte copies from the row start
-  // rounded down to 16 bytes, the last one cut at the end of the pages)
-  if (npf > 0) {
-    const int np = npf;
-    const int nch = (7 + np + 7) / 8;                   // copies per row (covers the offset)
-    for (int e = tid; e < 2 * D * nch; e += kRfThreads) {
-      const int which = e / (D * nch), rem = e % (D * nch);
-      const int dim = rem / nch, ch = rem % nch;
-      const int64_t start = (bh * D + dim) * a.npc + p0;
-      const int64_t h0 = (start & ~7ll) + ch * 8;
-      const int64_t end = start + np;
-      if (h0 < end) {
-        const int bytes = (int)min((int64_t)16, (end - h0) * 2);
-        cp_async16((which ? bmx : bmn) + dim * a.rs + ch * 8, (which ? a.kmax : a.kmin) + h0, bytes);
-      }
-    }
-  }
   // the newest token's page, always attended, is staged now by the warp that attends to it
   const int ns = n > 0 ? (n - 1) / kPage : 0;          // candidate (full) pages; page ns is the newest
   const bool tail_warp = rank == kCl - 1 && warp == kRfWarps - 1 && n > 0;
@@ -230,6 +213,23 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
     if (i < D && half == 0 && rk < a.rd) dims[rk] = i;
   }
   __syncthreads();
+  // ---- 1. the chosen dims' bounds of this CTA's pages, row t for the t-th dim (16-byte copies from
+  // the row start rounded down to 16 bytes, the last one cut at the end of the pages)
+  if (npf > 0) {
+    const int nch = (7 + npf + 7) / 8;                 // copies per row (covers the offset)
+    for (int e = tid; e < 2 * a.rd * nch; e += kRfThreads) {
+      const int which = e / (a.rd * nch), rem = e % (a.rd * nch);
+      const int t = rem / nch, ch = rem % nch;
+      const int64_t start = (bh * D + dims[t]) * a.npc + p0;
+      const int64_t h0 = (start & ~7ll) + ch * 8;
+      const int64_t end = start + npf;
+      if (h0 < end) {
+        const int bytes = (int)min((int64_t)16, (end - h0) * 2);
+        cp_async16((which ? bmx : bmn) + t * a.rs + ch * 8, (which ? a.kmax : a.kmin) + h0, bytes);
+      }
+    }
+  }
+  cp_async_commit();
   if (tid < a.rd) {
     const int d = dims[tid];
     float P = 0.f, N = 0.f;
@@ -248,9 +248,8 @@ __global__ void __cluster_dims__(kCl, 1, 1) __launch_bounds__(kRfThreads, 2) roc
     const int pl = e % np, sl = e / np;
     float acc = 0.f;
     for (int t = sl; t < a.rd; t += kRfSlices) {
-      const int d = dims[t];
-      const int off = (int)(((bh * D + d) * a.npc + p0) & 7);
-      const int i = d * a.rs + off + pl;
+      const int off = (int)(((bh * D + dims[t]) * a.npc + p0) & 7);
+      const int i = t * a.rs + off + pl;
       acc += __half2float(bmx[i]) * pn[0][t] + __half2float(bmn[i]) * pn[1][t];
     }
     part[sl * sp + pl] = acc;
