@@ -26,7 +26,8 @@
  *    NULL is the legacy default stream).  Arguments are validated on the host
  *    before anything is launched: a bad argument returns an error code and
  *    launches nothing.  A launch failure returns MKV_ERR_CUDA.  A condition
- *    only the device can see (outlier storage full) sets a bit of the status
+ *    only the device can see (outlier storage full, a bounded wait that ran
+ *    out) sets a bit of the status
  *    word that mkv_get_status() reports.  No call aborts or throws.
  *  - mkv_last_error() returns a thread-local text for the last failure.
  *  - Shapes: B batch entries, Hq query heads, Hkv key/value heads,
@@ -59,7 +60,7 @@ typedef enum {
   MKV_ERR_CUDA = 3,         /* a CUDA call or launch failed                  */
   MKV_ERR_CAPACITY = 4,     /* a device-side store ran out of room           */
   MKV_ERR_WORKSPACE = 5,    /* ws is NULL or ws_bytes below the required size */
-  MKV_ERR_TIMEOUT = 6       /* reserved: no kernel of this library waits     */
+  MKV_ERR_TIMEOUT = 6       /* a bounded device-side wait ran out            */
 } mkv_status;
 
 typedef enum { MKV_FP16 = 0, MKV_KVQUANT = 1, MKV_H2O = 2, MKV_ROCKET = 3 } mkv_method;
@@ -68,6 +69,8 @@ typedef enum { MKV_QUANT_UNIFORM = 0, MKV_QUANT_NUQ = 1 } mkv_quant_mode;
 /* Status-word bits (mkv_get_status). */
 #define MKV_FLAG_K_OUTLIER_OVERFLOW 0x1u  /* a key-outlier CSR region is full */
 #define MKV_FLAG_CACHE_FULL 0x2u          /* an append found no free slot; dropped */
+#define MKV_FLAG_WAIT_TIMEOUT 0x4u        /* a prefill-scoring CTA gave up waiting on the
+                                             tensor core; that call's scores are invalid */
 
 /* One configuration (a row of Table 1, with its parameters).  Host POD. */
 typedef struct {
@@ -218,7 +221,8 @@ mkv_status mkv_select_config(const mkv_candidate* cands, int32_t n, double L_max
 mkv_status mkv_rope_table(int32_t D, float theta, int64_t T_max, float* table, void* stream);
 
 /* Synchronizes `stream`, then returns the status word in *flags (host) and
- * clears it.  MKV_ERR_CAPACITY if any bit was set. */
+ * clears it.  MKV_ERR_TIMEOUT if MKV_FLAG_WAIT_TIMEOUT was set, else
+ * MKV_ERR_CAPACITY if any bit was set. */
 mkv_status mkv_get_status(void* stream, uint32_t* flags);
 
 /* Thread-local description of the last error (never NULL). */
@@ -332,7 +336,9 @@ mkv_status mkv_quantize_kv(const mkv_config* cfg, const mkv_quant_params* qparam
  * causal softmax probability of key j; keeps the h2o_recent newest positions
  * and the h2o_heavy best others (acc desc, position asc), compacted in
  * ascending position into slots 0..; sets pos, acc, slot and T_len[b] = T.
- * Needs ws (mkv_workspace_size with T_cap >= T). */
+ * q_prompt and full_k must be 16-byte aligned (MKV_ERR_INVALID_ARG).
+ * Needs ws (mkv_workspace_size with T_cap >= T).  A scoring CTA whose bounded
+ * wait on the tensor core ran out sets MKV_FLAG_WAIT_TIMEOUT. */
 mkv_status mkv_h2o_prefill(const mkv_config* cfg, const void* q_prompt, const void* full_k,
                            const void* full_v, int64_t T, mkv_cache* cache, void* ws,
                            size_t ws_bytes, void* stream);
@@ -358,7 +364,9 @@ mkv_status mkv_h2o_update(const mkv_config* cfg, mkv_cache* cache, void* ws, siz
  * the snap_keep - W best (score desc, position asc) plus the window, gathers
  * them in ascending position into slots 0..keep-1 of `cache`, fills kmin/kmax
  * of every full page and sets T_len[b] = keep.  keep >= T copies everything.
- * kept_pos (optional, int32 [B][Hkv][keep]) receives the kept positions. */
+ * kept_pos (optional, int32 [B][Hkv][keep]) receives the kept positions.
+ * q_window and full_k must be 16-byte aligned (MKV_ERR_INVALID_ARG); a
+ * scoring wait that ran out sets MKV_FLAG_WAIT_TIMEOUT as for H2O. */
 mkv_status mkv_snap_compress(const mkv_config* cfg, const void* q_window, const void* full_k,
                              const void* full_v, int64_t T, mkv_cache* cache, int32_t* kept_pos,
                              void* ws, size_t ws_bytes, void* stream);

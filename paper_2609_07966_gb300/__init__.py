@@ -21,6 +21,7 @@ MKV_FP16, MKV_KVQUANT, MKV_H2O, MKV_ROCKET = range(4)
 MKV_QUANT_UNIFORM, MKV_QUANT_NUQ = range(2)
 MKV_FLAG_K_OUTLIER_OVERFLOW = 0x1
 MKV_FLAG_CACHE_FULL = 0x2
+MKV_FLAG_WAIT_TIMEOUT = 0x4
 
 _STATUS_NAMES = {0: "MKV_OK", 1: "MKV_ERR_INVALID_ARG", 2: "MKV_ERR_UNSUPPORTED", 3: "MKV_ERR_CUDA",
                  4: "MKV_ERR_CAPACITY", 5: "MKV_ERR_WORKSPACE", 6: "MKV_ERR_TIMEOUT"}
@@ -167,7 +168,7 @@ def mkv_get_status(stream=None) -> int:
     """Status-word bits (0 when clean).  Synchronizes the stream."""
     f = ctypes.c_uint32(0)
     st = lib().mkv_get_status(_stream(stream), ctypes.byref(f))
-    if st not in (MKV_OK, MKV_ERR_CAPACITY):
+    if st not in (MKV_OK, MKV_ERR_CAPACITY, MKV_ERR_TIMEOUT):
         raise MkvError(st, "mkv_get_status", mkv_last_error())
     return f.value
 

@@ -96,7 +96,7 @@ __global__ void __launch_bounds__(1024) h2o_update_kernel(const float* __restric
 cudaError_t launch_h2o_keep(const mkv_config& c, const void* full_k, const void* full_v, int64_t T,
                             const mkv_cache& cache, const PrefillWs& ws, cudaStream_t st) {
   const int units = c.B * c.Hkv;
-  int32_t* n_keep = reinterpret_cast<int32_t*>(ws.row_l);   // row stats are dead after scoring
+  int32_t* n_keep = reinterpret_cast<int32_t*>(ws.row_st);   // row stats are dead after scoring
   h2o_keep_kernel<<<units, kSelThreads, 0, st>>>(ws.score, T, c.h2o_heavy, c.h2o_recent, ws.keep, n_keep);
   cudaError_t e = cudaPeekAtLastError();
   if (e != cudaSuccess) return e;

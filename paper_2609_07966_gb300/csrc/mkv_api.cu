@@ -97,8 +97,7 @@ PrefillWs prefill_ws(const mkv_config& c, int64_t T, void* base) {
     return r;
   };
   PrefillWs w{};
-  w.row_m = static_cast<float*>(take((size_t)c.B * c.Hq * T * 4));
-  w.row_l = static_cast<float*>(take((size_t)c.B * c.Hq * T * 4));
+  w.row_st = static_cast<float2*>(take((size_t)c.B * c.Hq * (T + 128) * 8));
   w.score = static_cast<float*>(take((size_t)c.B * c.Hkv * T * 4));
   w.keep = static_cast<int32_t*>(take((size_t)c.B * c.Hkv * T * 4));
   w.bytes = off;
@@ -317,6 +316,11 @@ mkv_status mkv_get_status(void* stream, uint32_t* flags) {
   MKV_CUDA(take_status_kvquant(flags, as_stream(stream)));
   MKV_CUDA(take_status_rocket(flags, as_stream(stream)));
   MKV_CUDA(take_status_decode(flags, as_stream(stream)));
+  MKV_CUDA(take_status_prefill(flags, as_stream(stream)));
+  if (*flags & MKV_FLAG_WAIT_TIMEOUT) {
+    set_error("device status flags 0x%x (a bounded wait ran out)", *flags);
+    return MKV_ERR_TIMEOUT;
+  }
   if (*flags != 0) {
     set_error("device status flags 0x%x", *flags);
     return MKV_ERR_CAPACITY;
@@ -438,6 +442,8 @@ mkv_status mkv_h2o_prefill(const mkv_config* cfg, const void* q_prompt, const vo
   MKV_REQUIRE(cfg->method == MKV_H2O, MKV_ERR_INVALID_ARG, "h2o_prefill is for H2O");
   MKV_TRY(check_cache(cfg, cache));
   MKV_REQUIRE(q_prompt && full_k && full_v && T >= 1, MKV_ERR_INVALID_ARG, "prompt tensors NULL or T < 1");
+  MKV_REQUIRE((((uintptr_t)q_prompt | (uintptr_t)full_k) & 15) == 0, MKV_ERR_INVALID_ARG,
+              "q_prompt and full_k must be 16-byte aligned (tensor-core scoring reads them by TMA)");
   const PrefillWs need = prefill_ws(*cfg, T, nullptr);
   MKV_REQUIRE(ws != nullptr && ws_bytes >= need.bytes, MKV_ERR_WORKSPACE,
               "workspace %zu bytes < %zu needed", ws_bytes, need.bytes);
@@ -467,6 +473,8 @@ mkv_status mkv_snap_compress(const mkv_config* cfg, const void* q_window, const 
   MKV_TRY(check_cache(cfg, cache));
   MKV_REQUIRE(q_window && full_k && full_v && T >= cfg->snap_window, MKV_ERR_INVALID_ARG,
               "prompt tensors NULL or T < snap_window");
+  MKV_REQUIRE((((uintptr_t)q_window | (uintptr_t)full_k) & 15) == 0, MKV_ERR_INVALID_ARG,
+              "q_window and full_k must be 16-byte aligned (tensor-core scoring reads them by TMA)");
   MKV_REQUIRE(cache->T_cap >= std::min<int64_t>(T, cfg->snap_keep), MKV_ERR_INVALID_ARG,
               "cache T_cap below the kept tokens");
   const PrefillWs need = prefill_ws(*cfg, T, nullptr);

@@ -59,8 +59,7 @@ DecodeWs decode_ws(const mkv_config& c, int64_t T_cap, void* base);
 
 // Prefill workspace (H2O prefill, SnapKV compression): scores and selection.
 struct PrefillWs {
-  float* row_m;    // [B][Hq][T]  per-query-row max (log2 domain)
-  float* row_l;    // [B][Hq][T]  per-query-row sum
+  float2* row_st;  // [B][Hq][T + 128] per-query-row (max, sum) partials, then merged (-max, 1 / sum)
   float* score;    // [B][Hkv][T] accumulated column sums
   int32_t* keep;   // [B][Hkv][T] kept positions (ascending)
   size_t bytes;
@@ -144,5 +143,6 @@ cudaError_t take_status_kvquant(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_append(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_rocket(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_decode(uint32_t* flags, cudaStream_t st);
+cudaError_t take_status_prefill(uint32_t* flags, cudaStream_t st);
 
 }  // namespace mkv

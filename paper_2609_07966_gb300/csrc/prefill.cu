@@ -4,304 +4,459 @@
 // -- H2O: every prompt row (p_i = i), the accumulated attention a token
 //    receives from later tokens;
 // -- SnapKV: the W rows of the observation window (p_i = T - W + i).
-// Two tensor-core passes (m16n8k16, fp16 in, fp32 accumulate):
-//   pass 1: per query row, running max m_i and sum l_i of 2^(s - m_i) over
-//           its causal keys (key range split across CTAs, merged in pass 2);
-//   pass 2: per key block, sum of 2^(s - m_i) / l_i over the query rows, the
-//           product computed transposed (keys as the M dimension) so each key's
-//           column sum stays in the registers of the lanes that own it.
+//
+// Two passes on the 5th-generation tensor cores (tcgen05.mma kind::f16: fp16 operands, fp32
+// accumulator in tensor memory), each a stream of 128 x 128 x D tile products with a softmax
+// epilogue:
+//   pass 1 (rows): a CTA holds 128 query rows (the group's G heads, 128 / G rows each) and streams
+//           128-key tiles; it keeps per row the running max m and sum l of 2^(s - m) over the
+//           causal keys.  When the rows are few (an observation window) the key range is split
+//           across CTAs; a small kernel merges the splits into (-m, 1 / l) per row, laid out in the
+//           order of pass 2's query tiles;
+//   pass 2 (columns): a CTA holds 128 keys and streams the 128-row query tiles that can see
+//           them, summing 2^(s - m_i) / l_i over the rows with p_i >= j for each key j.
+// The held operand is the MMA's A (M = 128 lanes of the accumulator), a streamed tile its B
+// (N = 128 columns).  Each CTA is warp-specialised:
+//   warp 0 (one thread) loads operand tiles by TMA (tensor maps with the 128-byte swizzle, the
+//           K-major layout the MMA reads) into a ring of kS stages, and in pass 2 each tile's 128
+//           row statistics by a bulk copy beside it;
+//   warp 1 (one thread) issues the D / 16 MMAs of a tile into one of two tensor-memory
+//           accumulator buffers, then commits to the stage's and the buffer's mbarriers;
+//   warps 2..17 read a finished accumulator (warp w: lanes 32 (w % 4) .. + 31, the lane quarter
+//           it may access, and column quarter (w - 2) / 4) and release the buffer.
+// Loads, products and epilogues of different tiles overlap; nothing in the tile loop waits on a
+// CTA-wide barrier.  Every wait is bounded: on a timeout the role raises MKV_FLAG_WAIT_TIMEOUT and
+// sets a flag that ends the other roles' waits; the CTA then waits (bounded) for the copies and
+// products it already issued and still frees its tensor memory.
+#include <cuda.h>   // CUtensorMap and its enums; the encoder is fetched from the driver at run time
 #include <math.h>
 
 #include <algorithm>
 
 #include "mkv_common.cuh"
 #include "mkv_internal.h"
+#include "mkv_tc.cuh"
 
 namespace mkv {
 
+__device__ uint32_t g_status_prefill;   // MKV_FLAG_* bits raised by the scoring passes
+
+cudaError_t take_status_prefill(uint32_t* flags, cudaStream_t st) {
+  uint32_t v = 0, zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbolAsync(&v, g_status_prefill, sizeof(v), 0, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemcpyToSymbolAsync(g_status_prefill, &zero, sizeof(zero), 0, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  *flags |= v;
+  return e;
+}
+
 namespace {
 
-constexpr int kT = 128;   // threads: 4 warps
+constexpr int kTM = 128;                 // rows of the held operand (the MMA's M)
+constexpr int kTN = 128;                 // rows of a streamed tile (the MMA's N)
+constexpr int kEpiWarps = 16;            // four lane quarters x four column quarters
+constexpr int kThr = (2 + kEpiWarps) * 32;
+constexpr int kCQ = kTN / 4;             // accumulator columns an epilogue thread reads per tile
+constexpr int kS = 4;                    // operand stages
+constexpr int kStatBytes = kTN * 8;      // one query tile's (-m, 1 / l)
+constexpr uint32_t kWaitLimit = 1u << 22;
 
 struct ScoreArgs {
-  const __half* q;      // [B][Hq][R][D]
-  const __half* k;      // [B][Hkv][T][D]
   int64_t R, T, pos0;   // query rows, keys, position of query row 0
-  int Hq, Hkv, G, rpb;  // rpb = rows per block (64 / G)
+  int Hq, Hkv, G, rpb;  // rpb = rows per head in a 128-row block (128 / G, a power of two)
+  int rowblocks;        // ceil(R / rpb)
   int n_ksplit, tiles_per_split;
   float scale_log2;
-  float* row_m;         // [B][Hq][R][n_ksplit]
-  float* row_l;
-  float* score;         // [B][Hkv][T]
+  float2* row_st;       // [B Hkv][rowblocks][n_ksplit][128]: pass 1's (m, l); merged (-m, 1 / l) at split 0
+  float* score;         // [B Hkv][T]
 };
 
-// query row q in [0, 64) of row block rb -> (head in group, row index)
-__device__ __forceinline__ void qrow_map(const ScoreArgs& a, int rb, int q, int& gh, int64_t& i) {
-  gh = q / a.rpb;
-  i = (int64_t)rb * a.rpb + q % a.rpb;
+template <int D>
+struct Layout {
+  static constexpr int ATOM = kTM * 128;                  // 128 rows x 64 fp16 (one swizzle atom column)
+  static constexpr int TILE = (D / 64) * ATOM;            // one 128-row operand tile
+  static constexpr int A_OFF = 0;
+  static constexpr int B_OFF = TILE;                      // [kS] streamed tiles
+  static constexpr int ST_OFF = B_OFF + kS * TILE;        // [kS] pass 2: the tile's row statistics
+  static constexpr int MRG_OFF = ST_OFF + kS * kStatBytes;   // [4][128] the column quarters' partials
+  static constexpr int CTL_OFF = MRG_OFF + 4 * kTM * 8;
+  static constexpr int BYTES = CTL_OFF + 256;
+  static constexpr int ALLOC = BYTES + 1024;              // slack to align the base to 1024 B
+};
+
+struct Ctl {
+  uint64_t full[kS];     // stage s loaded (TMA transaction bytes)
+  uint64_t empty[kS];    // stage s's operand read by the tensor core
+  uint64_t sempty[kS];   // stage s's row statistics read by every epilogue warp (pass 2)
+  uint64_t tfull[2];     // accumulator buffer b holds a finished product
+  uint64_t tempty[2];    // accumulator buffer b read by every epilogue warp
+  uint64_t abar;         // the held operand loaded
+  uint32_t tslot;        // tensor-memory base address
+  int fail;              // a wait ran out: every role stops
+  int issued;            // tiles whose loads were issued
+  int mma_issued;        // tiles whose products were issued
+};
+static_assert(sizeof(Ctl) <= 256, "control block");
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return p + ((1024u - (smem_addr(p) & 1023u)) & 1023u);
+}
+
+// Bounded wait of one role: false when it ran out (the flag is then raised) or another role did.
+__device__ __forceinline__ bool role_wait(uint64_t* bar, uint32_t parity, volatile int* fail) {
+  for (uint32_t it = 0; it < kWaitLimit; ++it) {
+    if (tc_mbar_try(bar, parity)) return true;
+    if (*fail) return false;
+  }
+  *fail = 1;
+  atomicOr(&g_status_prefill, MKV_FLAG_WAIT_TIMEOUT);
+  return false;
+}
+
+// D[tmem] = A (128 rows) x B (128 rows)^T over K = D: D / 16 MMAs, issued by one thread
+template <int D>
+__device__ __forceinline__ void issue_tile(uint32_t d_tmem, uint32_t a_s, uint32_t b_s) {
+  constexpr uint32_t kId = tc_idesc_f16(kTM, kTN);
+#pragma unroll
+  for (int kk = 0; kk < D / 16; ++kk) {
+    const uint32_t off = (uint32_t)((kk >> 2) * Layout<D>::ATOM + (kk & 3) * 32);
+    tc_mma(d_tmem, tc_desc_sw128(a_s + off), tc_desc_sw128(b_s + off), kId, kk > 0 ? 1u : 0u);
+  }
+}
+
+// Barriers and tensor memory of a CTA; returns the tensor-memory base (2 x 128 columns).
+__device__ __forceinline__ uint32_t cta_setup(Ctl* ctl) {
+  if ((threadIdx.x >> 5) == 0) tc_alloc(&ctl->tslot, 2 * kTN);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kS; ++s) {
+      tc_mbar_init(&ctl->full[s], 1);
+      tc_mbar_init(&ctl->empty[s], 1);
+      tc_mbar_init(&ctl->sempty[s], kEpiWarps);
+    }
+    for (int b = 0; b < 2; ++b) {
+      tc_mbar_init(&ctl->tfull[b], 1);
+      tc_mbar_init(&ctl->tempty[b], kEpiWarps);
+    }
+    tc_mbar_init(&ctl->abar, 1);
+    tc_fence_mbar_init();
+    ctl->fail = 0;
+    ctl->issued = 0;
+    ctl->mma_issued = 0;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  return ctl->tslot;
+}
+
+// After every role has returned: on a failure, wait (bounded) for the copies and products already
+// issued; then free the tensor memory.
+__device__ __forceinline__ void cta_teardown(Ctl* ctl, uint32_t tbase) {
+  tc_fence_before();
+  __syncthreads();
+  if (threadIdx.x == 0 && ctl->fail) {
+    for (int t = std::max(0, ctl->issued - kS); t < ctl->issued; ++t)
+      tc_mbar_wait(&ctl->full[t % kS], (uint32_t)((t / kS) & 1), kWaitLimit);
+    if (ctl->mma_issued > 0) {
+      const int t = ctl->mma_issued - 1;
+      tc_mbar_wait(&ctl->tfull[t & 1], (uint32_t)((t >> 1) & 1), kWaitLimit);
+    }
+  }
+  __syncthreads();
+  tc_fence_after();
+  if ((threadIdx.x >> 5) == 0) tc_dealloc(tbase, 2 * kTN);
+}
+
+// The three roles over `ntiles` streamed tiles.  issue_a(bar) loads the held operand;
+// issue_b(t, s, bar) loads tile t into stage s; epi(t, col, s) reads tile t's accumulator (columns
+// from tensor-memory address col, lane 0) and, with kStats, the statistics of stage s.
+template <int D, bool kStats, typename IssueA, typename IssueB, typename Epi>
+__device__ __forceinline__ void run_roles(uint8_t* sm, Ctl* ctl, uint32_t tbase, int ntiles, IssueA issue_a,
+                                          IssueB issue_b, Epi epi) {
+  using L = Layout<D>;
+  volatile int* fail = &ctl->fail;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (ntiles <= 0) return;
+  if (warp == 0) {
+    if (lane == 0) {                      // producer
+      issue_a(&ctl->abar);
+      for (int t = 0; t < ntiles; ++t) {
+        const int s = t % kS, n = t / kS;
+        if (n > 0) {
+          if (!role_wait(&ctl->empty[s], (uint32_t)((n - 1) & 1), fail)) break;
+          if (kStats && !role_wait(&ctl->sempty[s], (uint32_t)((n - 1) & 1), fail)) break;
+        }
+        issue_b(t, s, &ctl->full[s]);
+        ctl->issued = t + 1;
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {                      // MMA issuer
+      const uint32_t a_s = smem_addr(sm + L::A_OFF);
+      if (role_wait(&ctl->abar, 0, fail)) {
+        for (int t = 0; t < ntiles; ++t) {
+          const int s = t % kS, bf = t & 1, u = t >> 1;
+          if (!role_wait(&ctl->full[s], (uint32_t)((t / kS) & 1), fail)) break;
+          if (u > 0 && !role_wait(&ctl->tempty[bf], (uint32_t)((u - 1) & 1), fail)) break;
+          tc_fence_after();
+          issue_tile<D>(tbase + (uint32_t)(bf * kTN), a_s, smem_addr(sm + L::B_OFF + s * L::TILE));
+          tc_commit(&ctl->empty[s]);
+          tc_commit(&ctl->tfull[bf]);
+          ctl->mma_issued = t + 1;
+        }
+      }
+    }
+  } else {                                // epilogue warps
+    for (int t = 0; t < ntiles; ++t) {
+      const int s = t % kS, bf = t & 1;
+      bool ok = role_wait(&ctl->tfull[bf], (uint32_t)((t >> 1) & 1), fail);
+      // the statistics came with the stage's operand: their copy completed that phase of full[s]
+      if (kStats) ok = ok && role_wait(&ctl->full[s], (uint32_t)((t / kS) & 1), fail);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      epi(t, tbase + (uint32_t)(bf * kTN), s);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        tc_mbar_arrive(&ctl->tempty[bf]);
+        if (kStats) tc_mbar_arrive(&ctl->sempty[s]);
+      }
+    }
+  }
 }
 
 // ---------------------------------------------------------------- pass 1
 template <int D>
-__global__ void __launch_bounds__(kT) rowstats_kernel(const ScoreArgs a) {
-  constexpr int ROWB = D * 2, NC = D / 8, KC = D / 16, TILE = 64 * ROWB;
-  extern __shared__ __align__(128) uint8_t smem[];   // [2][64 keys][D] swizzled
-  const int ks = blockIdx.x, rb = blockIdx.y;
-  const int64_t bh = blockIdx.z;
-  const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, r = lane & 3;
+__global__ void __launch_bounds__(kThr, 1)
+    rowstats_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                       const ScoreArgs a) {
+  using L = Layout<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = align1024(smem_raw);
+  Ctl* ctl = reinterpret_cast<Ctl*>(sm + L::CTL_OFF);
+  const int ks = blockIdx.x;
+  const int rb = a.rowblocks - 1 - (int)blockIdx.y;      // the row blocks with the most keys first
+  const int bh = (int)blockIdx.z;
+  const int b = bh / a.Hkv, kvh = bh % a.Hkv;
+  const int warp = threadIdx.x >> 5;
+  const int lq = warp & 3, cq = (warp - 2) >> 2;         // (epilogue warps) lane and column quarter
+  const int lr = lq * 32 + (threadIdx.x & 31);           // accumulator lane = query row of the block
 
-  // the CTA's rows: positions of its last valid row bound the causal key range
-  const int64_t row_lo = (int64_t)rb * a.rpb;
-  const int64_t row_hi = std::min<int64_t>(row_lo + a.rpb, a.R);   // exclusive
-  const int64_t key_end_causal = a.pos0 + row_hi;                   // keys < this may be attended
-  const int64_t k_begin = (int64_t)ks * a.tiles_per_split * 64;
-  const int64_t k_end = std::min<int64_t>(std::min<int64_t>(k_begin + (int64_t)a.tiles_per_split * 64, a.T),
-                                          key_end_causal);
-  const int ntiles = k_end > k_begin ? (int)ceil_div_dev(k_end - k_begin, 64) : 0;
+  // the block's last valid row bounds its causal key range
+  const int64_t row_hi = std::min<int64_t>((int64_t)rb * a.rpb + a.rpb, a.R);   // exclusive
+  const int64_t k_begin = (int64_t)ks * a.tiles_per_split * kTN;
+  const int64_t k_end = std::min<int64_t>(std::min<int64_t>(k_begin + (int64_t)a.tiles_per_split * kTN, a.T),
+                                          a.pos0 + row_hi);
+  const int ntiles = k_end > k_begin ? (int)ceil_div_dev(k_end - k_begin, kTN) : 0;
+  const int64_t irow = (int64_t)rb * a.rpb + (lr & (a.rpb - 1));
+  const int64_t lim = irow < a.R ? std::min<int64_t>(k_end - 1, a.pos0 + irow) : -1;   // last key it sees
+  const int plane0 = b * a.Hq + kvh * a.G;               // the group's first query head
 
-  // A fragments: query rows 16*warp + g and + 8
-  uint32_t qa[KC][4];
-  int64_t pos_row[2];
-  bool valid_row[2];
-  int gh_row[2];
-  int64_t i_row[2];
+  const uint32_t tbase = cta_setup(ctl);
+  float m_run = -INFINITY, l_run = 0.f;
+  run_roles<D, false>(
+      sm, ctl, tbase, ntiles,
+      [&](uint64_t* bar) {                // head g's rows of the block are tile rows g rpb ..
+        tc_mbar_expect_tx(bar, L::TILE);
+        for (int g = 0; g < a.G; ++g)
+          for (int at = 0; at < D / 64; ++at)
+            tma_load_3d(sm + L::A_OFF + at * L::ATOM + g * a.rpb * 128, &qmap, at * 64, rb * a.rpb, plane0 + g, bar);
+      },
+      [&](int t, int s, uint64_t* bar) {
+        tc_mbar_expect_tx(bar, L::TILE);
+        for (int at = 0; at < D / 64; ++at)
+          tma_load_3d(sm + L::B_OFF + s * L::TILE + at * L::ATOM, &kmap, at * 64, (int)(k_begin + (int64_t)t * kTN),
+                      bh, bar);
+      },
+      [&](int t, uint32_t col, int) {
+        const int64_t jc = k_begin + (int64_t)t * kTN + cq * kCQ;
+        float v[kCQ];
+        tc_ld32(col + ((uint32_t)(lq * 32) << 16) + (uint32_t)(cq * kCQ), v);
+        float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};   // max of the raw products
+        if (jc + kCQ - 1 <= lim) {
 #pragma unroll
-  for (int hh = 0; hh < 2; ++hh) {
-    const int q = 16 * warp + g + 8 * hh;
-    qrow_map(a, rb, q, gh_row[hh], i_row[hh]);
-    valid_row[hh] = gh_row[hh] < a.G && i_row[hh] < a.R;
-    pos_row[hh] = a.pos0 + i_row[hh];
-  }
+          for (int e = 0; e < kCQ; ++e) mx[e & 3] = fmaxf(mx[e & 3], v[e]);
+        } else {
 #pragma unroll
-  for (int kc = 0; kc < KC; ++kc) {
-#pragma unroll
-    for (int hh = 0; hh < 2; ++hh) {
-      uint32_t lo = 0, hi = 0;
-      if (valid_row[hh]) {
-        const __half* qr = a.q + (((int64_t)b * a.Hq + (int64_t)kvh * a.G + gh_row[hh]) * a.R + i_row[hh]) * D;
-        lo = *reinterpret_cast<const uint32_t*>(qr + kc * 16 + 2 * r);
-        hi = *reinterpret_cast<const uint32_t*>(qr + kc * 16 + 2 * r + 8);
-      }
-      qa[kc][hh] = lo;        // a0 (row g) / a1 (row g+8)
-      qa[kc][2 + hh] = hi;    // a2 / a3
-    }
-  }
-
-  const __half* kbase = a.k + bh * a.T * D;
-  auto load_tile = [&](int t, int stage) {
-    uint8_t* Ks = smem + stage * TILE;
-    const int col = tid % NC;
-    for (int rr = tid / NC; rr < 64; rr += kT / NC) {
-      const int64_t j = k_begin + (int64_t)t * 64 + rr;
-      const bool ok = j < k_end;
-      cp_async16(Ks + rr * ROWB + ((col ^ (rr & 7)) << 4), kbase + (ok ? j : 0) * D + col * 8, ok ? 16 : 0);
-    }
-  };
-
-  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-  if (ntiles > 0) load_tile(0, 0);
-  cp_async_commit();
-  for (int t = 0; t < ntiles; ++t) {
-    cp_async_wait<0>();
-    __syncthreads();
-    if (t + 1 < ntiles) load_tile(t + 1, (t + 1) & 1);
-    cp_async_commit();
-    const uint8_t* Ks = smem + (t & 1) * TILE;
-    float sc[8][4];
-#pragma unroll
-    for (int n = 0; n < 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
-    const int mi = lane >> 3, row = lane & 7;
-#pragma unroll
-    for (int kc = 0; kc < KC; ++kc) {
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {     // pairs of n-tiles (16 keys)
-        uint32_t bk[4];
-        const int tok = np * 16 + (mi >> 1) * 8 + row;
-        const int ch = kc * 2 + (mi & 1);
-        ldsm_x4(bk, Ks + tok * ROWB + ((ch ^ (tok & 7)) << 4));
-        mma16816(sc[2 * np], qa[kc][0], qa[kc][1], qa[kc][2], qa[kc][3], bk[0], bk[1]);
-        mma16816(sc[2 * np + 1], qa[kc][0], qa[kc][1], qa[kc][2], qa[kc][3], bk[2], bk[3]);
-      }
-    }
-#pragma unroll
-    for (int hh = 0; hh < 2; ++hh) {
-      float mx = -INFINITY;
-      float x[16];
-#pragma unroll
-      for (int n = 0; n < 8; ++n) {
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int64_t j = k_begin + (int64_t)t * 64 + n * 8 + 2 * r + e;
-          const bool ok = valid_row[hh] && j < k_end && j <= pos_row[hh];
-          const float v = ok ? sc[n][2 * hh + e] * a.scale_log2 : -INFINITY;
-          x[n * 2 + e] = v;
-          mx = fmaxf(mx, v);
+          for (int e = 0; e < kCQ; ++e) {
+            v[e] = jc + e <= lim ? v[e] : -INFINITY;
+            mx[e & 3] = fmaxf(mx[e & 3], v[e]);
+          }
         }
-      }
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      const float m_new = fmaxf(m_run[hh], mx);
-      if (m_new != -INFINITY) {
-        float s = 0.f;
+        // the scale is positive: the max of the scaled products is the scaled max
+        const float m_new = fmaxf(m_run, fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * a.scale_log2);
+        if (m_new != -INFINITY) {
+          float sp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int e = 0; e < 16; ++e) s += exp2f(x[e] - m_new);
-        l_run[hh] = l_run[hh] * exp2f(m_run[hh] - m_new) + s;
-        m_run[hh] = m_new;
+          for (int e = 0; e < kCQ; ++e) sp[e & 3] += ex2_approx(fmaf(v[e], a.scale_log2, -m_new));
+          l_run = l_run * ex2_approx(m_run - m_new) + ((sp[0] + sp[1]) + (sp[2] + sp[3]));
+          m_run = m_new;
+        }
+      });
+  // the four column quarters of each row merged into this split's (m, l)
+  float2* mrg = reinterpret_cast<float2*>(sm + L::MRG_OFF);
+  if (warp >= 2) mrg[cq * kTM + lr] = make_float2(m_run, l_run);
+  __syncthreads();
+  if (warp >= 2 && cq == 0) {
+    float M = -INFINITY;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) M = fmaxf(M, mrg[q * kTM + lr].x);
+    float l = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 o = mrg[q * kTM + lr];
+        l += o.y * ex2_approx(o.x - M);
       }
     }
+    a.row_st[(((int64_t)bh * a.rowblocks + rb) * a.n_ksplit + ks) * kTM + lr] = make_float2(M, l);
   }
-  cp_async_wait<0>();
-#pragma unroll
-  for (int hh = 0; hh < 2; ++hh) {
-    float l = l_run[hh];
-    l += __shfl_xor_sync(0xffffffffu, l, 1);
-    l += __shfl_xor_sync(0xffffffffu, l, 2);
-    if (r == 0 && valid_row[hh]) {
-      const int64_t idx = (((int64_t)b * a.Hq + (int64_t)kvh * a.G + gh_row[hh]) * a.R + i_row[hh]) * a.n_ksplit + ks;
-      a.row_m[idx] = m_run[hh];
-      a.row_l[idx] = l;
-    }
+  cta_teardown(ctl, tbase);
+}
+
+// ---------------------------------------------------------------- a row's key splits merged in place:
+// (-m, 1 / l) of the whole row into its split-0 entry; (-inf, 0) for a row past the query rows, so
+// that it adds 2^-inf * 0 = 0 in pass 2
+__global__ void rowmerge_kernel(float2* __restrict__ row_st, int ns, int rowblocks, int rpb, int64_t R, int64_t n) {
+  const int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (e >= n) return;
+  const int64_t blk = e / kTM;
+  const int c = (int)(e % kTM);
+  float2* p = row_st + blk * ns * kTM + c;
+  float M = -INFINITY;
+  for (int s = 0; s < ns; ++s) M = fmaxf(M, p[s * kTM].x);
+  float Ls = 0.f;
+  for (int s = 0; s < ns; ++s) {
+    const float2 x = p[s * kTM];
+    if (x.x != -INFINITY) Ls += x.y * exp2f(x.x - M);
   }
+  const bool valid = (int64_t)(blk % rowblocks) * rpb + (c & (rpb - 1)) < R && M != -INFINITY && Ls > 0.f;
+  p[0] = valid ? make_float2(-M, 1.f / Ls) : make_float2(-INFINITY, 0.f);
 }
 
 // ---------------------------------------------------------------- pass 2
 template <int D>
-__global__ void __launch_bounds__(kT) colsum_kernel(const ScoreArgs a) {
-  constexpr int ROWB = D * 2, NC = D / 8, KC = D / 16, TILE = 64 * ROWB;
-  extern __shared__ __align__(128) uint8_t smem[];   // [2][64 query rows][D], then stats [2][64] (m, 1/l), pos
-  float2* stats = reinterpret_cast<float2*>(smem + 2 * TILE);       // [2][64]
-  int64_t* qpos = reinterpret_cast<int64_t*>(stats + 128);          // [2][64]
-  const int kb = blockIdx.x;
-  const int64_t bh = blockIdx.y;
-  const int b = (int)(bh / a.Hkv), kvh = (int)(bh % a.Hkv);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, r = lane & 3;
-  const int64_t j0 = (int64_t)kb * 64;
-  if (j0 >= a.T) return;
+__global__ void __launch_bounds__(kThr, 1)
+    colsum_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                     const ScoreArgs a) {
+  using L = Layout<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = align1024(smem_raw);
+  Ctl* ctl = reinterpret_cast<Ctl*>(sm + L::CTL_OFF);
+  const int bh = (int)blockIdx.y;
+  const int b = bh / a.Hkv, kvh = bh % a.Hkv;
+  const int warp = threadIdx.x >> 5;
+  const int lq = warp & 3, cq = (warp - 2) >> 2;         // (epilogue warps) lane and column quarter
+  const int lr = lq * 32 + (threadIdx.x & 31);           // accumulator lane = key of the block
+  const int64_t j0 = (int64_t)blockIdx.x * kTM;
+  const int64_t jrel = j0 + lr - a.pos0;                  // rows i >= jrel see this key
 
-  // A fragments: keys j0 + 16*warp + g (+8)
-  uint32_t ka[KC][4];
-  const __half* kbase = a.k + bh * a.T * D;
-#pragma unroll
-  for (int kc = 0; kc < KC; ++kc) {
-#pragma unroll
-    for (int hh = 0; hh < 2; ++hh) {
-      const int64_t j = j0 + 16 * warp + g + 8 * hh;
-      uint32_t lo = 0, hi = 0;
-      if (j < a.T) {
-        lo = *reinterpret_cast<const uint32_t*>(kbase + j * D + kc * 16 + 2 * r);
-        hi = *reinterpret_cast<const uint32_t*>(kbase + j * D + kc * 16 + 2 * r + 8);
-      }
-      ka[kc][hh] = lo;
-      ka[kc][2 + hh] = hi;
-    }
-  }
-  // query-row blocks whose rows can see key j0: rows i with pos0 + i >= j0
+  // the query-row blocks whose rows can see key j0: rows i with pos0 + i >= j0
   const int64_t first_row = std::max<int64_t>(0, j0 - a.pos0);
   const int rb_begin = (int)(first_row / a.rpb);
-  const int rb_end = (int)ceil_div_dev(a.R, a.rpb);
-  const int nblk = rb_end - rb_begin;
+  const int ntiles = std::max(0, a.rowblocks - rb_begin);
+  const int plane0 = b * a.Hq + kvh * a.G;
+  const float2* stats = a.row_st + (int64_t)bh * a.rowblocks * a.n_ksplit * kTM;
 
-  auto load_block = [&](int t, int stage) {
-    const int rb = rb_begin + t;
-    uint8_t* Qs = smem + stage * TILE;
-    const int col = tid % NC;
-    for (int q = tid / NC; q < 64; q += kT / NC) {
-      int gh;
-      int64_t i;
-      qrow_map(a, rb, q, gh, i);
-      const bool ok = gh < a.G && i < a.R;
-      const __half* src = a.q + (((int64_t)b * a.Hq + (int64_t)kvh * a.G + (ok ? gh : 0)) * a.R + (ok ? i : 0)) * D;
-      cp_async16(Qs + q * ROWB + ((col ^ (q & 7)) << 4), src + col * 8, ok ? 16 : 0);
-    }
-    if (tid < 64) {
-      int gh;
-      int64_t i;
-      qrow_map(a, rb, tid, gh, i);
-      float2 st = make_float2(INFINITY, 0.f);       // (m, 1/l); invalid row -> p = 0
-      int64_t p = -1;
-      if (gh < a.G && i < a.R) {
-        const int64_t idx = (((int64_t)b * a.Hq + (int64_t)kvh * a.G + gh) * a.R + i) * a.n_ksplit;
-        float M = -INFINITY;
-        for (int s = 0; s < a.n_ksplit; ++s) M = fmaxf(M, a.row_m[idx + s]);
-        float L = 0.f;
-        for (int s = 0; s < a.n_ksplit; ++s) {
-          const float ms = a.row_m[idx + s];
-          if (ms != -INFINITY) L += a.row_l[idx + s] * exp2f(ms - M);
+  const uint32_t tbase = cta_setup(ctl);
+  float acc = 0.f;
+  run_roles<D, true>(
+      sm, ctl, tbase, ntiles,
+      [&](uint64_t* bar) {
+        tc_mbar_expect_tx(bar, L::TILE);
+        for (int at = 0; at < D / 64; ++at)
+          tma_load_3d(sm + L::A_OFF + at * L::ATOM, &kmap, at * 64, (int)j0, bh, bar);
+      },
+      [&](int t, int s, uint64_t* bar) {
+        const int rb = rb_begin + t;
+        tc_mbar_expect_tx(bar, L::TILE + kStatBytes);
+        for (int g = 0; g < a.G; ++g)
+          for (int at = 0; at < D / 64; ++at)
+            tma_load_3d(sm + L::B_OFF + s * L::TILE + at * L::ATOM + g * a.rpb * 128, &qmap, at * 64, rb * a.rpb,
+                        plane0 + g, bar);
+        bulk_load(sm + L::ST_OFF + s * kStatBytes, stats + (int64_t)rb * a.n_ksplit * kTM, kStatBytes, bar);
+      },
+      [&](int t, uint32_t col, int s) {
+        const int64_t i0 = (int64_t)(rb_begin + t) * a.rpb;   // row index of the tile's first row per head
+        const float2* s2 = reinterpret_cast<const float2*>(sm + L::ST_OFF + s * kStatBytes) + cq * kCQ;
+        float v[kCQ];
+        tc_ld32(col + ((uint32_t)(lq * 32) << 16) + (uint32_t)(cq * kCQ), v);
+        float sp[4] = {0.f, 0.f, 0.f, 0.f};
+        if (i0 >= j0 + kTM - 1 - a.pos0) {   // every row of the tile sees every key of the block
+#pragma unroll
+          for (int e = 0; e < kCQ; ++e) {
+            const float2 w = s2[e];
+            sp[e & 3] = fmaf(ex2_approx(fmaf(v[e], a.scale_log2, w.x)), w.y, sp[e & 3]);
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < kCQ; ++e) {
+            const float2 w = s2[e];
+            const float p = ex2_approx(fmaf(v[e], a.scale_log2, w.x)) * w.y;
+            if (i0 + ((cq * kCQ + e) & (a.rpb - 1)) >= jrel) sp[e & 3] += p;
+          }
         }
-        st = make_float2(M, L > 0.f ? 1.f / L : 0.f);
-        p = a.pos0 + i;
-      }
-      stats[stage * 64 + tid] = st;
-      qpos[stage * 64 + tid] = p;
-    }
-  };
+        acc += (sp[0] + sp[1]) + (sp[2] + sp[3]);
+      });
+  // the four column quarters of each key summed
+  float* mrg = reinterpret_cast<float*>(sm + L::MRG_OFF);
+  if (warp >= 2) mrg[cq * kTM + lr] = acc;
+  __syncthreads();
+  if (warp >= 2 && cq == 0 && j0 + lr < a.T)
+    a.score[(int64_t)bh * a.T + j0 + lr] = (mrg[lr] + mrg[kTM + lr]) + (mrg[2 * kTM + lr] + mrg[3 * kTM + lr]);
+  cta_teardown(ctl, tbase);
+}
 
-  float col[2] = {0.f, 0.f};
-  if (nblk > 0) load_block(0, 0);
-  cp_async_commit();
-  for (int t = 0; t < nblk; ++t) {
-    cp_async_wait<0>();
-    __syncthreads();
-    if (t + 1 < nblk) load_block(t + 1, (t + 1) & 1);
-    cp_async_commit();
-    const uint8_t* Qs = smem + (t & 1) * TILE;
-    const float2* st = stats + (t & 1) * 64;
-    const int64_t* qp = qpos + (t & 1) * 64;
-    float sc[8][4];
-#pragma unroll
-    for (int n = 0; n < 8; ++n) sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
-    const int mi = lane >> 3, row = lane & 7;
-#pragma unroll
-    for (int kc = 0; kc < KC; ++kc) {
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        uint32_t bq[4];
-        const int qq = np * 16 + (mi >> 1) * 8 + row;
-        const int ch = kc * 2 + (mi & 1);
-        ldsm_x4(bq, Qs + qq * ROWB + ((ch ^ (qq & 7)) << 4));
-        mma16816(sc[2 * np], ka[kc][0], ka[kc][1], ka[kc][2], ka[kc][3], bq[0], bq[1]);
-        mma16816(sc[2 * np + 1], ka[kc][0], ka[kc][1], ka[kc][2], ka[kc][3], bq[2], bq[3]);
-      }
-    }
-#pragma unroll
-    for (int n = 0; n < 8; ++n) {
-#pragma unroll
-      for (int e = 0; e < 2; ++e) {
-        const int q = n * 8 + 2 * r + e;
-        const float2 s2 = st[q];
-        const int64_t pq = qp[q];
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-          const int64_t j = j0 + 16 * warp + g + 8 * hh;
-          if (pq >= j) col[hh] += exp2f(sc[n][2 * hh + e] * a.scale_log2 - s2.x) * s2.y;
-        }
-      }
-    }
-  }
-  cp_async_wait<0>();
-#pragma unroll
-  for (int hh = 0; hh < 2; ++hh) {
-    float v = col[hh];
-    v += __shfl_xor_sync(0xffffffffu, v, 1);
-    v += __shfl_xor_sync(0xffffffffu, v, 2);
-    const int64_t j = j0 + 16 * warp + g + 8 * hh;
-    if (r == 0 && j < a.T) a.score[bh * a.T + j] = v;
-  }
+// ---------------------------------------------------------------- host side
+using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                 const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encoder() {
+  static const EncodeTiled fn = []() -> EncodeTiled {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return nullptr;
+    return reinterpret_cast<EncodeTiled>(p);
+  }();
+  return fn;
+}
+
+// fp16 [planes][rows][D] read in boxes of 64 x box_rows x 1 with the 128-byte swizzle; rows past
+// the end read as zero
+cudaError_t make_map(CUtensorMap* m, const void* base, int D, int64_t rows, int64_t planes, int box_rows) {
+  const EncodeTiled enc = encoder();
+  if (enc == nullptr) return cudaErrorNotSupported;
+  const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)planes};
+  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)rows * D * 2};
+  const cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
+  const cuuint32_t es[3] = {1, 1, 1};
+  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
 template <int D>
-cudaError_t launch_scores_t(const ScoreArgs& a, int rowblocks, int units, int keyblocks, cudaStream_t st) {
-  const size_t smem1 = 2 * 64 * D * 2;
-  const size_t smem2 = 2 * 64 * D * 2 + 128 * sizeof(float2) + 128 * sizeof(int64_t);
-  cudaError_t e = cudaFuncSetAttribute(rowstats_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
+cudaError_t launch_scores_t(const CUtensorMap& qm, const CUtensorMap& km, const ScoreArgs& a, int units, int keyblocks,
+                            cudaStream_t st) {
+  // at most two CTAs (2 x 256 of the 512 tensor-memory columns) share an SM, so no allocation waits
+  constexpr int smem = Layout<D>::ALLOC > 80 * 1024 ? Layout<D>::ALLOC : 80 * 1024;
+  static_assert(smem <= 227 * 1024, "shared memory");
+  cudaError_t e = cudaFuncSetAttribute(rowstats_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(colsum_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem2);
+  e = cudaFuncSetAttribute(colsum_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  rowstats_kernel<D><<<dim3(a.n_ksplit, rowblocks, units), kT, smem1, st>>>(a);
+  rowstats_tc_kernel<D><<<dim3(a.n_ksplit, a.rowblocks, units), kThr, smem, st>>>(qm, km, a);
   e = cudaPeekAtLastError();
   if (e != cudaSuccess) return e;
-  colsum_kernel<D><<<dim3(keyblocks, units), kT, smem2, st>>>(a);
+  const int64_t n = (int64_t)units * a.rowblocks * kTM;
+  rowmerge_kernel<<<(unsigned)ceil_div(n, 256), 256, 0, st>>>(a.row_st, a.n_ksplit, a.rowblocks, a.rpb, a.R, n);
+  e = cudaPeekAtLastError();
+  if (e != cudaSuccess) return e;
+  colsum_tc_kernel<D><<<dim3(keyblocks, units), kThr, smem, st>>>(qm, km, a);
   return cudaPeekAtLastError();
 }
 
@@ -309,33 +464,36 @@ cudaError_t launch_scores_t(const ScoreArgs& a, int rowblocks, int units, int ke
 
 cudaError_t launch_prefill_scores(const mkv_config& c, const void* q, int64_t q_rows, int64_t T,
                                   const void* full_k, const PrefillWs& ws, cudaStream_t st) {
+  if (q_rows <= 0 || T <= 0) return cudaSuccess;
   ScoreArgs a{};
-  a.q = static_cast<const __half*>(q);
-  a.k = static_cast<const __half*>(full_k);
   a.R = q_rows;
   a.T = T;
   a.pos0 = T - q_rows;
   a.Hq = c.Hq;
   a.Hkv = c.Hkv;
   a.G = c.Hq / c.Hkv;
-  a.rpb = 64 / a.G;
+  a.rpb = kTM / a.G;
+  a.rowblocks = (int)ceil_div(q_rows, a.rpb);
   const float scale = c.softmax_scale > 0.f ? c.softmax_scale : 1.0f / sqrtf((float)c.D);
   a.scale_log2 = scale * kLog2e;
   const int units = c.B * c.Hkv;
-  const int rowblocks = (int)ceil_div(q_rows, a.rpb);
-  const int64_t tiles = ceil_div(T, 64);
-  // split the key range only when there are few row blocks (observation window)
-  int64_t ns = std::max<int64_t>(1, ceil_div(4 * kNumSMs, (int64_t)rowblocks * units));
-  ns = std::min<int64_t>(ns, std::min<int64_t>(tiles, T / std::max<int64_t>(q_rows, 1)));
+  const int64_t tiles = ceil_div(T, kTN);
+  if (a.rowblocks > 65535 || T > INT32_MAX - kTN) return cudaErrorInvalidConfiguration;
+  // split the key range only when the row blocks are fewer than the SMs (an observation window);
+  // the splits' partials stay within the row-statistics workspace of B Hq (T + 128) entries
+  int64_t ns = ceil_div(kNumSMs, (int64_t)a.rowblocks * units);
+  ns = std::min<int64_t>(ns, std::min<int64_t>(tiles, (T + kTM) / ((int64_t)a.rowblocks * a.rpb)));
   ns = std::max<int64_t>(ns, 1);
   a.tiles_per_split = (int)ceil_div(tiles, ns);
   a.n_ksplit = (int)ceil_div(tiles, a.tiles_per_split);
-  a.row_m = ws.row_m;
-  a.row_l = ws.row_l;
+  a.row_st = ws.row_st;
   a.score = ws.score;
-  const int keyblocks = (int)tiles;
-  if (c.D == 128) return launch_scores_t<128>(a, rowblocks, units, keyblocks, st);
-  return launch_scores_t<64>(a, rowblocks, units, keyblocks, st);
+  CUtensorMap qm, km;
+  cudaError_t e = make_map(&qm, q, c.D, q_rows, (int64_t)c.B * c.Hq, a.rpb);
+  if (e == cudaSuccess) e = make_map(&km, full_k, c.D, T, units, kTN);
+  if (e != cudaSuccess) return e;
+  if (c.D == 128) return launch_scores_t<128>(qm, km, a, units, (int)tiles, st);
+  return launch_scores_t<64>(qm, km, a, units, (int)tiles, st);
 }
 
 }  // namespace mkv

@@ -276,7 +276,8 @@ cudaError_t launch_snap_keep(const mkv_config& c, const void* full_k, const void
   const bool identity = T <= c.snap_keep;
   const int64_t n = identity ? T : c.snap_keep;
   if (!identity) {
-    snap_keep_kernel<<<units, kSelThreads, 0, st>>>(ws.score, T, c.snap_window, c.snap_pool, c.snap_keep, ws.row_m,
+    snap_keep_kernel<<<units, kSelThreads, 0, st>>>(ws.score, T, c.snap_window, c.snap_pool, c.snap_keep,
+                                                    reinterpret_cast<float*>(ws.row_st),
                                                     ws.keep);
     cudaError_t e = cudaPeekAtLastError();
     if (e != cudaSuccess) return e;
