@@ -524,6 +524,80 @@ def measure_config(name, w, dev, seed, method, steps, warmup, peak, no_graph=Fal
     return row
 
 
+def tensor_peak():
+    """(dense fp16/bf16 TFLOP/s burst peak, how it was obtained): fp16 runs at the bf16 rate."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        if "bf16_tflops" in d:
+            return d["bf16_tflops"], "measured (cuBLAS bf16 burst; fp16 has the same tensor rate)"
+    return 1900.0, "fallback"
+
+
+def measure_setup(dev, seed, reps=5, warmup=3):
+    """The prefill-side calls timed apart from decode, one layer each: mkv_h2o_prefill on the H2O
+    workload (causal scores over the whole prompt, then the heavy + recent keep and gather) and
+    mkv_snap_compress on the RocketKV workload (the observation window's scores, pooling, keep and
+    gather).  Their scoring is two tcgen05 products of the causal Q K^T (row statistics, then column
+    sums): FLOPs = 2 passes x 2 D per causal (query row, key) pair per query head -- the least an
+    exact column sum does without storing the T x T scores."""
+    import torch
+    import paper_2609_07966_gb300 as mkv
+    from paper_2609_07966_gb300 import caches
+    peak, kind = tensor_peak()
+    out = {}
+    for name in ("h2o20", "rocket1024"):
+        w = WORKLOADS[name]()
+        x = synth.device_layer_inputs(w, seed, 0, device=dev, n_tokens=w.T, with_prompt_queries=True)
+        kp = x["k"][:, :, :w.T].contiguous()
+        vp = x["v"][:, :, :w.T].contiguous()
+        if name == "h2o20":
+            cfg = mkv.config(mkv.MKV_H2O, w.B, w.Hq, w.Hkv, w.D, h2o_heavy=w.h2o_heavy, h2o_recent=w.h2o_recent)
+            T_cap = w.h2o_heavy + w.h2o_recent + 1
+            qp = x["q_prompt"].contiguous()
+            rows, pairs = w.T, w.T * (w.T + 1) / 2
+            call = "mkv_h2o_prefill"
+        else:
+            cfg = mkv.config(mkv.MKV_ROCKET, w.B, w.Hq, w.Hkv, w.D, snap_window=w.snap_window,
+                             snap_pool=w.snap_pool, snap_keep=w.snap_keep, page_size=w.page,
+                             topk_pages=w.topk_pages, topq_dims=w.topq_dims)
+            T_cap = (min(w.T, w.snap_keep) + 15) // 16 * 16
+            qp = x["q_prompt"][:, :, w.T - w.snap_window:].contiguous()
+            W = w.snap_window
+            rows, pairs = W, W * (w.T - W) + W * (W + 1) / 2
+            call = "mkv_snap_compress"
+        del x
+        cache = caches.alloc_cache(cfg, T_cap, device=dev)
+        ws, nws = caches.workspace(cfg, max(w.T, T_cap), device=dev)
+        if name == "h2o20":
+            fn = lambda: mkv.mkv_h2o_prefill(cfg, qp.data_ptr(), kp.data_ptr(), vp.data_ptr(), w.T, cache.c,
+                                             ws.data_ptr(), nws)
+        else:
+            fn = lambda: mkv.mkv_snap_compress(cfg, qp.data_ptr(), kp.data_ptr(), vp.data_ptr(), w.T, cache.c, 0,
+                                               ws.data_ptr(), nws)
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        st = torch.cuda.current_stream()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+        for a, b in ev:
+            a.record(st)
+            fn()
+            b.record(st)
+        torch.cuda.synchronize()
+        ms = statistics.median(a.elapsed_time(b) for a, b in ev)
+        flops = 2 * 2 * w.D * pairs * w.B * w.Hq
+        tf = flops / (ms * 1e-3) / 1e12
+        out[name] = {"call": call, "workload": f"{w.name}, one layer", "batch": w.B, "context": w.T,
+                     "query_rows": rows, "ms": ms, "status": mkv.mkv_get_status(),
+                     "roofline": {"bound": "tensor", "achieved": tf, "peak": peak, "unit": "TFLOP/s",
+                                  "frac": tf / peak, "peak_kind": kind, "flops_per_call": flops,
+                                  "note": "the whole call (scoring, keep, gather) timed; FLOPs of the scoring"}}
+        del qp, kp, vp, cache, ws
+        torch.cuda.empty_cache()
+    return out
+
+
 # --------------------------------------------------------------------------- CPU oracle arm
 
 def oracle_tokens_per_s(name: str, w, budget_s: float, seed: int = 0):
@@ -614,6 +688,8 @@ def main():
                     help="1: also measure the ten configurations at contexts 4K/16K/64K/128K (batch 32/16/4/1)")
     ap.add_argument("--sweep-steps", type=int, default=5, help="timed steps per sweep configuration")
     ap.add_argument("--cpu-all-cores", type=int, default=1, help="1: also time the oracle on every host core")
+    ap.add_argument("--setup", type=int, default=1,
+                    help="1: also time the prefill-side calls (H2O prefill, SnapKV compression) on their workloads")
     ap.add_argument("--profile", action="store_true",
                     help="profiling only: run warmup + steps and exit (for ncu), no JSON line")
     args = ap.parse_args()
@@ -727,6 +803,8 @@ def main():
                 line["sweep"][wx.name] = measure_config(wx.name, wx, dev, args.seed, meth, args.sweep_steps, 3,
                                                         peak, args.no_graph, synthetic_h2o_cache=True)
         line["sweep_wall_s"] = time.perf_counter() - t_sw
+    if world == 1 and args.setup:
+        line["setup"] = measure_setup(dev, args.seed)
     if rank == 0:
         if world == 1:
             v, sample = oracle_tokens_per_s(args.workload, w, args.cpu_budget, seed=args.seed)

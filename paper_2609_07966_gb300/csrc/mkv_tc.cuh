@@ -74,6 +74,13 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const void* map, int x, i
       "l"(map), "r"(x), "r"(y), "r"(z), "r"(smem_addr(bar))
       : "memory");
 }
+__device__ __forceinline__ void tma_load_4d(void* dst, const void* map, int x, int y, int z, int w, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::
+          "r"(smem_addr(dst)),
+      "l"(map), "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_addr(bar))
+      : "memory");
+}
 // bulk copy of `bytes` (a multiple of 16; both addresses 16-byte aligned) into shared memory
 __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
@@ -132,6 +139,18 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, float (&v)[32]) {
     v[i] = __uint_as_float(r0[i]);
     v[16 + i] = __uint_as_float(r1[i]);
   }
+}
+
+// 64 consecutive fp32 columns (four loads in flight, one wait)
+__device__ __forceinline__ void tc_ld64(uint32_t taddr, float (&v)[64]) {
+  uint32_t r[4][16];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) tc_ld16_issue(taddr + 16 * k, r[k]);
+  tc_wait_ld();
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[16 * k + i] = __uint_as_float(r[k][i]);
 }
 
 // 2^x by the special-function unit's approximation (one instruction; results below the normal

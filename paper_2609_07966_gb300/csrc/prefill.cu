@@ -20,10 +20,13 @@
 //   warp 0 (one thread) loads operand tiles by TMA (tensor maps with the 128-byte swizzle, the
 //           K-major layout the MMA reads) into a ring of kS stages, and in pass 2 each tile's 128
 //           row statistics by a bulk copy beside it;
-//   warp 1 (one thread) issues the D / 16 MMAs of a tile into one of two tensor-memory
-//           accumulator buffers, then commits to the stage's and the buffer's mbarriers;
-//   warps 2..17 read a finished accumulator (warp w: lanes 32 (w % 4) .. + 31, the lane quarter
-//           it may access, and column quarter (w - 2) / 4) and release the buffer.
+//   warp 1 (one thread) issues the D / 16 MMAs of tile t into tensor-memory accumulator buffer
+//           t % 4 (all 512 columns; one CTA per SM), then commits to the stage's and the buffer's
+//           mbarriers;
+//   warps 2..17 read finished accumulators in two groups of eight: group g takes the tiles
+//           t = g mod 2, so the groups work a tile apart and one group's exponentials overlap the
+//           other's loads and reductions; warp w reads lanes 32 (w % 4) .. + 31 (the lane quarter
+//           it may access) and one half of the 128 columns.
 // Loads, products and epilogues of different tiles overlap; nothing in the tile loop waits on a
 // CTA-wide barrier.  Every wait is bounded: on a timeout the role raises MKV_FLAG_WAIT_TIMEOUT and
 // sets a flag that ends the other roles' waits; the CTA then waits (bounded) for the copies and
@@ -54,10 +57,12 @@ namespace {
 
 constexpr int kTM = 128;                 // rows of the held operand (the MMA's M)
 constexpr int kTN = 128;                 // rows of a streamed tile (the MMA's N)
-constexpr int kEpiWarps = 16;            // four lane quarters x four column quarters
+constexpr int kGroupWarps = 8;           // an epilogue group: four lane quarters x two column halves
+constexpr int kEpiWarps = 2 * kGroupWarps;
 constexpr int kThr = (2 + kEpiWarps) * 32;
-constexpr int kCQ = kTN / 4;             // accumulator columns an epilogue thread reads per tile
-constexpr int kS = 4;                    // operand stages
+constexpr int kCH = kTN / 2;             // accumulator columns an epilogue thread reads per tile
+constexpr int kNB = 4;                   // tensor-memory accumulator buffers of 128 columns
+constexpr int kS = 4;                    // operand stages (even: stage s's tiles all go to group s % 2)
 constexpr int kStatBytes = kTN * 8;      // one query tile's (-m, 1 / l)
 constexpr uint32_t kWaitLimit = 1u << 22;
 
@@ -78,7 +83,7 @@ struct Layout {
   static constexpr int A_OFF = 0;
   static constexpr int B_OFF = TILE;                      // [kS] streamed tiles
   static constexpr int ST_OFF = B_OFF + kS * TILE;        // [kS] pass 2: the tile's row statistics
-  static constexpr int MRG_OFF = ST_OFF + kS * kStatBytes;   // [4][128] the column quarters' partials
+  static constexpr int MRG_OFF = ST_OFF + kS * kStatBytes;   // [4][128] the (group, half) partials
   static constexpr int CTL_OFF = MRG_OFF + 4 * kTM * 8;
   static constexpr int BYTES = CTL_OFF + 256;
   static constexpr int ALLOC = BYTES + 1024;              // slack to align the base to 1024 B
@@ -87,9 +92,9 @@ struct Layout {
 struct Ctl {
   uint64_t full[kS];     // stage s loaded (TMA transaction bytes)
   uint64_t empty[kS];    // stage s's operand read by the tensor core
-  uint64_t sempty[kS];   // stage s's row statistics read by every epilogue warp (pass 2)
-  uint64_t tfull[2];     // accumulator buffer b holds a finished product
-  uint64_t tempty[2];    // accumulator buffer b read by every epilogue warp
+  uint64_t sempty[kS];   // stage s's row statistics read by its epilogue group (pass 2)
+  uint64_t tfull[kNB];   // accumulator buffer b holds a finished product
+  uint64_t tempty[kNB];  // accumulator buffer b read by its epilogue group
   uint64_t abar;         // the held operand loaded
   uint32_t tslot;        // tensor-memory base address
   int fail;              // a wait ran out: every role stops
@@ -113,29 +118,32 @@ __device__ __forceinline__ bool role_wait(uint64_t* bar, uint32_t parity, volati
   return false;
 }
 
-// D[tmem] = A (128 rows) x B (128 rows)^T over K = D: D / 16 MMAs, issued by one thread
+// D[tmem] = A (128 rows) x B (128 rows)^T over K = D: D / 16 MMAs, issued by one thread.  `a` and
+// `b` are the shared-memory descriptors of the tiles' first K step; a K step adds a compile-time
+// offset to the start-address field (no carry: shared addresses stay below 2^18).
 template <int D>
-__device__ __forceinline__ void issue_tile(uint32_t d_tmem, uint32_t a_s, uint32_t b_s) {
+__device__ __forceinline__ void issue_tile(uint32_t d_tmem, uint64_t a, uint64_t b) {
   constexpr uint32_t kId = tc_idesc_f16(kTM, kTN);
 #pragma unroll
   for (int kk = 0; kk < D / 16; ++kk) {
-    const uint32_t off = (uint32_t)((kk >> 2) * Layout<D>::ATOM + (kk & 3) * 32);
-    tc_mma(d_tmem, tc_desc_sw128(a_s + off), tc_desc_sw128(b_s + off), kId, kk > 0 ? 1u : 0u);
+    constexpr int kAtom = Layout<D>::ATOM;
+    const uint64_t off = (uint64_t)(((kk >> 2) * kAtom + (kk & 3) * 32) >> 4);
+    tc_mma(d_tmem, a + off, b + off, kId, kk > 0 ? 1u : 0u);
   }
 }
 
-// Barriers and tensor memory of a CTA; returns the tensor-memory base (2 x 128 columns).
+// Barriers and tensor memory of a CTA; returns the tensor-memory base (kNB x 128 columns).
 __device__ __forceinline__ uint32_t cta_setup(Ctl* ctl) {
-  if ((threadIdx.x >> 5) == 0) tc_alloc(&ctl->tslot, 2 * kTN);
+  if ((threadIdx.x >> 5) == 0) tc_alloc(&ctl->tslot, kNB * kTN);
   if (threadIdx.x == 0) {
     for (int s = 0; s < kS; ++s) {
       tc_mbar_init(&ctl->full[s], 1);
       tc_mbar_init(&ctl->empty[s], 1);
-      tc_mbar_init(&ctl->sempty[s], kEpiWarps);
+      tc_mbar_init(&ctl->sempty[s], kGroupWarps);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kNB; ++b) {
       tc_mbar_init(&ctl->tfull[b], 1);
-      tc_mbar_init(&ctl->tempty[b], kEpiWarps);
+      tc_mbar_init(&ctl->tempty[b], kGroupWarps);
     }
     tc_mbar_init(&ctl->abar, 1);
     tc_fence_mbar_init();
@@ -159,17 +167,18 @@ __device__ __forceinline__ void cta_teardown(Ctl* ctl, uint32_t tbase) {
       tc_mbar_wait(&ctl->full[t % kS], (uint32_t)((t / kS) & 1), kWaitLimit);
     if (ctl->mma_issued > 0) {
       const int t = ctl->mma_issued - 1;
-      tc_mbar_wait(&ctl->tfull[t & 1], (uint32_t)((t >> 1) & 1), kWaitLimit);
+      tc_mbar_wait(&ctl->tfull[t % kNB], (uint32_t)((t / kNB) & 1), kWaitLimit);
     }
   }
   __syncthreads();
   tc_fence_after();
-  if ((threadIdx.x >> 5) == 0) tc_dealloc(tbase, 2 * kTN);
+  if ((threadIdx.x >> 5) == 0) tc_dealloc(tbase, kNB * kTN);
 }
 
 // The three roles over `ntiles` streamed tiles.  issue_a(bar) loads the held operand;
-// issue_b(t, s, bar) loads tile t into stage s; epi(t, col, s) reads tile t's accumulator (columns
-// from tensor-memory address col, lane 0) and, with kStats, the statistics of stage s.
+// issue_b(t, s, bar) loads tile t into stage s; epi(t, col, s) reads the thread's half of tile t's
+// accumulator (columns from tensor-memory address col, lane 0) and, with kStats, the statistics
+// of stage s.
 template <int D, bool kStats, typename IssueA, typename IssueB, typename Epi>
 __device__ __forceinline__ void run_roles(uint8_t* sm, Ctl* ctl, uint32_t tbase, int ntiles, IssueA issue_a,
                                           IssueB issue_b, Epi epi) {
@@ -192,29 +201,31 @@ __device__ __forceinline__ void run_roles(uint8_t* sm, Ctl* ctl, uint32_t tbase,
     }
   } else if (warp == 1) {
     if (lane == 0) {                      // MMA issuer
-      const uint32_t a_s = smem_addr(sm + L::A_OFF);
+      const uint64_t a_desc = tc_desc_sw128(smem_addr(sm + L::A_OFF));
+      const uint64_t b_desc = tc_desc_sw128(smem_addr(sm + L::B_OFF));
       if (role_wait(&ctl->abar, 0, fail)) {
         for (int t = 0; t < ntiles; ++t) {
-          const int s = t % kS, bf = t & 1, u = t >> 1;
+          const int s = t % kS, bf = t % kNB, u = t / kNB;
           if (!role_wait(&ctl->full[s], (uint32_t)((t / kS) & 1), fail)) break;
           if (u > 0 && !role_wait(&ctl->tempty[bf], (uint32_t)((u - 1) & 1), fail)) break;
           tc_fence_after();
-          issue_tile<D>(tbase + (uint32_t)(bf * kTN), a_s, smem_addr(sm + L::B_OFF + s * L::TILE));
+          issue_tile<D>(tbase + (uint32_t)(bf * kTN), a_desc, b_desc + (uint64_t)((s * L::TILE) >> 4));
           tc_commit(&ctl->empty[s]);
           tc_commit(&ctl->tfull[bf]);
           ctl->mma_issued = t + 1;
         }
       }
     }
-  } else {                                // epilogue warps
-    for (int t = 0; t < ntiles; ++t) {
-      const int s = t % kS, bf = t & 1;
-      bool ok = role_wait(&ctl->tfull[bf], (uint32_t)((t >> 1) & 1), fail);
+  } else {                                // epilogue warps: group (warp - 2) / 8 takes every other tile
+    const int grp = (warp - 2) / kGroupWarps, half = ((warp - 2) >> 2) & 1;
+    for (int t = grp; t < ntiles; t += 2) {
+      const int s = t % kS, bf = t % kNB;
+      bool ok = role_wait(&ctl->tfull[bf], (uint32_t)((t / kNB) & 1), fail);
       // the statistics came with the stage's operand: their copy completed that phase of full[s]
       if (kStats) ok = ok && role_wait(&ctl->full[s], (uint32_t)((t / kS) & 1), fail);
       if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
-      epi(t, tbase + (uint32_t)(bf * kTN), s);
+      epi(t, tbase + (uint32_t)(bf * kTN + half * kCH), s);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
@@ -239,7 +250,8 @@ __global__ void __launch_bounds__(kThr, 1)
   const int bh = (int)blockIdx.z;
   const int b = bh / a.Hkv, kvh = bh % a.Hkv;
   const int warp = threadIdx.x >> 5;
-  const int lq = warp & 3, cq = (warp - 2) >> 2;         // (epilogue warps) lane and column quarter
+  const int lq = warp & 3, cq = (warp - 2) >> 2;         // (epilogue warps) lane quarter; group x half
+  const int hf = cq & 1;                                 // column half of the tile
   const int lr = lq * 32 + (threadIdx.x & 31);           // accumulator lane = query row of the block
 
   // the block's last valid row bounds its causal key range
@@ -250,35 +262,33 @@ __global__ void __launch_bounds__(kThr, 1)
   const int ntiles = k_end > k_begin ? (int)ceil_div_dev(k_end - k_begin, kTN) : 0;
   const int64_t irow = (int64_t)rb * a.rpb + (lr & (a.rpb - 1));
   const int64_t lim = irow < a.R ? std::min<int64_t>(k_end - 1, a.pos0 + irow) : -1;   // last key it sees
-  const int plane0 = b * a.Hq + kvh * a.G;               // the group's first query head
 
   const uint32_t tbase = cta_setup(ctl);
   float m_run = -INFINITY, l_run = 0.f;
   run_roles<D, false>(
       sm, ctl, tbase, ntiles,
-      [&](uint64_t* bar) {                // head g's rows of the block are tile rows g rpb ..
+      [&](uint64_t* bar) {                // one box of G heads x rpb rows: head g's rows are tile rows g rpb ..
         tc_mbar_expect_tx(bar, L::TILE);
-        for (int g = 0; g < a.G; ++g)
-          for (int at = 0; at < D / 64; ++at)
-            tma_load_3d(sm + L::A_OFF + at * L::ATOM + g * a.rpb * 128, &qmap, at * 64, rb * a.rpb, plane0 + g, bar);
+        for (int at = 0; at < D / 64; ++at)
+          tma_load_4d(sm + L::A_OFF + at * L::ATOM, &qmap, at * 64, rb * a.rpb, kvh * a.G, b, bar);
       },
       [&](int t, int s, uint64_t* bar) {
         tc_mbar_expect_tx(bar, L::TILE);
         for (int at = 0; at < D / 64; ++at)
-          tma_load_3d(sm + L::B_OFF + s * L::TILE + at * L::ATOM, &kmap, at * 64, (int)(k_begin + (int64_t)t * kTN),
-                      bh, bar);
+          tma_load_4d(sm + L::B_OFF + s * L::TILE + at * L::ATOM, &kmap, at * 64, (int)(k_begin + (int64_t)t * kTN),
+                      kvh, b, bar);
       },
       [&](int t, uint32_t col, int) {
-        const int64_t jc = k_begin + (int64_t)t * kTN + cq * kCQ;
-        float v[kCQ];
-        tc_ld32(col + ((uint32_t)(lq * 32) << 16) + (uint32_t)(cq * kCQ), v);
+        const int64_t jc = k_begin + (int64_t)t * kTN + hf * kCH;
+        float v[kCH];
+        tc_ld64(col + ((uint32_t)(lq * 32) << 16), v);
         float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};   // max of the raw products
-        if (jc + kCQ - 1 <= lim) {
+        if (jc + kCH - 1 <= lim) {
 #pragma unroll
-          for (int e = 0; e < kCQ; ++e) mx[e & 3] = fmaxf(mx[e & 3], v[e]);
+          for (int e = 0; e < kCH; ++e) mx[e & 3] = fmaxf(mx[e & 3], v[e]);
         } else {
 #pragma unroll
-          for (int e = 0; e < kCQ; ++e) {
+          for (int e = 0; e < kCH; ++e) {
             v[e] = jc + e <= lim ? v[e] : -INFINITY;
             mx[e & 3] = fmaxf(mx[e & 3], v[e]);
           }
@@ -288,12 +298,12 @@ __global__ void __launch_bounds__(kThr, 1)
         if (m_new != -INFINITY) {
           float sp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-          for (int e = 0; e < kCQ; ++e) sp[e & 3] += ex2_approx(fmaf(v[e], a.scale_log2, -m_new));
+          for (int e = 0; e < kCH; ++e) sp[e & 3] += ex2_approx(fmaf(v[e], a.scale_log2, -m_new));
           l_run = l_run * ex2_approx(m_run - m_new) + ((sp[0] + sp[1]) + (sp[2] + sp[3]));
           m_run = m_new;
         }
       });
-  // the four column quarters of each row merged into this split's (m, l)
+  // the (group, half) partials of each row merged into this split's (m, l)
   float2* mrg = reinterpret_cast<float2*>(sm + L::MRG_OFF);
   if (warp >= 2) mrg[cq * kTM + lr] = make_float2(m_run, l_run);
   __syncthreads();
@@ -346,7 +356,8 @@ __global__ void __launch_bounds__(kThr, 1)
   const int bh = (int)blockIdx.y;
   const int b = bh / a.Hkv, kvh = bh % a.Hkv;
   const int warp = threadIdx.x >> 5;
-  const int lq = warp & 3, cq = (warp - 2) >> 2;         // (epilogue warps) lane and column quarter
+  const int lq = warp & 3, cq = (warp - 2) >> 2;         // (epilogue warps) lane quarter; group x half
+  const int hf = cq & 1;                                 // column half of the tile
   const int lr = lq * 32 + (threadIdx.x & 31);           // accumulator lane = key of the block
   const int64_t j0 = (int64_t)blockIdx.x * kTM;
   const int64_t jrel = j0 + lr - a.pos0;                  // rows i >= jrel see this key
@@ -355,7 +366,6 @@ __global__ void __launch_bounds__(kThr, 1)
   const int64_t first_row = std::max<int64_t>(0, j0 - a.pos0);
   const int rb_begin = (int)(first_row / a.rpb);
   const int ntiles = std::max(0, a.rowblocks - rb_begin);
-  const int plane0 = b * a.Hq + kvh * a.G;
   const float2* stats = a.row_st + (int64_t)bh * a.rowblocks * a.n_ksplit * kTM;
 
   const uint32_t tbase = cta_setup(ctl);
@@ -365,40 +375,38 @@ __global__ void __launch_bounds__(kThr, 1)
       [&](uint64_t* bar) {
         tc_mbar_expect_tx(bar, L::TILE);
         for (int at = 0; at < D / 64; ++at)
-          tma_load_3d(sm + L::A_OFF + at * L::ATOM, &kmap, at * 64, (int)j0, bh, bar);
+          tma_load_4d(sm + L::A_OFF + at * L::ATOM, &kmap, at * 64, (int)j0, kvh, b, bar);
       },
       [&](int t, int s, uint64_t* bar) {
         const int rb = rb_begin + t;
         tc_mbar_expect_tx(bar, L::TILE + kStatBytes);
-        for (int g = 0; g < a.G; ++g)
-          for (int at = 0; at < D / 64; ++at)
-            tma_load_3d(sm + L::B_OFF + s * L::TILE + at * L::ATOM + g * a.rpb * 128, &qmap, at * 64, rb * a.rpb,
-                        plane0 + g, bar);
+        for (int at = 0; at < D / 64; ++at)
+          tma_load_4d(sm + L::B_OFF + s * L::TILE + at * L::ATOM, &qmap, at * 64, rb * a.rpb, kvh * a.G, b, bar);
         bulk_load(sm + L::ST_OFF + s * kStatBytes, stats + (int64_t)rb * a.n_ksplit * kTM, kStatBytes, bar);
       },
       [&](int t, uint32_t col, int s) {
         const int64_t i0 = (int64_t)(rb_begin + t) * a.rpb;   // row index of the tile's first row per head
-        const float2* s2 = reinterpret_cast<const float2*>(sm + L::ST_OFF + s * kStatBytes) + cq * kCQ;
-        float v[kCQ];
-        tc_ld32(col + ((uint32_t)(lq * 32) << 16) + (uint32_t)(cq * kCQ), v);
+        const float2* s2 = reinterpret_cast<const float2*>(sm + L::ST_OFF + s * kStatBytes) + hf * kCH;
+        float v[kCH];
+        tc_ld64(col + ((uint32_t)(lq * 32) << 16), v);
         float sp[4] = {0.f, 0.f, 0.f, 0.f};
         if (i0 >= j0 + kTM - 1 - a.pos0) {   // every row of the tile sees every key of the block
 #pragma unroll
-          for (int e = 0; e < kCQ; ++e) {
+          for (int e = 0; e < kCH; ++e) {
             const float2 w = s2[e];
             sp[e & 3] = fmaf(ex2_approx(fmaf(v[e], a.scale_log2, w.x)), w.y, sp[e & 3]);
           }
         } else {
 #pragma unroll
-          for (int e = 0; e < kCQ; ++e) {
+          for (int e = 0; e < kCH; ++e) {
             const float2 w = s2[e];
             const float p = ex2_approx(fmaf(v[e], a.scale_log2, w.x)) * w.y;
-            if (i0 + ((cq * kCQ + e) & (a.rpb - 1)) >= jrel) sp[e & 3] += p;
+            if (i0 + ((hf * kCH + e) & (a.rpb - 1)) >= jrel) sp[e & 3] += p;
           }
         }
         acc += (sp[0] + sp[1]) + (sp[2] + sp[3]);
       });
-  // the four column quarters of each key summed
+  // the (group, half) partials of each key summed
   float* mrg = reinterpret_cast<float*>(sm + L::MRG_OFF);
   if (warp >= 2) mrg[cq * kTM + lr] = acc;
   __syncthreads();
@@ -424,16 +432,17 @@ EncodeTiled encoder() {
   return fn;
 }
 
-// fp16 [planes][rows][D] read in boxes of 64 x box_rows x 1 with the 128-byte swizzle; rows past
-// the end read as zero
-cudaError_t make_map(CUtensorMap* m, const void* base, int D, int64_t rows, int64_t planes, int box_rows) {
+// fp16 [n3][n2][rows][D] read in boxes of 64 x box_rows x box2 x 1 with the 128-byte swizzle (a box's
+// 128-byte rows land in shared memory in order: row, then dimension 2); rows past the end read as zero
+cudaError_t make_map(CUtensorMap* m, const void* base, int D, int64_t rows, int64_t n2, int64_t n3, int box_rows,
+                     int box2) {
   const EncodeTiled enc = encoder();
   if (enc == nullptr) return cudaErrorNotSupported;
-  const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)planes};
-  const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)rows * D * 2};
-  const cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
-  const cuuint32_t es[3] = {1, 1, 1};
-  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+  const cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)rows, (cuuint64_t)n2, (cuuint64_t)n3};
+  const cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)rows * D * 2, (cuuint64_t)n2 * rows * D * 2};
+  const cuuint32_t box[4] = {64, (cuuint32_t)box_rows, (cuuint32_t)box2, 1};
+  const cuuint32_t es[4] = {1, 1, 1, 1};
+  const CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
@@ -442,8 +451,8 @@ cudaError_t make_map(CUtensorMap* m, const void* base, int D, int64_t rows, int6
 template <int D>
 cudaError_t launch_scores_t(const CUtensorMap& qm, const CUtensorMap& km, const ScoreArgs& a, int units, int keyblocks,
                             cudaStream_t st) {
-  // at most two CTAs (2 x 256 of the 512 tensor-memory columns) share an SM, so no allocation waits
-  constexpr int smem = Layout<D>::ALLOC > 80 * 1024 ? Layout<D>::ALLOC : 80 * 1024;
+  // one CTA per SM (it takes all 512 tensor-memory columns), so no allocation waits
+  constexpr int smem = Layout<D>::ALLOC > 116 * 1024 ? Layout<D>::ALLOC : 116 * 1024;
   static_assert(smem <= 227 * 1024, "shared memory");
   cudaError_t e = cudaFuncSetAttribute(rowstats_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
@@ -489,8 +498,8 @@ cudaError_t launch_prefill_scores(const mkv_config& c, const void* q, int64_t q_
   a.row_st = ws.row_st;
   a.score = ws.score;
   CUtensorMap qm, km;
-  cudaError_t e = make_map(&qm, q, c.D, q_rows, (int64_t)c.B * c.Hq, a.rpb);
-  if (e == cudaSuccess) e = make_map(&km, full_k, c.D, T, units, kTN);
+  cudaError_t e = make_map(&qm, q, c.D, q_rows, c.Hq, c.B, a.rpb, a.G);   // q [B][Hq][R][D]: G heads per box
+  if (e == cudaSuccess) e = make_map(&km, full_k, c.D, T, c.Hkv, c.B, kTN, 1);   // k [B][Hkv][T][D]
   if (e != cudaSuccess) return e;
   if (c.D == 128) return launch_scores_t<128>(qm, km, a, units, (int)tiles, st);
   return launch_scores_t<64>(qm, km, a, units, (int)tiles, st);
