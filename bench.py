@@ -534,7 +534,7 @@ def tensor_peak():
     return 1900.0, "fallback"
 
 
-def measure_setup(dev, seed, reps=5, warmup=3):
+def measure_setup(dev, seed, reps=5, warmup=3, batch=None):
     """The prefill-side calls timed apart from decode, one layer each: mkv_h2o_prefill on the H2O
     workload (causal scores over the whole prompt, then the heavy + recent keep and gather) and
     mkv_snap_compress on the RocketKV workload (the observation window's scores, pooling, keep and
@@ -548,6 +548,9 @@ def measure_setup(dev, seed, reps=5, warmup=3):
     out = {}
     for name in ("h2o20", "rocket1024"):
         w = WORKLOADS[name]()
+        if batch is not None:
+            import dataclasses
+            w = dataclasses.replace(w, B=batch)
         x = synth.device_layer_inputs(w, seed, 0, device=dev, n_tokens=w.T, with_prompt_queries=True)
         kp = x["k"][:, :, :w.T].contiguous()
         vp = x["v"][:, :, :w.T].contiguous()
@@ -690,6 +693,10 @@ def main():
     ap.add_argument("--cpu-all-cores", type=int, default=1, help="1: also time the oracle on every host core")
     ap.add_argument("--setup", type=int, default=1,
                     help="1: also time the prefill-side calls (H2O prefill, SnapKV compression) on their workloads")
+    ap.add_argument("--only-setup", type=int, default=0,
+                    help="profiling: time only the prefill-side calls and print their JSON (not a bench line)")
+    ap.add_argument("--setup-batch", type=int, default=None,
+                    help="profiling: batch of the prefill-side workloads (a smaller case for ncu)")
     ap.add_argument("--profile", action="store_true",
                     help="profiling only: run warmup + steps and exit (for ncu), no JSON line")
     args = ap.parse_args()
@@ -732,6 +739,9 @@ def main():
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
+    if args.only_setup:
+        print(json.dumps({"setup": measure_setup(dev, args.seed, batch=args.setup_batch)}))
+        return
 
     total = args.warmup + args.steps
     runner = Runner(args.workload, w, dev, args.seed + rank, extra_steps=4 * total + 8)
@@ -804,7 +814,7 @@ def main():
                                                         peak, args.no_graph, synthetic_h2o_cache=True)
         line["sweep_wall_s"] = time.perf_counter() - t_sw
     if world == 1 and args.setup:
-        line["setup"] = measure_setup(dev, args.seed)
+        line["setup"] = measure_setup(dev, args.seed, batch=args.setup_batch)
     if rank == 0:
         if world == 1:
             v, sample = oracle_tokens_per_s(args.workload, w, args.cpu_budget, seed=args.seed)
