@@ -200,8 +200,9 @@ __device__ __forceinline__ void cta_teardown(Ctl<TN>* ctl, uint32_t tbase) {
 // The three roles over `ntiles` streamed tiles.  issue_a(bar) loads the held operand;
 // issue_b(t, s, bar) loads tile t into stage s; epi(t, col, s) reads the thread's half of tile t's
 // accumulator (kHalf columns from tensor-memory address col, lane 0) and, with kStats, the
-// statistics of stage s.
-template <int D, int TN, bool kStats, typename IssueA, typename IssueB, typename Epi>
+// statistics of stage s.  With kStreamA the streamed tile is the MMA's A operand and the held one its
+// B (the accumulator's lanes then follow the streamed rows).
+template <int D, int TN, bool kStats, bool kStreamA = false, typename IssueA, typename IssueB, typename Epi>
 __device__ __forceinline__ void run_roles(uint8_t* sm, Ctl<TN>* ctl, uint32_t tbase, int ntiles, IssueA issue_a,
                                           IssueB issue_b, Epi epi) {
   using L = Layout<D, TN>;
@@ -233,7 +234,11 @@ __device__ __forceinline__ void run_roles(uint8_t* sm, Ctl<TN>* ctl, uint32_t tb
           if (!role_wait(&ctl->full[s], (uint32_t)((t / kS) & 1), fail)) break;
           if (u > 0 && !role_wait(&ctl->tempty[bf], (uint32_t)((u - 1) & 1), fail)) break;
           tc_fence_after();
-          issue_tile<D, TN>(tbase + (uint32_t)(bf * TN), a_desc, b_desc + (uint64_t)((s * L::TILE_B) >> 4));
+          const uint64_t stage = b_desc + (uint64_t)((s * L::TILE_B) >> 4);
+          if (kStreamA)
+            issue_tile<D, TN>(tbase + (uint32_t)(bf * TN), stage, a_desc);
+          else
+            issue_tile<D, TN>(tbase + (uint32_t)(bf * TN), a_desc, stage);
           tc_commit(&ctl->empty[s]);
           tc_commit(&ctl->tfull[bf]);
           ctl->mma_issued = t + 1;
@@ -242,6 +247,9 @@ __device__ __forceinline__ void run_roles(uint8_t* sm, Ctl<TN>* ctl, uint32_t tb
     }
   } else {                                // epilogue warps: group (warp - 2) / 8 takes every other tile
     const int grp = (warp - 2) / kGroupWarps, half = ((warp - 2) >> 2) & 1;
+    // the held operand's phase: what came with it (statistics held beside it) is visible after it
+    const bool held = role_wait(&ctl->abar, 0, fail);
+    if (!__all_sync(0xffffffffu, held)) return;
     for (int t = grp; t < ntiles; t += 2) {
       const int s = t % kS, bf = t % kNB;
       bool ok = role_wait(&ctl->tfull[bf], (uint32_t)((t / kNB) & 1), fail);
@@ -469,6 +477,78 @@ __global__ void __launch_bounds__(kThr, 1)
   cta_teardown(ctl, tbase);
 }
 
+// ---------------------------------------------------------------- pass 2 over one query block
+// When the query rows fit one 128-row block (an observation window of at most 128 / G rows), pass 2's
+// CTAs would each meet a single tile; instead a CTA holds the query block and its statistics (the
+// MMA's B) and streams a run of 128-key tiles as the MMA's A.  Each key's sum over the block's rows
+// comes from the two column halves of the tile and is added to the zeroed score (two float adds onto
+// 0, so the result does not depend on their order).
+template <int D>
+__global__ void __launch_bounds__(kThr, 1)
+    colsum_window_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                         const ScoreArgs a, int tiles_per_cta) {
+  using L = Layout<D, kTN2>;
+  static_assert(L::ATOM_A == L::ATOM_B, "A and B tiles of 128 rows");
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = align1024(smem_raw);
+  Ctl<kTN2>* ctl = reinterpret_cast<Ctl<kTN2>*>(sm + L::CTL_OFF);
+  const int bh = (int)blockIdx.y;
+  const int b = bh / a.Hkv, kvh = bh % a.Hkv;
+  const int warp = threadIdx.x >> 5;
+  const int lq = warp & 3, cq = (warp - 2) >> 2;         // (epilogue warps) lane quarter; group x half
+  const int hf = cq & 1;                                 // column half = rows hf * 64 .. of the block
+  const int lr = lq * 32 + (threadIdx.x & 31);           // accumulator lane = key of the tile
+  const int64_t t_begin = (int64_t)blockIdx.x * tiles_per_cta;
+  const int ntiles = (int)std::max<int64_t>(0, std::min<int64_t>(ceil_div_dev(a.T, kBlk) - t_begin, tiles_per_cta));
+  const float2* stats = a.row_st + (int64_t)bh * a.n_ksplit * kTM;   // the unit's one block, split 0
+
+  const uint32_t tbase = cta_setup(ctl);
+  run_roles<D, kTN2, false, true>(
+      sm, ctl, tbase, ntiles,
+      [&](uint64_t* bar) {                // the query block and its statistics
+        tc_mbar_expect_tx(bar, L::TILE_A + kStatBytes);
+        for (int at = 0; at < D / 64; ++at)
+          tma_load_4d(sm + L::A_OFF + at * L::ATOM_A, &qmap, at * 64, 0, kvh * a.G, b, bar);
+        bulk_load(sm + L::ST_OFF, stats, kStatBytes, bar);
+      },
+      [&](int t, int s, uint64_t* bar) {  // 128 keys
+        tc_mbar_expect_tx(bar, L::TILE_B);
+        for (int at = 0; at < D / 64; ++at)
+          tma_load_4d(sm + L::B_OFF + s * L::TILE_B + at * L::ATOM_B, &kmap, at * 64, (int)((t_begin + t) * kBlk),
+                      kvh, b, bar);
+      },
+      [&](int t, uint32_t col, int) {
+        const int64_t jt = (t_begin + t) * kBlk;
+        const int64_t jrel = jt + lr - a.pos0;   // rows i >= jrel see this key
+        const float4* s4 = reinterpret_cast<const float4*>(sm + L::ST_OFF) + hf * 32;
+        const uint64_t sc2 = pk2(a.scale_log2, a.scale_log2);
+        uint64_t sp2[2] = {0ull, 0ull};
+        float v[64];
+        tc_ld64(col + ((uint32_t)(lq * 32) << 16), v);
+        if (0 >= jt + kBlk - 1 - a.pos0) {   // every row of the window sees every key of the tile
+#pragma unroll
+          for (int q = 0; q < 32; ++q) {
+            const float4 w = s4[q];
+            const float2 x = upk2(ffma2(pk2(v[2 * q], v[2 * q + 1]), sc2, pk2(w.x, w.y)));
+            sp2[q & 1] = ffma2(pk2(ex2_approx(x.x), ex2_approx(x.y)), pk2(w.z, w.w), sp2[q & 1]);
+          }
+        } else {
+#pragma unroll
+          for (int q = 0; q < 32; ++q) {
+            const float4 w = s4[q];
+            const int c = hf * 64 + 2 * q;
+            const float2 x = upk2(ffma2(pk2(v[2 * q], v[2 * q + 1]), sc2, pk2(w.x, w.y)));
+            const float p0 = (c & (a.rpb - 1)) >= jrel ? ex2_approx(x.x) * w.z : 0.f;
+            const float p1 = ((c + 1) & (a.rpb - 1)) >= jrel ? ex2_approx(x.y) * w.w : 0.f;
+            sp2[q & 1] = fadd2(sp2[q & 1], pk2(p0, p1));
+          }
+        }
+        const float2 s0 = upk2(sp2[0]), s1 = upk2(sp2[1]);
+        if (jt + lr < a.T) atomicAdd(a.score + (int64_t)bh * a.T + jt + lr, (s0.x + s0.y) + (s1.x + s1.y));
+      });
+  cta_teardown(ctl, tbase);
+}
+
 // ---------------------------------------------------------------- host side
 using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -520,6 +600,15 @@ cudaError_t launch_scores_t(const CUtensorMap& qm, const CUtensorMap& k256, cons
                                                                             a.rowblocks, a.R);
   e = cudaPeekAtLastError();
   if (e != cudaSuccess) return e;
+  if (a.rowblocks == 1) {                 // one query block: hold it, stream runs of key tiles
+    e = cudaFuncSetAttribute(colsum_window_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+    if (e == cudaSuccess) e = cudaMemsetAsync(a.score, 0, (size_t)units * a.T * sizeof(float), st);
+    if (e != cudaSuccess) return e;
+    const int64_t per = ceil_div((int64_t)keyblocks, ceil_div(kNumSMs, (int64_t)units));
+    colsum_window_kernel<D><<<dim3((unsigned)ceil_div((int64_t)keyblocks, per), units), kThr, smem2, st>>>(
+        qm, k128, a, (int)per);
+    return cudaPeekAtLastError();
+  }
   colsum_tc_kernel<D><<<dim3(keyblocks, units), kThr, smem2, st>>>(qm, k128, a);
   return cudaPeekAtLastError();
 }
