@@ -225,6 +225,15 @@ mkv_status mkv_rope_table(int32_t D, float theta, int64_t T_max, float* table, v
  * MKV_ERR_CAPACITY if any bit was set. */
 mkv_status mkv_get_status(void* stream, uint32_t* flags);
 
+/* Diagnostic of the device wait-timeout path (no counterpart in the paper):
+ * launches one CTA whose bounded mbarrier wait, the routine the prefill
+ * scoring's waits use, can never complete (nothing arrives on its barrier);
+ * after about `ms` milliseconds (1..1000, else MKV_ERR_INVALID_ARG) it gives
+ * up and sets MKV_FLAG_WAIT_TIMEOUT, so the next mkv_get_status returns
+ * MKV_ERR_TIMEOUT with that bit, and the context stays usable.  Asynchronous
+ * on `stream`; it reads and writes no caller memory. */
+mkv_status mkv_wait_timeout_selftest(int32_t ms, void* stream);
+
 /* Thread-local description of the last error (never NULL). */
 const char* mkv_last_error(void);
 

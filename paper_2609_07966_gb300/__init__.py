@@ -76,6 +76,7 @@ _SIGS = {
     "mkv_cache_bytes": [_CFG, ctypes.c_int64, ctypes.POINTER(ctypes.c_size_t), ctypes.POINTER(ctypes.c_size_t)],
     "mkv_rope_table": [ctypes.c_int32, ctypes.c_float, ctypes.c_int64, _P, _P],
     "mkv_get_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
+    "mkv_wait_timeout_selftest": [ctypes.c_int32, _P],
     "mkv_append_kv": [_CFG, _P, _P, _CACHE, _P],
     "mkv_decode_attention": [_CFG, _P, _CACHE, _QP, _P, _P, _P, ctypes.c_size_t, _P],
     "mkv_kvquant_calibrate": [_CFG, _P, _P, ctypes.c_int64, ctypes.c_int64, _QP, _P, ctypes.c_size_t, _P],
@@ -171,6 +172,11 @@ def mkv_get_status(stream=None) -> int:
     if st not in (MKV_OK, MKV_ERR_CAPACITY, MKV_ERR_TIMEOUT):
         raise MkvError(st, "mkv_get_status", mkv_last_error())
     return f.value
+
+
+def mkv_wait_timeout_selftest(ms: int, stream=None):
+    """Launch the device wait-timeout diagnostic (include/mkv.h); read the flag with mkv_get_status."""
+    _call("mkv_wait_timeout_selftest", ms, _stream(stream))
 
 
 def mkv_append_kv(cfg, k_new: int, v_new: int, cache: mkv_cache, stream=None):

@@ -309,6 +309,12 @@ mkv_status mkv_rope_table(int32_t D, float theta, int64_t T_max, float* table, v
   return MKV_OK;
 }
 
+mkv_status mkv_wait_timeout_selftest(int32_t ms, void* stream) {
+  MKV_REQUIRE(ms >= 1 && ms <= 1000, MKV_ERR_INVALID_ARG, "ms = %d outside [1, 1000]", ms);
+  MKV_CUDA(launch_wait_selftest(ms, as_stream(stream)));
+  return MKV_OK;
+}
+
 mkv_status mkv_get_status(void* stream, uint32_t* flags) {
   MKV_REQUIRE(flags != nullptr, MKV_ERR_INVALID_ARG, "flags is NULL");
   *flags = 0;

@@ -144,5 +144,6 @@ cudaError_t take_status_append(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_rocket(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_decode(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_prefill(uint32_t* flags, cudaStream_t st);
+cudaError_t launch_wait_selftest(int ms, cudaStream_t st);
 
 }  // namespace mkv

@@ -50,11 +50,19 @@ __device__ __forceinline__ bool tc_mbar_try(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait on phase `parity` of `bar`: false if it did not complete within `limit` tries.
-__device__ __forceinline__ bool tc_mbar_wait(uint64_t* bar, uint32_t parity, uint32_t limit) {
-  for (uint32_t it = 0; it < limit; ++it)
-    if (tc_mbar_try(bar, parity)) return true;
-  return false;
+// The GPU's global nanosecond clock
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Bounded wait on phase `parity` of `bar`: false if it has not completed within `ns` nanoseconds.
+__device__ __forceinline__ bool tc_mbar_wait(uint64_t* bar, uint32_t parity, uint64_t ns) {
+  if (tc_mbar_try(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (!tc_mbar_try(bar, parity))
+    if (globaltimer_ns() - t0 > ns) return false;
+  return true;
 }
 __device__ __forceinline__ void tc_mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");

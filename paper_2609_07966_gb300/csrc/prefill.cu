@@ -62,7 +62,7 @@ constexpr int kGroupWarps = 8;           // an epilogue group: four lane quarter
 constexpr int kEpiWarps = 2 * kGroupWarps;
 constexpr int kThr = (2 + kEpiWarps) * 32;
 constexpr int kStatBytes = kBlk * 8;     // one query block's (-m, 1 / l)
-constexpr uint32_t kWaitLimit = 1u << 22;
+constexpr uint64_t kWaitNs = 1000000000ull;   // a bounded wait gives up after 1 s
 
 // A streamed tile of TN rows (the MMA's N).  Pass 1 streams 256-key tiles: one MMA instruction and
 // one barrier round trip per 256 keys.  Pass 2 streams 128-row query blocks: its heavier epilogue
@@ -124,11 +124,15 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return p + ((1024u - (smem_addr(p) & 1023u)) & 1023u);
 }
 
-// Bounded wait of one role: false when it ran out (the flag is then raised) or another role did.
-__device__ __forceinline__ bool role_wait(uint64_t* bar, uint32_t parity, volatile int* fail) {
-  for (uint32_t it = 0; it < kWaitLimit; ++it) {
+// Bounded wait of one role: false when it ran out after `ns` nanoseconds (the flag is then raised
+// and MKV_FLAG_WAIT_TIMEOUT set) or another role did.
+__device__ __forceinline__ bool role_wait(uint64_t* bar, uint32_t parity, volatile int* fail, uint64_t ns = kWaitNs) {
+  if (tc_mbar_try(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
     if (tc_mbar_try(bar, parity)) return true;
     if (*fail) return false;
+    if (globaltimer_ns() - t0 > ns) break;
   }
   *fail = 1;
   atomicOr(&g_status_prefill, MKV_FLAG_WAIT_TIMEOUT);
@@ -186,10 +190,10 @@ __device__ __forceinline__ void cta_teardown(Ctl<TN>* ctl, uint32_t tbase) {
   __syncthreads();
   if (threadIdx.x == 0 && ctl->fail) {
     for (int t = std::max(0, ctl->issued - C::kS); t < ctl->issued; ++t)
-      tc_mbar_wait(&ctl->full[t % C::kS], (uint32_t)((t / C::kS) & 1), kWaitLimit);
+      tc_mbar_wait(&ctl->full[t % C::kS], (uint32_t)((t / C::kS) & 1), kWaitNs);
     if (ctl->mma_issued > 0) {
       const int t = ctl->mma_issued - 1;
-      tc_mbar_wait(&ctl->tfull[t % C::kNB], (uint32_t)((t / C::kNB) & 1), kWaitLimit);
+      tc_mbar_wait(&ctl->tfull[t % C::kNB], (uint32_t)((t / C::kNB) & 1), kWaitNs);
     }
   }
   __syncthreads();
@@ -613,7 +617,25 @@ cudaError_t launch_scores_t(const CUtensorMap& qm, const CUtensorMap& k256, cons
   return cudaPeekAtLastError();
 }
 
+// The timeout path of role_wait, exercised without a fault: an mbarrier that nothing arrives on
+__global__ void wait_selftest_kernel(uint64_t ns) {
+  __shared__ uint64_t bar;
+  __shared__ int fail;
+  if (threadIdx.x == 0) {
+    tc_mbar_init(&bar, 1);
+    tc_fence_mbar_init();
+    fail = 0;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) role_wait(&bar, 0, &fail, ns);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(int ms, cudaStream_t st) {
+  wait_selftest_kernel<<<1, 32, 0, st>>>((uint64_t)ms * 1000000ull);
+  return cudaPeekAtLastError();
+}
 
 cudaError_t launch_prefill_scores(const mkv_config& c, const void* q, int64_t q_rows, int64_t T,
                                   const void* full_k, const PrefillWs& ws, cudaStream_t st) {

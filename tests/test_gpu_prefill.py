@@ -40,3 +40,19 @@ def test_full_keep_scores_every_position(G, D, T):
             ref = h2o.prefill_scores(QP[b, h * G:(h + 1) * G], K[b, h])
             np.testing.assert_array_equal(pos[b, h, :T], np.arange(T))
             np.testing.assert_allclose(acc[b, h, :T], ref, rtol=2e-4, atol=1e-5, err_msg=f"b{b} h{h}")
+
+
+def test_wait_timeout_raises_status_and_context_survives():
+    """A bounded device wait that nothing completes (the prefill's wait routine) gives up, raises
+    MKV_FLAG_WAIT_TIMEOUT (mkv_get_status: MKV_ERR_TIMEOUT), and the next scoring call runs clean."""
+    torch = torch_cuda()
+    import time
+    assert mkv.mkv_get_status() == 0
+    t0 = time.perf_counter()
+    mkv.mkv_wait_timeout_selftest(20)
+    flags = mkv.mkv_get_status()
+    waited = time.perf_counter() - t0
+    assert flags & mkv.MKV_FLAG_WAIT_TIMEOUT
+    assert 0.015 < waited < 5.0, waited
+    assert mkv.mkv_get_status() == 0                     # the word was cleared
+    test_full_keep_scores_every_position(4, 128, 1000)  # the context is still usable
