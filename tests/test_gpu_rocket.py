@@ -143,6 +143,24 @@ def test_shapes_lockstep(G, D, fused):
                to_dev(Q, dev), dev, False, [(0, 1), (1, 0)], f"G{G}D{D}", fused)
 
 
+@pytest.mark.parametrize("G,D,W", [(8, 64, 40), (4, 128, 100), (2, 128, 130)])
+def test_window_spanning_query_blocks(G, D, W):
+    """Observation windows longer than one 128-row query block (W > 128/G): the prefill scoring's
+    column sums over several query blocks with the window's position offset (the one-block window
+    kernel does not apply), its row statistics over split key ranges; kept sets in lockstep."""
+    torch = torch_cuda()
+    dev = torch.device("cuda")
+    rng = np.random.default_rng(100 * G + W)
+    B, Hkv, T, steps = 2, 2, 1500, 3
+    Hq = G * Hkv
+    K = rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16)
+    V = rng.standard_normal((B, Hkv, T + steps, D)).astype(np.float16)
+    QW = rng.standard_normal((B, Hq, W, D)).astype(np.float16)
+    Q = rng.standard_normal((steps, B, Hq, D)).astype(np.float16)
+    run_rocket(B, Hq, Hkv, D, T, steps, W, 7, 400, 6, D // 4, to_dev(K, dev), to_dev(V, dev), to_dev(QW, dev),
+               to_dev(Q, dev), dev, False, [(0, 1), (1, 0)], f"W{W}G{G}D{D}")
+
+
 @pytest.mark.parametrize("fused", [False, True, "step"])
 def test_full_size_lockstep(fused):
     """B=4, T=32768 -> keep 4096, W=32, pool 7, top-64 pages over top-32 dims: one layer in
