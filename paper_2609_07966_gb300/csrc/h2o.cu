@@ -81,8 +81,10 @@ __global__ void h2o_gather_kernel(const __half* __restrict__ full_k, const __hal
   }
 }
 
-// One CTA per (batch, kv-head): score update and eviction.
-__global__ void __launch_bounds__(1024) h2o_update_kernel(const float* __restrict__ logits, const float* __restrict__ m_tot,
+// One CTA per (batch, kv-head): score update and eviction (1024 threads: a unit's slots in one round
+// of loads).
+constexpr int kUpdThreads = 1024;
+__global__ void __launch_bounds__(kUpdThreads) h2o_update_kernel(const float* __restrict__ logits, const float* __restrict__ m_tot,
                                                          const float* __restrict__ l_tot, int Hkv, int G, int64_t T_cap,
                                                          int H, int R, const int32_t* __restrict__ T_len,
                                                          int32_t* __restrict__ pos, float* __restrict__ acc,
@@ -110,7 +112,7 @@ cudaError_t launch_h2o_keep(const mkv_config& c, const void* full_k, const void*
 }
 
 cudaError_t launch_h2o_update(const mkv_config& c, const mkv_cache& cache, const DecodeWs& ws, cudaStream_t st) {
-  return launch_pdl(h2o_update_kernel, dim3(c.B * c.Hkv), dim3(1024), 0, st, (const float*)ws.logits,
+  return launch_pdl(h2o_update_kernel, dim3(c.B * c.Hkv), dim3(kUpdThreads), 0, st, (const float*)ws.logits,
                     (const float*)ws.m_tot, (const float*)ws.l_tot, c.Hkv, c.Hq / c.Hkv, cache.T_cap, c.h2o_heavy,
                     c.h2o_recent, (const int32_t*)cache.T_len, cache.pos, cache.acc, cache.slot);
 }

@@ -5,13 +5,20 @@
 // under (acc desc, position asc) among all but the `recent` newest positions is
 // evicted and its slot becomes the next append slot; otherwise the first free
 // slot is.  Logits are read with L2-coherent loads (the decode CTAs of the
-// unit wrote them).
+// unit wrote them).  The group's (m, 1 / l) are read once per CTA; 2^x comes from the
+// special-function unit's approximation (relative error about 2^-22).
 #pragma once
 
 #include "mkv_common.cuh"
 #include "mkv_select.cuh"
 
 namespace mkv {
+
+__device__ __forceinline__ float h2o_ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits, const float* __restrict__ m_tot,
                                                 const float* __restrict__ l_tot, int Hkv, int G, int64_t T_cap,
@@ -20,17 +27,19 @@ __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits
                                                 int32_t* __restrict__ slot_out, int64_t bh) {
   const int b = (int)(bh / Hkv), kvh = (int)(bh % Hkv);
   const int64_t newest = (int64_t)T_len[b] - 1;
+  __shared__ float s_m[8], s_il[8];
+  if (threadIdx.x < G) {
+    const int64_t hq = (int64_t)b * Hkv * G + (int64_t)kvh * G + threadIdx.x;
+    s_m[threadIdx.x] = __ldcg(m_tot + hq);
+    const float l = __ldcg(l_tot + hq);
+    s_il[threadIdx.x] = l > 0.f ? 1.f / l : 0.f;
+  }
+  __syncthreads();
   float m[8], il[8];                  // G <= 8; unrolled so both stay in registers
 #pragma unroll
   for (int h = 0; h < 8; ++h) {
-    m[h] = 0.f;
-    il[h] = 0.f;
-    if (h < G) {
-      const int64_t hq = (int64_t)b * Hkv * G + (int64_t)kvh * G + h;
-      m[h] = __ldcg(m_tot + hq);
-      const float l = __ldcg(l_tot + hq);
-      il[h] = l > 0.f ? 1.f / l : 0.f;
-    }
+    m[h] = h < G ? s_m[h] : 0.f;
+    il[h] = h < G ? s_il[h] : 0.f;
   }
   int held = 0;
   uint64_t best = ~0ull;          // minimum key among candidates -> evicted
@@ -53,12 +62,12 @@ __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits
         const float* lg = logits + (bh * T_cap + s) * G;
         if (G == 4) {
           const float4 x = __ldcg(reinterpret_cast<const float4*>(lg));
-          add[u] = exp2f(x.x - m[0]) * il[0] + exp2f(x.y - m[1]) * il[1] + exp2f(x.z - m[2]) * il[2] +
-                   exp2f(x.w - m[3]) * il[3];
+          add[u] = h2o_ex2(x.x - m[0]) * il[0] + h2o_ex2(x.y - m[1]) * il[1] + h2o_ex2(x.z - m[2]) * il[2] +
+                   h2o_ex2(x.w - m[3]) * il[3];
         } else {
 #pragma unroll
           for (int h = 0; h < 8; ++h)
-            if (h < G) add[u] += exp2f(__ldcg(lg + h) - m[h]) * il[h];
+            if (h < G) add[u] += h2o_ex2(__ldcg(lg + h) - m[h]) * il[h];
         }
       }
     }
