@@ -35,7 +35,7 @@ __global__ void __launch_bounds__(kSelThreads) h2o_keep_kernel(const float* __re
   const int heavy = (int)(n_cand < (int64_t)H ? n_cand : (int64_t)H);
   uint64_t thr = ~0ull;
   if (heavy > 0) {
-    thr = block_kth_largest((int)n_cand, heavy, [&](int i) { return rank_key(s[i], (uint32_t)i); }, hist);
+    thr = block_kth_largest_score((int)n_cand, heavy, [&](int i) { return s[i]; }, hist);
   }
   // stream compaction in ascending position
   int64_t base = 0;

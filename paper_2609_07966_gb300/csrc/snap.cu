@@ -30,23 +30,27 @@ __device__ __forceinline__ float pooled_at(const float* s, int64_t n, int64_t j,
   return m;
 }
 
-// One CTA per (batch, kv-head): keep list (ascending) of the compressed cache.
+constexpr int kPooledSmem = 51200;      // pooled scores kept in shared memory up to this many positions
+
+// One CTA per (batch, kv-head): keep list (ascending) of the compressed cache.  The pooled scores
+// live in shared memory when they fit (dynamic, n floats), else in the workspace.
 __global__ void __launch_bounds__(kSelThreads) snap_keep_kernel(const float* __restrict__ score, int64_t T, int W,
                                                                 int pool, int keep, float* __restrict__ pooled_ws,
                                                                 int32_t* __restrict__ keep_out) {
   __shared__ int hist[256];
   __shared__ int warp_sums[32];
+  extern __shared__ float pooled_sm[];
   const int64_t bh = blockIdx.x;
   const int64_t n = T - W;                        // prefix positions compete
   const float* s = score + bh * T;
-  float* pooled = pooled_ws + bh * T;
+  float* pooled = n <= kPooledSmem ? pooled_sm : pooled_ws + bh * T;
   int32_t* out = keep_out + bh * T;
   const int r = pool / 2;
   for (int64_t j = threadIdx.x; j < n; j += blockDim.x) pooled[j] = pooled_at(s, n, j, r);
   __syncthreads();
   const int k = keep - W;
   uint64_t thr = ~0ull;
-  if (k > 0) thr = block_kth_largest((int)n, k, [&](int i) { return rank_key(pooled[i], (uint32_t)i); }, hist);
+  if (k > 0) thr = block_kth_largest_score((int)n, k, [&](int i) { return pooled[i]; }, hist);
   int64_t base = 0;
   for (int64_t i0 = 0; i0 < T; i0 += blockDim.x) {
     const int64_t i = i0 + threadIdx.x;
@@ -255,7 +259,7 @@ __global__ void __launch_bounds__(kSelThreads) rocket_select_kernel(const __half
     base = total;
   } else {
     uint64_t thr = ~0ull;
-    if (k > 0) thr = block_kth_largest(ns, k, [&](int i) { return rank_key(ssc[i], (uint32_t)i); }, hist);
+    if (k > 0) thr = block_kth_largest_score(ns, k, [&](int i) { return ssc[i]; }, hist);
     for (int i0 = 0; i0 < ns; i0 += blockDim.x) {
       const int i = i0 + threadIdx.x;
       const int flag = (i < ns && k > 0 && rank_key(ssc[i], (uint32_t)i) >= thr) ? 1 : 0;
@@ -276,7 +280,11 @@ cudaError_t launch_snap_keep(const mkv_config& c, const void* full_k, const void
   const bool identity = T <= c.snap_keep;
   const int64_t n = identity ? T : c.snap_keep;
   if (!identity) {
-    snap_keep_kernel<<<units, kSelThreads, 0, st>>>(ws.score, T, c.snap_window, c.snap_pool, c.snap_keep,
+    const int64_t n_pre = T - c.snap_window;
+    const int smem = n_pre <= kPooledSmem ? (int)(n_pre * sizeof(float)) : 0;
+    cudaError_t ea = cudaFuncSetAttribute(snap_keep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (ea != cudaSuccess) return ea;
+    snap_keep_kernel<<<units, kSelThreads, smem, st>>>(ws.score, T, c.snap_window, c.snap_pool, c.snap_keep,
                                                     reinterpret_cast<float*>(ws.row_st),
                                                     ws.keep);
     cudaError_t e = cudaPeekAtLastError();
