@@ -10,12 +10,10 @@
 
 namespace mkv {
 
-// Operand tile layout (K-major, 128-byte swizzle): a row's K extent is cut into atoms of 64 fp16
-// (128 B); an atom of R rows is R * 128 B, rows in 8-row groups of 1024 B, and the 16-byte chunk c
-// of row r sits at chunk c ^ (r % 8).  Atoms start 1024-byte aligned.
-__host__ __device__ __forceinline__ uint32_t sw128_off(int row, int c) {
-  return (uint32_t)((row >> 3) * 1024 + (row & 7) * 128 + ((c ^ (row & 7)) << 4));
-}
+// Operand tile layout (K-major, 128-byte swizzle, as TMA writes it with the 128-byte swizzle mode
+// into a 1024-byte aligned destination): a row's K extent is cut into atoms of 64 fp16 (128 B); an
+// atom of R rows is R * 128 B, rows in 8-row groups of 1024 B, and the 16-byte chunk c of row r sits
+// at chunk c ^ (r % 8).
 
 // Shared-memory matrix descriptor of such a tile starting at shared address `start`: start >> 4 in
 // bits [0,14), leading byte offset >> 4 in [16,30) (unused by swizzled K-major tiles), stride byte
@@ -72,16 +70,9 @@ __device__ __forceinline__ void tc_mbar_expect_tx(uint64_t* bar, uint32_t bytes)
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
                : "memory");
 }
-// TMA: the box at coordinates (x, y, z) of the tensor map at generic address `map` into shared
-// memory at `dst`, completing `bytes` of `bar`'s transaction count (x * element size must be a
+// TMA: the box at coordinates (x, y, z, w) of the tensor map at generic address `map` into shared
+// memory at `dst`, completing its bytes of `bar`'s transaction count (x * element size must be a
 // multiple of 16 bytes; rows outside the tensor are zero-filled)
-__device__ __forceinline__ void tma_load_3d(void* dst, const void* map, int x, int y, int z, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::
-          "r"(smem_addr(dst)),
-      "l"(map), "r"(x), "r"(y), "r"(z), "r"(smem_addr(bar))
-      : "memory");
-}
 __device__ __forceinline__ void tma_load_4d(void* dst, const void* map, int x, int y, int z, int w, uint64_t* bar) {
   asm volatile(
       "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];" ::
@@ -120,13 +111,11 @@ __device__ __forceinline__ void tc_commit(uint64_t* bar) {
 }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-// generic-proxy writes to shared memory made visible to the tensor core's (async-proxy) reads
-__device__ __forceinline__ void tc_fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_mbar_init() {
   asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
 // 32 TMEM lanes x 16 consecutive fp32 columns: thread i of the warp gets lane (address lane + i).
-// The registers are valid only after tc_wait_ld().
+// The registers are valid only after a tcgen05.wait::ld (tc_wait_ld_regs).
 __device__ __forceinline__ void tc_ld16_issue(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
@@ -134,34 +123,9 @@ __device__ __forceinline__ void tc_ld16_issue(uint32_t taddr, uint32_t (&r)[16])
         "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
 }
-__device__ __forceinline__ void tc_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-
-// 32 consecutive fp32 columns (two loads in flight, one wait)
-__device__ __forceinline__ void tc_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r0[16], r1[16];
-  tc_ld16_issue(taddr, r0);
-  tc_ld16_issue(taddr + 16, r1);
-  tc_wait_ld();
-#pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    v[i] = __uint_as_float(r0[i]);
-    v[16 + i] = __uint_as_float(r1[i]);
-  }
-}
-
-// 32 consecutive fp32 columns into r without waiting; tc_wait_ld32(r) then makes them readable.
-// The wait names the registers, so the compiler orders every use of r after it.
-__device__ __forceinline__ void tc_ld32_issue(uint32_t taddr, uint32_t (&r)[32]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-}
-__device__ __forceinline__ void tc_wait_ld32(uint32_t (&r)[32]) {
+// Wait for this thread's tensor-memory loads.  The wait names the 32 loaded registers of r, so
+// the compiler orders every use of them after it (a second wait, already satisfied, covers more).
+__device__ __forceinline__ void tc_wait_ld_regs(uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
                : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
                  "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
@@ -172,16 +136,20 @@ __device__ __forceinline__ void tc_wait_ld32(uint32_t (&r)[32]) {
                : "memory");
 }
 
-// 64 consecutive fp32 columns (four loads in flight, one wait)
+// 64 consecutive fp32 columns (four loads in flight, then the wait)
 __device__ __forceinline__ void tc_ld64(uint32_t taddr, float (&v)[64]) {
-  uint32_t r[4][16];
+  uint32_t r0[32], r1[32];
+  tc_ld16_issue(taddr, *reinterpret_cast<uint32_t(*)[16]>(&r0[0]));
+  tc_ld16_issue(taddr + 16, *reinterpret_cast<uint32_t(*)[16]>(&r0[16]));
+  tc_ld16_issue(taddr + 32, *reinterpret_cast<uint32_t(*)[16]>(&r1[0]));
+  tc_ld16_issue(taddr + 48, *reinterpret_cast<uint32_t(*)[16]>(&r1[16]));
+  tc_wait_ld_regs(r0);
+  tc_wait_ld_regs(r1);
 #pragma unroll
-  for (int k = 0; k < 4; ++k) tc_ld16_issue(taddr + 16 * k, r[k]);
-  tc_wait_ld();
-#pragma unroll
-  for (int k = 0; k < 4; ++k)
-#pragma unroll
-    for (int i = 0; i < 16; ++i) v[16 * k + i] = __uint_as_float(r[k][i]);
+  for (int i = 0; i < 32; ++i) {
+    v[i] = __uint_as_float(r0[i]);
+    v[32 + i] = __uint_as_float(r1[i]);
+  }
 }
 
 // Packed fp32 pairs (Blackwell): each lane of fma.rn.f32x2 / add.rn.f32x2 rounds as its scalar form
