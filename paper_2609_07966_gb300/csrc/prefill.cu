@@ -6,32 +6,33 @@
 // -- SnapKV: the W rows of the observation window (p_i = T - W + i).
 //
 // Two passes on the 5th-generation tensor cores (tcgen05.mma kind::f16: fp16 operands, fp32
-// accumulator in tensor memory), each a stream of 128 x 256 x D tile products with a softmax
-// epilogue:
+// accumulator in tensor memory), each a stream of 128 x N x D tile products with a softmax epilogue:
 //   pass 1 (rows): a CTA holds 128 query rows (the group's G heads, 128 / G rows each) and streams
-//           256-key tiles; it keeps per row the running max m and sum l of 2^(s - m) over the
-//           causal keys.  When the rows are few (an observation window) the key range is split
-//           across CTAs; a small kernel merges the splits into (-m, 1 / l) per row, laid out in the
-//           order of pass 2's query blocks;
-//   pass 2 (columns): a CTA holds 128 keys and streams the query rows that can see them, two
-//           128-row blocks per tile, summing 2^(s - m_i) / l_i over the rows with p_i >= j per key j.
-// The held operand is the MMA's A (M = 128 lanes of the accumulator), a streamed tile its B
-// (N = 256 columns: at this width one MMA instruction and one barrier round trip serve twice the
-// work of a 128-wide tile).  Each CTA is warp-specialised:
+//           256-key tiles (N = 256: one MMA instruction and one barrier round trip per 256 keys); it
+//           keeps per row the running max m and sum l of 2^(s - m) over the causal keys.  When the
+//           rows are few (an observation window) the key range is split across CTAs; a small kernel
+//           merges the splits into (-m, 1 / l) per row, laid out in the order of pass 2's query blocks;
+//   pass 2 (columns): a CTA holds 128 keys and streams the 128-row query blocks that can see them
+//           (N = 128, four accumulator buffers: its epilogue is the heavier one), summing
+//           2^(s - m_i) / l_i over the rows with p_i >= j for each key j;
+//   pass 2 over one query block (colsum_window_kernel): when the window's rows fit one block, a
+//           CTA holds that block and streams a run of 128-key tiles instead.
+// The held operand is the MMA's A (M = 128 lanes of the accumulator), a streamed tile its B (the
+// window kernel swaps them).  Each CTA is warp-specialised, one per SM (all 512 tensor-memory
+// columns):
 //   warp 0 (one thread) loads operand tiles by TMA (tensor maps with the 128-byte swizzle, the
-//           K-major layout the MMA reads) into a ring of kS stages, and in pass 2 each query block's
+//           K-major layout the MMA reads) into a ring of stages, and in pass 2 each query block's
 //           128 row statistics by a bulk copy beside it;
-//   warp 1 (one thread) issues the D / 16 MMAs of tile t into tensor-memory accumulator buffer
-//           t % 2 (2 x 256 columns: all of tensor memory, one CTA per SM), then commits to the
-//           stage's and the buffer's mbarriers;
+//   warp 1 (one thread) issues the D / 16 MMAs of tile t into accumulator buffer t % (buffers),
+//           then commits to the stage's and the buffer's mbarriers;
 //   warps 2..17 read finished accumulators in two groups of eight: group g takes the tiles
-//           t = g mod 2 (so buffer g), and the groups work a tile apart, one group's exponentials
-//           overlapping the other's loads and reductions; warp w reads lanes 32 (w % 4) .. + 31
-//           (the lane quarter it may access) and one half of the 256 columns, 64 at a time.
+//           t = g mod 2, so the groups work a tile apart and one group's exponentials overlap the
+//           other's loads and reductions; warp w reads lanes 32 (w % 4) .. + 31 (the lane quarter it
+//           may access) and one half of the tile's columns, 64 at a time.
 // Loads, products and epilogues of different tiles overlap; nothing in the tile loop waits on a
-// CTA-wide barrier.  Every wait is bounded: on a timeout the role raises MKV_FLAG_WAIT_TIMEOUT and
-// sets a flag that ends the other roles' waits; the CTA then waits (bounded) for the copies and
-// products it already issued and still frees its tensor memory.
+// CTA-wide barrier.  Every wait is bounded (1 s of the GPU's global timer): on a timeout the role
+// raises MKV_FLAG_WAIT_TIMEOUT and sets a flag that ends the other roles' waits; the CTA then waits
+// (bounded) for the copies and products it already issued and still frees its tensor memory.
 #include <cuda.h>   // CUtensorMap and its enums; the encoder is fetched from the driver at run time
 #include <math.h>
 
