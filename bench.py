@@ -534,6 +534,14 @@ def tensor_peak():
     return 1900.0, "fallback"
 
 
+def prefill_scoring_flops(B: int, Hq: int, D: int, T: int, rows: int) -> float:
+    """FLOPs of the prefill scoring for `rows` query rows at positions T - rows .. T - 1 over T keys:
+    2 products (row statistics, then column sums) x 2 D per causal (row, key) pair per query head."""
+    W = rows
+    pairs = W * (T - W) + W * (W + 1) / 2          # row i (position T - W + i) sees T - W + i + 1 keys
+    return 2 * 2 * D * pairs * B * Hq
+
+
 def measure_setup(dev, seed, reps=5, warmup=3, batch=None):
     """The prefill-side calls timed apart from decode, one layer each: mkv_h2o_prefill on the H2O
     workload (causal scores over the whole prompt, then the heavy + recent keep and gather) and
@@ -558,7 +566,7 @@ def measure_setup(dev, seed, reps=5, warmup=3, batch=None):
             cfg = mkv.config(mkv.MKV_H2O, w.B, w.Hq, w.Hkv, w.D, h2o_heavy=w.h2o_heavy, h2o_recent=w.h2o_recent)
             T_cap = w.h2o_heavy + w.h2o_recent + 1
             qp = x["q_prompt"].contiguous()
-            rows, pairs = w.T, w.T * (w.T + 1) / 2
+            rows = w.T
             call = "mkv_h2o_prefill"
         else:
             cfg = mkv.config(mkv.MKV_ROCKET, w.B, w.Hq, w.Hkv, w.D, snap_window=w.snap_window,
@@ -566,8 +574,7 @@ def measure_setup(dev, seed, reps=5, warmup=3, batch=None):
                              topk_pages=w.topk_pages, topq_dims=w.topq_dims)
             T_cap = (min(w.T, w.snap_keep) + 15) // 16 * 16
             qp = x["q_prompt"][:, :, w.T - w.snap_window:].contiguous()
-            W = w.snap_window
-            rows, pairs = W, W * (w.T - W) + W * (W + 1) / 2
+            rows = w.snap_window
             call = "mkv_snap_compress"
         del x
         cache = caches.alloc_cache(cfg, T_cap, device=dev)
@@ -589,7 +596,7 @@ def measure_setup(dev, seed, reps=5, warmup=3, batch=None):
             b.record(st)
         torch.cuda.synchronize()
         ms = statistics.median(a.elapsed_time(b) for a, b in ev)
-        flops = 2 * 2 * w.D * pairs * w.B * w.Hq
+        flops = prefill_scoring_flops(w.B, w.Hq, w.D, w.T, rows)
         tf = flops / (ms * 1e-3) / 1e12
         out[name] = {"call": call, "workload": f"{w.name}, one layer", "batch": w.B, "context": w.T,
                      "query_rows": rows, "ms": ms, "status": mkv.mkv_get_status(),

@@ -36,3 +36,13 @@ def test_committed_traffic_record_is_well_formed():
         assert os.path.exists(os.path.join(bench.ROOT, e["summary"]))
         assert e["dram_bytes_read"] > 0 and e["dram_bytes_write"] >= 0
         assert len(e["source_sha256"]) == 64
+
+
+def test_prefill_scoring_flops_counts_causal_pairs():
+    """The setup roofline's FLOPs: 2 products x 2 D per causal (query row, key) pair per query head,
+    against a brute-force count of the visible pairs (H2O: every row; SnapKV: a window)."""
+    import bench
+    for (B, Hq, D, T, rows) in [(1, 1, 64, 7, 7), (2, 4, 128, 50, 50), (1, 2, 64, 40, 8), (3, 8, 128, 33, 1)]:
+        pos0 = T - rows
+        pairs = sum(1 for i in range(rows) for j in range(T) if j <= pos0 + i)
+        assert bench.prefill_scoring_flops(B, Hq, D, T, rows) == 2 * 2 * D * pairs * B * Hq
