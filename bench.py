@@ -138,6 +138,16 @@ class Runner:
         self.q, self.kn, self.vn, self.out, self.pidx = [], [], [], [], []
         # prefill-side calls need workspace for the whole prompt
         self.ws, self.nws = caches.workspace(self.cfg, max(self.T_cap, w.T), device=dev)
+        if self.method == "h2o":
+            # layer l's score update reads the logits its decode left in the workspace, and nothing of
+            # layer l + 1 depends on it: it runs on a side stream while the next layer decodes, the
+            # layers alternating between two workspaces (a decode first waits for the last update
+            # that read its workspace)
+            self.ws_alt, _ = caches.workspace(self.cfg, max(self.T_cap, w.T), device=dev)
+            self.side = torch.cuda.Stream(device=dev)
+            self.overlap = True                 # False: the updates in line on the main stream
+            self.dec_ev = [torch.cuda.Event() for _ in range(2)]
+            self.upd_ev = [torch.cuda.Event() for _ in range(2)]
         if self.method == "kvquant":
             self.rope = torch.empty((self.T_cap, D // 2, 2), dtype=torch.float32, device=dev)
             mkv.mkv_rope_table(D, w.theta, self.T_cap, self.rope.data_ptr())
@@ -269,6 +279,11 @@ class Runner:
             out = self.out[l] if out is None else out
             mkv.mkv_rocket_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, 0, out.data_ptr())
             return
+        torch = self.torch
+        ws = self.ws if self.method != "h2o" or l % 2 == 0 else self.ws_alt
+        if self.method == "h2o" and self.overlap and l >= 2:
+            # (layers 0 and 1 follow the previous step's updates, joined at its end)
+            torch.cuda.current_stream().wait_event(self.upd_ev[l % 2])
         if self.method in ("fp16", "h2o") and self.step_fused:
             # append and attention in one launch, then (H2O) the update
             kn = self.kn[l] if kn is None else kn
@@ -277,24 +292,40 @@ class Runner:
             out = self.out[l] if out is None else out
             try:
                 mkv.mkv_decode_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, out.data_ptr(),
-                                    self.ws.data_ptr(), self.nws)
+                                    ws.data_ptr(), self.nws)
             except mkv.MkvError as e:
                 # too many splits for the step's ticket counter: nothing was launched; two calls instead
                 if e.status != mkv.MKV_ERR_UNSUPPORTED:
                     raise
                 self.step_fused = False
                 return self.layer_step(l, q, kn, vn, out)
+        else:
+            self.append(l, kn, vn)
             if self.method == "h2o":
-                mkv.mkv_h2o_update(self.cfg, cache.c, self.ws.data_ptr(), self.nws)
-            return
-        self.append(l, kn, vn)
-        self.decode(l, q, out)
-        if self.method == "h2o":
-            mkv.mkv_h2o_update(self.cfg, cache.c, self.ws.data_ptr(), self.nws)
+                q = self.q[l] if q is None else q
+                out = self.out[l] if out is None else out
+                mkv.mkv_decode_attention(self.cfg, q.data_ptr(), cache.c, None, 0, out.data_ptr(), ws.data_ptr(),
+                                         self.nws)
+            else:
+                self.decode(l, q, out)
+        if self.method == "h2o" and self.overlap:   # the update on the side stream, after this decode
+            main = torch.cuda.current_stream()
+            self.dec_ev[l % 2].record(main)
+            self.side.wait_event(self.dec_ev[l % 2])
+            mkv.mkv_h2o_update(self.cfg, cache.c, ws.data_ptr(), self.nws, stream=self.side.cuda_stream)
+            self.upd_ev[l % 2].record(self.side)
+        elif self.method == "h2o":
+            mkv.mkv_h2o_update(self.cfg, cache.c, ws.data_ptr(), self.nws)
+
+    def join_side(self):
+        """The main stream waits for the side stream's score updates (end of a step)."""
+        if self.method == "h2o" and self.overlap:
+            self.torch.cuda.current_stream().wait_stream(self.side)
 
     def step(self):
         for l in range(self.w.L):
             self.layer_step(l)
+        self.join_side()
 
     def capture(self):
         torch = self.torch
@@ -419,6 +450,7 @@ def time_e2e(runner, steps, warmup):
         d_in.copy_(h_in, non_blocking=True)
         for l in range(w.L):
             runner.layer_step(l, views[3 * l], views[3 * l + 1], views[3 * l + 2], outs[l])
+        runner.join_side()
         h_out.copy_(d_out, non_blocking=True)
 
     for _ in range(warmup):
