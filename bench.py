@@ -236,6 +236,28 @@ class Runner:
                 t_split = time_decode_launches(self, 3)
                 self.rocket_fused = t_fused <= t_split
 
+    def choose_kvquant_step(self, reps=3):
+        """KVQuant: the one-launch step (mkv_kvquant_step) or quantize + decode, whichever is faster on
+        this shape (both leave the same cache and output bits); a few eager steps of each, timed with
+        CUDA events.  Returns both times (ms per step)."""
+        torch = self.torch
+        t = {}
+        for fused in (True, False):
+            self.step_fused = fused
+            self.step()
+            torch.cuda.synchronize()
+            st = torch.cuda.current_stream()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            for _ in range(reps):
+                self.step()
+            e1.record(st)
+            torch.cuda.synchronize()
+            t[fused] = e0.elapsed_time(e1) / reps
+        self.step_fused = t[True] <= t[False]
+        return {"one_launch_step": t[True], "quantize_then_decode": t[False],
+                "chosen": "one_launch_step" if self.step_fused else "quantize_then_decode"}
+
     def append(self, l, kn=None, vn=None):
         mkv = self.mkv
         cache, qp = self.layers[l]
@@ -284,15 +306,19 @@ class Runner:
         if self.method == "h2o" and self.overlap and l >= 2:
             # (layers 0 and 1 follow the previous step's updates, joined at its end)
             torch.cuda.current_stream().wait_event(self.upd_ev[l % 2])
-        if self.method in ("fp16", "h2o") and self.step_fused:
-            # append and attention in one launch, then (H2O) the update
+        if self.method in ("fp16", "h2o", "kvquant") and self.step_fused:
+            # append (KVQuant: quantize) and attention in one launch, then (H2O) the update
             kn = self.kn[l] if kn is None else kn
             vn = self.vn[l] if vn is None else vn
             q = self.q[l] if q is None else q
             out = self.out[l] if out is None else out
             try:
-                mkv.mkv_decode_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c, out.data_ptr(),
-                                    ws.data_ptr(), self.nws)
+                if self.method == "kvquant":
+                    mkv.mkv_kvquant_step(self.cfg, self.layers[l][1].c, q.data_ptr(), kn.data_ptr(), vn.data_ptr(),
+                                         cache.c, out.data_ptr(), ws.data_ptr(), self.nws)
+                else:
+                    mkv.mkv_decode_step(self.cfg, q.data_ptr(), kn.data_ptr(), vn.data_ptr(), cache.c,
+                                        out.data_ptr(), ws.data_ptr(), self.nws)
             except mkv.MkvError as e:
                 # too many splits for the step's ticket counter: nothing was launched; two calls instead
                 if e.status != mkv.MKV_ERR_UNSUPPORTED:
@@ -347,10 +373,10 @@ class Runner:
             self.step()
 
     def launches_per_step(self):
-        # per layer: FP16 / H2O append and attention in one launch (H2O: + score update); KVQuant
-        # quantize (which also stores the new length) + decode; RocketKV append, page choice and
-        # attention in one launch
-        per = {"fp16": 1 if self.step_fused else 2, "kvquant": 2, "h2o": 2 if self.step_fused else 3,
+        # per layer: FP16 / H2O / KVQuant append (KVQuant: quantize) and attention in one launch (H2O:
+        # + score update); RocketKV append, page choice and attention in one launch
+        per = {"fp16": 1 if self.step_fused else 2, "kvquant": 1 if self.step_fused else 2,
+               "h2o": 2 if self.step_fused else 3,
                "rocket": 1 if self.rocket_fused else 3}[self.method]
         return per * self.w.L
 
@@ -533,6 +559,7 @@ def measure_config(name, w, dev, seed, method, steps, warmup, peak, no_graph=Fal
     import torch
     rx = Runner(name, w, dev, seed, extra_steps=4 * (steps + warmup) + 8, method=method,
                 synthetic_h2o_cache=synthetic_h2o_cache)
+    paths = rx.choose_kvquant_step() if rx.method == "kvquant" else None
     if not no_graph:
         rx.capture()
     msx = time_steps(rx, steps, warmup)
@@ -547,6 +574,8 @@ def measure_config(name, w, dev, seed, method, steps, warmup, peak, no_graph=Fal
            "gpu_launches_per_step": rx.launches_per_step()}
     if rx.method == "h2o" and synthetic_h2o_cache:
         row["note"] = "decode cache filled directly with the budget's heavy + recent slots (no prefill scoring)"
+    if paths is not None:
+        row["step_paths_ms"] = paths
     if rx.method in ("fp16", "h2o") and not rx.step_fused:
         row["note"] = "append and attention as two launches (too many splits for the one-launch step)"
     if rx.method == "rocket" and not rx.rocket_fused:
@@ -784,6 +813,7 @@ def main():
 
     total = args.warmup + args.steps
     runner = Runner(args.workload, w, dev, args.seed + rank, extra_steps=4 * total + 8)
+    step_paths = runner.choose_kvquant_step() if runner.method == "kvquant" else None
     if not args.no_graph:
         runner.capture()
     if args.profile:
@@ -828,6 +858,8 @@ def main():
                          "avg_launch_ms": dec_ms},
             "kv_bytes": {"resident": res * w.L, "peak": pk * w.L, "unit": "bytes, all layers"},
             "clocks": clk}
+    if step_paths is not None:
+        line["step_paths_ms"] = step_paths     # the faster path is the timed one
     del runner
     torch.cuda.empty_cache()
     if world == 1 and args.per_config:

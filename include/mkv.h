@@ -421,6 +421,26 @@ mkv_status mkv_rocket_decode(const mkv_config* cfg, const void* q, const mkv_cac
 mkv_status mkv_decode_step(const mkv_config* cfg, const void* q, const void* k_new, const void* v_new,
                            mkv_cache* cache, void* out, void* ws, size_t ws_bytes, void* stream);
 
+/* A whole KVQuant decode step in one launch: mkv_quantize_kv of the step's
+ * token (n_tokens = 1) followed by mkv_decode_attention, with the same cache
+ * contents (codes, key-outlier CSR, value outliers and ranges, T_len) and the
+ * same output bits (Section 2.1, KVQuant paragraph: the token's key is
+ * quantized per channel before the rotary embedding, its value per token,
+ * with fp16 outliers).  k_new fp16 [B][Hkv][D] is the token's pre-rotation
+ * key, v_new fp16 [B][Hkv][D] its value; q, out, qparams, ws as
+ * mkv_decode_attention.  The decode CTA whose range holds a unit's new token
+ * quantizes it before it stages that chunk.  While the launch runs, the top 8
+ * bits of T_len[b] count the CTAs that read it (the last one stores the new
+ * length), so nothing else may read or write T_len of this cache during the
+ * call.  A batch entry whose cache is full is not appended
+ * (MKV_FLAG_CACHE_FULL) and attends to its existing tokens; key-outlier
+ * entries beyond k_out_cap raise MKV_FLAG_K_OUTLIER_OVERFLOW as in
+ * mkv_quantize_kv (both read by mkv_get_status).  MKV_ERR_UNSUPPORTED when
+ * T_cap >= 2^24: use the two calls then. */
+mkv_status mkv_kvquant_step(const mkv_config* cfg, const mkv_quant_params* qparams, const void* q,
+                            const void* k_new, const void* v_new, mkv_cache* cache, void* out, void* ws,
+                            size_t ws_bytes, void* stream);
+
 /* A whole RocketKV decode step in one launch: mkv_append_kv of the step's
  * token followed by mkv_rocket_decode, with the same cache contents, page
  * choice and output.  k_new, v_new fp16 [B][Hkv][D] (post-rotation keys),

@@ -89,6 +89,7 @@ _SIGS = {
     "mkv_rocket_decode": [_CFG, _P, _CACHE, _P, _P, _P],
     "mkv_rocket_step": [_CFG, _P, _P, _P, _CACHE, _P, _P, _P],
     "mkv_decode_step": [_CFG, _P, _P, _P, _CACHE, _P, _P, ctypes.c_size_t, _P],
+    "mkv_kvquant_step": [_CFG, _QP, _P, _P, _P, _CACHE, _P, _P, ctypes.c_size_t, _P],
     "mkv_select_config": [ctypes.POINTER(mkv_candidate), ctypes.c_int32, ctypes.c_double, ctypes.c_double,
                           ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int32)],
     "mkv_decode_attention_noalloc": [_CFG, _P, _CACHE, _P, _P],
@@ -238,6 +239,12 @@ def mkv_decode_step(cfg, q: int, k_new: int, v_new: int, cache: mkv_cache, out: 
                     stream=None):
     _call("mkv_decode_step", ctypes.byref(cfg), q, k_new, v_new, ctypes.byref(cache), out, ws, ws_bytes,
           _stream(stream))
+
+
+def mkv_kvquant_step(cfg, qparams, q: int, k_new: int, v_new: int, cache: mkv_cache, out: int, ws: int,
+                     ws_bytes: int, stream=None):
+    _call("mkv_kvquant_step", ctypes.byref(cfg), ctypes.byref(qparams), q, k_new, v_new, ctypes.byref(cache), out,
+          ws, ws_bytes, _stream(stream))
 
 
 def mkv_rocket_step(cfg, q: int, k_new: int, v_new: int, cache: mkv_cache, page_idx_out, out: int, stream=None):

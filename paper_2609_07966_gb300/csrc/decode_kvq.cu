@@ -36,11 +36,20 @@
 // online softmax, and O^T (dims x heads) += V^T P^T with P^T transposed in
 // registers (movmatrix).  Tile columns hold pair i at columns (2i, 2i+1) =
 // channels (i, i + D/2); the output is un-permuted at the end.
+//
+// Fused step (mkv_kvquant_step): the same launch first appends the step's token
+// to every unit.  Each CTA reads the lengths of the batch entries it touches
+// with a ticket in the top 8 bits of T_len[b] (the last of them stores the new
+// length) and takes every cache as holding the token.  The CTA whose range
+// holds a unit's new chunk row has its attention warps quantize the token while
+// the producers stage the first chunk; the producers wait for that (one named
+// barrier) before they copy the chunk that holds the token.
 #include <math.h>
 
 #include "mkv_common.cuh"
 #include "mkv_internal.h"
 #include "mkv_merge.cuh"
+#include "mkv_quant_token.cuh"
 
 namespace mkv {
 
@@ -56,6 +65,10 @@ constexpr int kEnt = 256;                              // key-outlier entries of
 constexpr int kBarProd = 1;                            // producers only
 constexpr int kBarFull = 2;                            // + buffer: tiles of a chunk are ready
 constexpr int kBarEmpty = 4;                           // + buffer: tiles may be overwritten
+constexpr int kBarQDone = 6;                           // fused step: the CTA's new tokens are quantized
+constexpr int kBarQGrp = 7;                            // fused step: the attention warps' quantizer
+constexpr int kMaxUnitsCta = 32;                      // units a CTA's range may touch (tables by unit & 31)
+constexpr int kNewTok = 1 << 30;                       // length flag: the step appended a token
 // Register split: the kernel is compiled for (and launched with) kRegLaunch registers a
 // thread; producer warpgroups give registers back, the consumer warpgroup takes them.
 constexpr int kRegLaunch = 96, kRegProd = 88, kRegCons = 128;
@@ -71,6 +84,35 @@ __device__ __forceinline__ void bar_sync(int id, int n) {
 __device__ __forceinline__ void bar_arrive(int id, int n) {
   __syncwarp();
   asm volatile("bar.arrive %0, %1;\n" ::"r"(id), "r"(n) : "memory");
+}
+
+__device__ uint32_t g_status_kvq;   // MKV_FLAG_* bits raised by the fused step
+
+// Fused step: what the quantizer of the step's token writes and reads.
+struct KvqStep {
+  const __half* k_new;    // [B][Hkv][D] pre-rotation key of the step's token
+  const __half* v_new;    // [B][Hkv][D]
+  int32_t* T_len;
+  uint8_t* k_codes;
+  uint8_t* v_codes;
+  float2* v_params;
+  uint32_t* v_out;
+  int32_t* k_out_off;
+  uint32_t* k_out;
+  const float* t_lo;      // [Hkv][D]
+  const float* t_hi;
+  const float* k_lo;
+  const float* k_scale;
+  const uint16_t* k_cb;   // [Hkv][D][K]
+  const uint16_t* v_cb;
+  int nuq;
+};
+
+// A load of cache data the kernel does not write, or (fused step) may have written: then coherent.
+template <bool kCoherent, typename T>
+__device__ __forceinline__ T ld_cache(const T* p) {
+  if constexpr (kCoherent) return __ldcg(p);
+  else return __ldg(p);
 }
 
 struct KvqArgs {
@@ -96,6 +138,8 @@ struct KvqArgs {
   float* part_l;
   float* part_o;
   MergeArgs merge;
+  int step;                // 1: fused step (append the token, then attend)
+  KvqStep st;
 };
 
 template <int D, int BITS>
@@ -139,7 +183,18 @@ struct KvqLayout {
   static constexpr int QS = VTB + D * K * 4;                 // [8][D] f32 query (as given, rotated)
   static constexpr int STG = QS + 8 * D * 4;                 // [NS][STAGE]
   static constexpr int BUFS = STG + NS * STAGE;              // [2][BUF]
-  static constexpr int BYTES = BUFS + 2 * BUF;
+  // fused step: the attention warps' quantizer scratch, and the lengths of the CTA's batch entries
+  static constexpr int NWQ = (D * BITS / 8 + 3) / 4;         // packed words of a code row
+  static constexpr int QT_KC = BUFS + 2 * BUF;               // [D] u8 key codes
+  static constexpr int QT_VC = QT_KC + D;                    // [D] u8 value codes
+  static constexpr int QT_ABS = QT_VC + D;                   // [D] f32
+  static constexpr int QT_W = QT_ABS + 4 * D;                // [2][NWQ] u32
+  static constexpr int QT_CNT = QT_W + 8 * NWQ;              // [4] int, then lo [4], hi [4]
+  static constexpr int QT_MX = QT_CNT + 48;                  // [2][32] u32
+  static constexpr int BLEN = QT_MX + 256;                   // [32] int per batch entry
+  static constexpr int ULEN = BLEN + 32 * 4;                 // [32] int per unit (unit & 31)
+  static constexpr int UCQ = ULEN + 32 * 4;                  // [32] int per unit (unit & 31)
+  static constexpr int BYTES = UCQ + 32 * 4;
 };
 
 // pair j's two `BITS`-wide codes from a group's realigned code words (j compile-time)
@@ -236,7 +291,64 @@ __device__ __forceinline__ uint32_t movm_trans(uint32_t x) {
   return y;
 }
 
+// Fused step: the step's token of every unit whose new chunk row this CTA holds, quantized by the
+// attention warps with one thread per channel c (Section 2.1, KVQuant paragraph); then the producers
+// may copy those chunks.
 template <int D, int BITS>
+__device__ __forceinline__ void quantize_new_tokens(const KvqArgs& a, int64_t x0, int64_t x1, uint8_t* smem, int c) {
+  using Lay = KvqLayout<D, BITS>;
+  constexpr int K = 1 << BITS;
+  const int* s_ulen = reinterpret_cast<const int*>(smem + Lay::ULEN);
+  const int cc = min(c, D - 1);            // threads c >= D only take part in the barriers
+  const QTokSmem scr{smem + Lay::QT_KC, smem + Lay::QT_VC, reinterpret_cast<float*>(smem + Lay::QT_ABS),
+                     reinterpret_cast<uint32_t*>(smem + Lay::QT_W), reinterpret_cast<int*>(smem + Lay::QT_CNT),
+                     reinterpret_cast<float*>(smem + Lay::QT_CNT + 16), reinterpret_cast<float*>(smem + Lay::QT_CNT + 32),
+                     reinterpret_cast<uint32_t*>(smem + Lay::QT_MX)};
+  bool any = false;
+  const int64_t u_lo = x0 / a.cpu;
+  for (int64_t u = u_lo; u <= (x1 - 1) / a.cpu; ++u) {
+    const int lv = s_ulen[u & 31];
+    if (!(lv & kNewTok)) continue;
+    const int64_t p = (lv & (kNewTok - 1)) - 1, xc = u * a.cpu + p / kChunk;
+    if (xc < x0 || xc >= x1) continue;       // another CTA holds this unit's new token
+    any = true;
+    const int64_t hc = (u % a.Hkv) * D + cc;
+    const float tlo = a.st.t_lo[hc], thi = a.st.t_hi[hc];
+    const float klo = a.st.k_lo ? a.st.k_lo[hc] : 0.f, ksc = a.st.k_scale ? a.st.k_scale[hc] : 0.f;
+    const __half xk = a.st.k_new[u * D + cc], xv = a.st.v_new[u * D + cc];
+    float kmu[15], vmu[15];
+#pragma unroll
+    for (int j = 0; j < 15; ++j) kmu[j] = vmu[j] = 0.f;
+    if (a.st.nuq) {
+      uint16_t kr[K], vr[K];
+#pragma unroll
+      for (int j = 0; j < K; ++j) {
+        kr[j] = a.st.k_cb[hc * K + j];
+        vr[j] = a.st.v_cb[hc * K + j];
+      }
+#pragma unroll
+      for (int j = 0; j + 1 < K; ++j) {
+        kmu[j] = fl32_mid(h2f(kr[j]), h2f(kr[j + 1]));
+        vmu[j] = fl32_mid(h2f(vr[j]), h2f(vr[j + 1]));
+      }
+    }
+    int32_t* off_row = a.st.k_out_off + u * (a.T_cap + 1);
+    const int32_t off = p == 0 ? 0 : __ldcg(off_row + p);
+    if (p == 0 && c == 0) off_row[0] = 0;
+    constexpr int RB = D * BITS / 8;
+    const QTokDst dst{a.st.k_out + u * a.k_out_cap, a.k_out_cap, a.st.v_out + u * a.T_cap * a.n_v,
+                      a.st.v_params + u * a.T_cap, a.st.k_codes + u * a.T_cap * RB, a.st.v_codes + u * a.T_cap * RB,
+                      off_row};
+    quantize_token(c, D, BITS, a.st.nuq != 0, a.n_v, kmu, vmu, tlo, thi, klo, ksc, xk, xv, p, off, dst, scr,
+                   &g_status_kvq, [] { bar_sync(kBarQGrp, kThr - kProdThr); });
+  }
+  if (any) __threadfence_block();          // the cache rows before the producers' copies
+  const int cq0 = reinterpret_cast<const int*>(smem + Lay::UCQ)[u_lo & 31];
+  if (cq0 >= 0 && cq0 < Lay::NS + 2) bar_arrive(kBarQDone, kThr);   // the producers wait for it
+}
+
+// kStep: the fused step (the step's token quantized by the launch); otherwise the cache as it is.
+template <int D, int BITS, bool kStep>
 __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   using Lay = KvqLayout<D, BITS>;
   constexpr int NP = Lay::NP, K = Lay::K, ROWW = Lay::ROWW, SROWW = Lay::SROWW, QP = Lay::QP;
@@ -256,6 +368,31 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   // this CTA's virtual chunks of the concatenated (batch, kv-head) units: one segment per unit
   const int64_t x0 = (int64_t)cta * a.c_tot / a.n_cta, x1 = ((int64_t)cta + 1) * a.c_tot / a.n_cta;
 
+  // Fused step: each CTA that touches batch entry b takes a ticket in the top 8 bits of T_len[b] as
+  // it reads the length (one thread per batch entry); the last one stores the new length, and the
+  // cache is taken as holding the step's token (kNewTok marks it).  The lengths then go to per-unit
+  // tables (unit & 31: a CTA's range spans at most 28 units) with the segment-relative chunk of the
+  // CTA's first new token (-1 elsewhere), so the roles' loops keep no extra registers for them.
+  int* s_blen = reinterpret_cast<int*>(smem + Lay::BLEN);
+  const int* s_ulen = reinterpret_cast<const int*>(smem + Lay::ULEN);
+  const int* s_ucq = reinterpret_cast<const int*>(smem + Lay::UCQ);
+  if (kStep) {
+    const int64_t b_lo = x0 / a.cpu / a.Hkv, nb = (x1 - 1) / a.cpu / a.Hkv - b_lo + 1;
+    if (tid < nb) {
+      const int64_t bb = b_lo + tid;
+      const unsigned old = atomicAdd(reinterpret_cast<unsigned*>(a.st.T_len) + bb, 1u << 24);
+      const int64_t f = cta_of_chunk(bb * a.Hkv * a.cpu, a.c_tot, a.n_cta);
+      const int64_t l = cta_of_chunk((bb + 1) * a.Hkv * a.cpu - 1, a.c_tot, a.n_cta);
+      const int64_t n0 = old & 0xffffffu;
+      const bool room = n0 < a.T_cap;
+      if ((int64_t)(old >> 24) == l - f) {            // the last reader of bb
+        a.st.T_len[bb] = (int32_t)(room ? n0 + 1 : n0);
+        if (!room) atomicOr(&g_status_kvq, MKV_FLAG_CACHE_FULL);
+      }
+      s_blen[tid] = room ? (int)(n0 + 1) | kNewTok : (int)min(n0, a.T_cap);
+    }
+  }
+
   // CTA-resident rotations by delta in [0, 64): coalesced reads of rope rows 0..63, all issued
   // before the transposed stores
   {
@@ -274,6 +411,24 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     }
   }
   __syncthreads();
+  if (kStep && warp == 0) {                // the per-unit tables (read after the first begin_unit)
+    const int64_t u_lo = x0 / a.cpu, b_lo = u_lo / a.Hkv;
+    const int64_t u = u_lo + lane;
+    const bool in = u <= (x1 - 1) / a.cpu;
+    int lv = 0, cq = -1;
+    if (in) {
+      lv = s_blen[(int)(u / a.Hkv - b_lo)];
+      if (lv & kNewTok) {
+        const int64_t xc = u * a.cpu + ((lv & (kNewTok - 1)) - 1) / kChunk;   // the new token's chunk
+        if (xc >= x0 && xc < x1) cq = (int)(xc - max(x0, u * a.cpu));
+      }
+    }
+    const unsigned own = __ballot_sync(0xffffffffu, cq >= 0);
+    if (in) {
+      reinterpret_cast<int*>(smem + Lay::ULEN)[u & 31] = lv;
+      reinterpret_cast<int*>(smem + Lay::UCQ)[u & 31] = own && lane == __ffs(own) - 1 ? cq : -1;
+    }
+  }
 
   // the four attention warps' (m, l, o) per query row, merged after both roles finish a segment
   float* wm = reinterpret_cast<float*>(stg);                // [4 warps][8 rows]
@@ -363,10 +518,18 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       const int64_t xe = min(x1, (bh + 1) * a.cpu);
       begin_unit(bh);
       const int b = (int)(bh / a.Hkv);
-      const int n_len = (int)min((int64_t)a.T_len[b], a.T_cap);
+      const int n_len = kStep ? s_ulen[bh & 31] & (kNewTok - 1) : (int)min((int64_t)a.T_len[b], a.T_cap);
       const int64_t v_begin = (x - bh * a.cpu) * kChunk;
       const int64_t v_end = min((xe - bh * a.cpu) * kChunk, (int64_t)n_len);
       const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
+      // Fused step: the attention warps quantize the CTA's new tokens before they attend to anything,
+      // so every copy made after the producers' first wait for a released buffer (chunk NS + 2 of the
+      // first segment on) or in a later segment (after a CTA barrier) reads the new rows.  A new token
+      // in one of the first segment's earlier chunks makes the producers wait for the quantizer here.
+      if (kStep && x == x0) {
+        const int cq = s_ucq[bh & 31];
+        if (cq >= 0 && cq < NS + 2) bar_sync(kBarQDone, kThr);
+      }
     const uint32_t* kc_base = reinterpret_cast<const uint32_t*>(a.k_codes) + bh * a.T_cap * ROWW;
     const uint32_t* vc_base = reinterpret_cast<const uint32_t*>(a.v_codes) + bh * a.T_cap * ROWW;
     const uint32_t* gents = a.k_out + bh * a.k_out_cap;
@@ -464,8 +627,9 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
       if (s < nchunks) {
         load_chunk(s, s);
         if (s == 0 && ptid < kEnt) {
-          const int e0 = __ldg(a.k_out_off + off_base + v_begin);
-          const int e1 = min(__ldg(a.k_out_off + off_base + min(v_begin + kChunk, (int64_t)n_len)), (int)a.k_out_cap);
+          const int e0 = ld_cache<kStep>(a.k_out_off + off_base + v_begin);
+          const int e1 = min(ld_cache<kStep>(a.k_out_off + off_base + min(v_begin + kChunk, (int64_t)n_len)),
+                             (int)a.k_out_cap);
           load_entries(0, e0, e1);
         }
       }
@@ -586,12 +750,17 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
     const int t0w = cw * 16;
     const int tokA = t0w + (mi & 1) * 8 + rowi, chA = mi >> 1;   // K slab as the A operand
     const int tokV = t0w + (mi >> 1) * 8 + rowi, chV = mi & 1;   // V^T slab as the A operand
+    bool q_todo = kStep;                     // fused step: quantize the CTA's new tokens first
     for (int64_t x = x0; x < x1;) {
       const int64_t bh = x / a.cpu;                           // this segment's unit
       const int64_t xe = min(x1, (bh + 1) * a.cpu);
       begin_unit(bh);
+      if (q_todo) {
+        quantize_new_tokens<D, BITS>(a, x0, x1, smem, tid - kProdThr);
+        q_todo = false;
+      }
       const int b = (int)(bh / a.Hkv);
-      const int n_len = (int)min((int64_t)a.T_len[b], a.T_cap);
+      const int n_len = kStep ? s_ulen[bh & 31] & (kNewTok - 1) : (int)min((int64_t)a.T_len[b], a.T_cap);
       const int64_t v_begin = (x - bh * a.cpu) * kChunk;
       const int64_t v_end = min((xe - bh * a.cpu) * kChunk, (int64_t)n_len);
       const int nchunks = v_end > v_begin ? (int)ceil_div_dev(v_end - v_begin, kChunk) : 0;
@@ -622,7 +791,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
         auto fetch = [&](int e) -> uint32_t {
           if (e < 0 || e >= e_hi) return 0xffff0000u;  // no entry: not a channel
           if (e - E0 < kEnt) return ents[e - E0];
-          return __ldg(gents + e);            // beyond the staged entries
+          return ld_cache<kStep>(gents + e);  // beyond the staged entries
         };
         auto fix = [&](uint32_t ev, int pass) {
           const int ch = (int)((ev >> 16) & 0xffu);
@@ -662,7 +831,7 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
           const int t = t0w + (e & 15), k = e >> 4;
           if (t0 + t >= n_len) continue;
           const uint32_t ev = a.n_v <= Lay::NVS ? reinterpret_cast<const uint32_t*>(B_ + Lay::B_VO)[k * kChunk + t]
-                                                : __ldg(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
+                                                : ld_cache<kStep>(a.v_out + (bh * a.T_cap + t0 + t) * a.n_v + k);
           const int chn = (int)(ev >> 16);
           if (chn >= D) continue;
           const int col = chn < NP ? 2 * chn : 2 * (chn - NP) + 1;
@@ -766,30 +935,47 @@ __global__ void __launch_bounds__(kThr, 1) decode_kvq_kernel(const KvqArgs a) {
   }
 }
 
-template <int D, int BITS>
-cudaError_t launch_kvq_t(const KvqArgs& a, cudaStream_t st) {
+template <int D, int BITS, bool kStep>
+cudaError_t launch_kvq_s(const KvqArgs& a, cudaStream_t st) {
   using Lay = KvqLayout<D, BITS>;
   static_assert(Lay::BYTES <= 227 * 1024, "one CTA per SM");
   static int checked = 0;                 // 1: attributes set and register count verified
   if (!checked) {
     cudaFuncAttributes attr;
-    cudaError_t e = cudaFuncGetAttributes(&attr, decode_kvq_kernel<D, BITS>);
+    cudaError_t e = cudaFuncGetAttributes(&attr, decode_kvq_kernel<D, BITS, kStep>);
     if (e != cudaSuccess) return e;
     // the register split above assumes exactly kRegLaunch registers a thread at launch
     if (attr.numRegs != kRegLaunch) return cudaErrorInvalidConfiguration;
-    e = cudaFuncSetAttribute(decode_kvq_kernel<D, BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, Lay::BYTES);
+    e = cudaFuncSetAttribute(decode_kvq_kernel<D, BITS, kStep>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             Lay::BYTES);
     if (e != cudaSuccess) return e;
     checked = 1;
   }
-  decode_kvq_kernel<D, BITS><<<a.n_cta, kThr, Lay::BYTES, st>>>(a);
+  decode_kvq_kernel<D, BITS, kStep><<<a.n_cta, kThr, Lay::BYTES, st>>>(a);
   return cudaPeekAtLastError();
+}
+
+template <int D, int BITS>
+cudaError_t launch_kvq_t(const KvqArgs& a, cudaStream_t st) {
+  return a.step ? launch_kvq_s<D, BITS, true>(a, st) : launch_kvq_s<D, BITS, false>(a, st);
 }
 
 }  // namespace
 
+int kvquant_step_max_units_per_cta() { return kMaxUnitsCta; }
+
+cudaError_t take_status_kvq_step(uint32_t* flags, cudaStream_t st) {
+  uint32_t zero = 0, v = 0;
+  cudaError_t e = cudaMemcpyFromSymbolAsync(&v, g_status_kvq, sizeof(v), 0, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemcpyToSymbolAsync(g_status_kvq, &zero, sizeof(zero), 0, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  *flags |= v;
+  return e;
+}
+
 cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_cache& cache,
                                   const mkv_quant_params& qp, void* out, const DecodeWs& ws, const Split& sp,
-                                  cudaStream_t st) {
+                                  cudaStream_t st, const void* k_new, const void* v_new) {
   KvqArgs a{};
   a.q = static_cast<const __half*>(q);
   a.k_codes = cache.k_codes;
@@ -819,6 +1005,25 @@ cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_
   a.part_l = ws.part_l;
   a.part_o = ws.part_o;
   a.merge = merge_args(c, ws, sp, out, false);
+  if (k_new) {
+    a.step = 1;
+    a.st.k_new = static_cast<const __half*>(k_new);
+    a.st.v_new = static_cast<const __half*>(v_new);
+    a.st.T_len = cache.T_len;
+    a.st.k_codes = cache.k_codes;
+    a.st.v_codes = cache.v_codes;
+    a.st.v_params = reinterpret_cast<float2*>(cache.v_params);
+    a.st.v_out = cache.v_out;
+    a.st.k_out_off = cache.k_out_off;
+    a.st.k_out = cache.k_out;
+    a.st.t_lo = qp.t_lo;
+    a.st.t_hi = qp.t_hi;
+    a.st.k_lo = qp.k_lo;
+    a.st.k_scale = qp.k_scale;
+    a.st.k_cb = qp.k_cb;
+    a.st.v_cb = qp.v_cb;
+    a.st.nuq = c.quant_mode == MKV_QUANT_NUQ;
+  }
   if (c.D == 128) {
     if (c.bits == 4) return launch_kvq_t<128, 4>(a, st);
     if (c.bits == 3) return launch_kvq_t<128, 3>(a, st);

@@ -13,14 +13,13 @@
 
 #include "mkv_common.cuh"
 #include "mkv_internal.h"
+#include "mkv_quant_token.cuh"
 
 namespace mkv {
 
 namespace {
 
 __device__ uint32_t g_status_kvquant;
-
-__device__ __forceinline__ float fl32_mid(float a, float b) { return __fmul_rn(__fadd_rn(a, b), 0.5f); }
 
 // ----------------------------------------------------------------- prepare
 
@@ -64,19 +63,13 @@ struct QuantArgs {
   int64_t T_cap;
 };
 
-__device__ __forceinline__ int uniform_code(float x, float lo, float scale, int L) {
-  if (scale == 0.f) return 0;
-  const float r = rintf(__fdiv_rn(__fsub_rn(x, lo), scale));
-  return (int)fminf(fmaxf(r, 0.f), (float)L);
-}
-
 // One CTA per (batch, kv-head), one thread per channel; tokens in order so the
 // key-outlier CSR is appended sequentially.  Every CTA reads T_len[b] once; the
 // last CTA of batch entry b to finish stores the new length: during the launch
 // the top 8 bits of T_len[b] count the finished CTAs (readers mask them off).
 __global__ void quantize_kernel(const QuantArgs a) {
   extern __shared__ uint8_t sm[];
-  const int D = a.D, K = 1 << a.bits, L = K - 1, NP = D / 2;
+  const int D = a.D, K = 1 << a.bits, L = K - 1;
   const int bh = blockIdx.x;
   const int b = bh / a.Hkv, h = bh % a.Hkv;
   const int c = threadIdx.x;   // channel
@@ -124,8 +117,6 @@ __global__ void quantize_kernel(const QuantArgs a) {
     finish(t_base);
     return;
   }
-  const int rowb = D * a.bits / 8;
-  const int nwords = (rowb + 3) / 4;
   float kmu[15], vmu[15];
   if (a.nuq) {
 #pragma unroll
@@ -137,144 +128,21 @@ __global__ void quantize_kernel(const QuantArgs a) {
     }
   }
   if (t_base == 0 && c == 0) off_row[0] = 0;
-  const int warp = c >> 5, lane = c & 31, nwarp = D >> 5;
-
+  const QTokDst dst{a.k_out + (int64_t)bh * a.k_out_cap, a.k_out_cap, a.v_out + (int64_t)bh * a.T_cap * a.n_v,
+                    a.v_params + (int64_t)bh * a.T_cap, a.k_codes + (int64_t)bh * a.T_cap * (D * a.bits / 8),
+                    a.v_codes + (int64_t)bh * a.T_cap * (D * a.bits / 8), off_row};
+  const QTokSmem scr{kcode, vcode, absx, words, s_cnt, s_lo, s_hi, &s_max[0][0]};
   for (int64_t i = 0; i < a.n_tokens; ++i) {
-    const int64_t t = t_base + i;
     const __half xk = xk_next, xv = xv_next;     // this token's key and value; the next one's in flight
     if (i + 1 < a.n_tokens) {
       xk_next = a.k_pre[src0 + (i + 1) * D];
       xv_next = a.v[src0 + (i + 1) * D];
     }
-    // ---- keys
-    const float x = __half2float(xk);
-    const bool kout = (x < tlo) || (x > thi);
-    int code;
-    if (a.nuq) {
-      code = 0;
-#pragma unroll
-      for (int j = 0; j < 15; ++j) code += (j < L && x > kmu[j]) ? 1 : 0;   // registers, no local array
-    } else {
-      code = uniform_code(x, klo, ksc, L);
-    }
-    kcode[c] = (uint8_t)code;
-    // rank of this outlier among the token's outliers (channel order)
-    const unsigned bal = __ballot_sync(0xffffffffu, kout);
-    if (lane == 0) s_cnt[warp] = __popc(bal);
-    // ---- values: rank by (|x| desc, channel asc).  With few value outliers the ranks 0..n_v-1 are
-    // taken by block-wide maxima of key = (|x| as fp16 magnitude bits << 8) | (255 - c), which orders
-    // like (|x| desc, channel asc) for finite values and is unique; the first round shares this
-    // barrier.  Otherwise each thread counts the channels ahead of it.
-    const float vx = __half2float(xv);
-    const bool few = a.n_v <= 8;
-    uint32_t vkey = ((uint32_t)(__half_as_ushort(xv) & 0x7fffu) << 8) | (uint32_t)(255 - c);
-    if (few) {
-      const uint32_t wmax = __reduce_max_sync(0xffffffffu, vkey);
-      if (lane == 0 && a.n_v > 0) s_max[0][warp] = wmax;
-    } else {
-      absx[c] = fabsf(vx);
-    }
-    __syncthreads();
-    int before = 0, total = 0;
-    for (int w = 0; w < nwarp; ++w) {
-      before += (w < warp) ? s_cnt[w] : 0;
-      total += s_cnt[w];
-    }
-    if (kout) {
-      const int64_t e = (int64_t)off + before + __popc(bal & ((1u << lane) - 1u));
-      if (e < a.k_out_cap) {
-        // (token position within its 64-token block << 24) | (channel << 16) | fp16 bits
-        a.k_out[(int64_t)bh * a.k_out_cap + e] =
-            ((uint32_t)(t & 63) << 24) | ((uint32_t)c << 16) | __half_as_ushort(xk);
-      } else {
-        atomicOr(&g_status_kvquant, MKV_FLAG_K_OUTLIER_OVERFLOW);
-      }
-    }
-    int rank = 0;
-    if (few) {
-      rank = a.n_v;                      // not among the n_v largest unless a round picks it
-      for (int r = 0; r < a.n_v; ++r) {
-        if (r > 0) {
-          const uint32_t wmax = __reduce_max_sync(0xffffffffu, vkey);
-          if (lane == 0) s_max[r & 1][warp] = wmax;
-          __syncthreads();
-        }
-        uint32_t m = s_max[r & 1][0];
-        for (int w = 1; w < nwarp; ++w) m = max(m, s_max[r & 1][w]);
-        if (vkey == m) {
-          rank = r;
-          vkey = 0u;                       // out of the later rounds (every live key is >= 128)
-        }
-      }
-    } else {
-      const float ax = absx[c];
-      for (int j = 0; j < D; ++j) {
-        const float o = absx[j];
-        rank += (o > ax || (o == ax && j < c)) ? 1 : 0;
-      }
-    }
-    const bool vout = rank < a.n_v;
-    // inlier range of the token's values
-    float lo = vout ? INFINITY : vx, hi = vout ? -INFINITY : vx;
-    for (int s = 16; s > 0; s >>= 1) {
-      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, s));
-      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, s));
-    }
-    if (lane == 0) {
-      s_lo[warp] = lo;
-      s_hi[warp] = hi;
-    }
-    __syncthreads();
-    lo = s_lo[0];
-    hi = s_hi[0];
-    for (int w = 1; w < nwarp; ++w) {
-      lo = fminf(lo, s_lo[w]);
-      hi = fmaxf(hi, s_hi[w]);
-    }
-    if (lo > hi) lo = hi = 0.f;   // no inlier
-    float scale;
-    int vc;
-    if (a.nuq) {
-      scale = __fsub_rn(hi, lo);
-      const float u = scale == 0.f ? 0.f : __fdiv_rn(__fsub_rn(vx, lo), scale);
-      vc = 0;
-#pragma unroll
-      for (int j = 0; j < 15; ++j) vc += (j < L && u > vmu[j]) ? 1 : 0;
-    } else {
-      scale = __fdiv_rn(__fsub_rn(hi, lo), (float)L);
-      vc = uniform_code(vx, lo, scale, L);
-    }
-    vcode[c] = (uint8_t)vc;
-    const int64_t slot = (int64_t)bh * a.T_cap + t;
-    if (vout) a.v_out[slot * a.n_v + rank] = ((uint32_t)c << 16) | __half_as_ushort(xv);
-    if (c == 0) a.v_params[slot] = make_float2(lo, scale);
-    for (int wi = c; wi < 2 * nwords; wi += D) words[wi] = 0u;
-    __syncthreads();
-    // pack pair i = channels (i, i + D/2) at bits [2*bits*i, 2*bits*(i+1))
-    if (c < NP) {
-      const uint32_t pk = (uint32_t)kcode[c] | ((uint32_t)kcode[c + NP] << a.bits);
-      const uint32_t pv = (uint32_t)vcode[c] | ((uint32_t)vcode[c + NP] << a.bits);
-      const int bit = 2 * a.bits * c;
-      const int w0 = bit >> 5, sh = bit & 31;
-      atomicOr(&words[w0], pk << sh);
-      atomicOr(&words[nwords + w0], pv << sh);
-      if (sh + 2 * a.bits > 32) {
-        atomicOr(&words[w0 + 1], pk >> (32 - sh));
-        atomicOr(&words[nwords + w0 + 1], pv >> (32 - sh));
-      }
-    }
-    __syncthreads();
-    for (int by = c; by < rowb; by += D) {
-      a.k_codes[slot * rowb + by] = reinterpret_cast<const uint8_t*>(words)[by];
-      a.v_codes[slot * rowb + by] = reinterpret_cast<const uint8_t*>(words + nwords)[by];
-    }
-    off += total;
-    if (c == 0) off_row[t + 1] = off;
-    __syncthreads();
+    off = quantize_token(c, D, a.bits, a.nuq != 0, a.n_v, kmu, vmu, tlo, thi, klo, ksc, xk, xv, t_base + i, off, dst,
+                         scr, &g_status_kvquant, [] { __syncthreads(); });
   }
   finish(t_base + a.n_tokens);
 }
-
 
 // ----------------------------------------------------------------- calibrate
 

@@ -323,6 +323,7 @@ mkv_status mkv_get_status(void* stream, uint32_t* flags) {
   MKV_CUDA(take_status_rocket(flags, as_stream(stream)));
   MKV_CUDA(take_status_decode(flags, as_stream(stream)));
   MKV_CUDA(take_status_prefill(flags, as_stream(stream)));
+  MKV_CUDA(take_status_kvq_step(flags, as_stream(stream)));
   if (*flags & MKV_FLAG_WAIT_TIMEOUT) {
     set_error("device status flags 0x%x (a bounded wait ran out)", *flags);
     return MKV_ERR_TIMEOUT;
@@ -382,8 +383,7 @@ mkv_status mkv_decode_step(const mkv_config* cfg, const void* q, const void* k_n
                            mkv_cache* cache, void* out, void* ws, size_t ws_bytes, void* stream) {
   MKV_TRY(check_config(cfg));
   MKV_REQUIRE(cfg->method == MKV_FP16 || cfg->method == MKV_H2O, MKV_ERR_INVALID_ARG,
-              "decode_step is for FP16 and H2O (KVQUANT: mkv_quantize_kv + mkv_decode_attention; ROCKET: "
-              "mkv_rocket_step)");
+              "decode_step is for FP16 and H2O (KVQUANT: mkv_kvquant_step; ROCKET: mkv_rocket_step)");
   MKV_TRY(check_cache(cfg, cache));
   MKV_REQUIRE(q && out && k_new && v_new, MKV_ERR_INVALID_ARG, "q/out/k_new/v_new NULL");
   MKV_REQUIRE(((uintptr_t)k_new | (uintptr_t)v_new) % 16 == 0, MKV_ERR_INVALID_ARG,
@@ -399,6 +399,49 @@ mkv_status mkv_decode_step(const mkv_config* cfg, const void* q, const void* k_n
               (long long)cache->T_cap, cfg->Hkv, sp.n_split);
   MKV_CUDA(launch_decode_fp16_family(*cfg, q, *cache, nullptr, out, decode_ws(*cfg, cache->T_cap, ws), sp,
                                      as_stream(stream), k_new, v_new));
+  return MKV_OK;
+}
+
+mkv_status mkv_kvquant_step(const mkv_config* cfg, const mkv_quant_params* qparams, const void* q,
+                            const void* k_new, const void* v_new, mkv_cache* cache, void* out, void* ws,
+                            size_t ws_bytes, void* stream) {
+  MKV_TRY(check_config(cfg));
+  MKV_REQUIRE(cfg->method == MKV_KVQUANT, MKV_ERR_INVALID_ARG, "kvquant_step is for KVQUANT");
+  MKV_TRY(check_cache(cfg, cache));
+  MKV_TRY(check_qparams(cfg, qparams, true));
+  MKV_REQUIRE(q && out && k_new && v_new, MKV_ERR_INVALID_ARG, "q/out/k_new/v_new NULL");
+  MKV_REQUIRE(qparams->rope && qparams->rope_len >= std::max<int64_t>(cache->T_cap, 64), MKV_ERR_INVALID_ARG,
+              "KVQUANT decode needs a rope table with rope_len >= max(T_cap, 64)");
+  MKV_REQUIRE(((uintptr_t)cache->k_codes | (uintptr_t)cache->v_codes) % 16 == 0, MKV_ERR_INVALID_ARG,
+              "KVQUANT decode stages k_codes / v_codes in 16-byte pieces: both must be 16-byte aligned");
+  MKV_REQUIRE(cache->k_out_cap <= INT32_MAX && cache->T_cap < INT32_MAX, MKV_ERR_UNSUPPORTED,
+              "KVQUANT decode indexes key outliers and tokens with 32 bits (k_out_cap %lld, T_cap %lld)",
+              (long long)cache->k_out_cap, (long long)cache->T_cap);
+  const DecodeWs need = decode_ws(*cfg, cache->T_cap, nullptr);
+  MKV_REQUIRE(ws != nullptr && ws_bytes >= need.bytes, MKV_ERR_WORKSPACE,
+              "workspace %zu bytes < %zu needed", ws_bytes, need.bytes);
+  const Split sp = decode_split(*cfg, cache->T_cap);
+  // Each (CTA, unit) pair of batch entry b takes a ticket in the top 8 bits of T_len[b] (at most 255
+  // of them); a CTA keeps its units' lengths in 32-entry tables (it spans at most 28 of the <= 4096
+  // units).
+  const int64_t units = (int64_t)cfg->B * cfg->Hkv, cpu = sp.chunks_per_unit, c_tot = cpu * units;
+  int64_t max_tickets = 0;
+  for (int64_t b = 0; b < cfg->B; ++b) {
+    int64_t t = 0;
+    for (int64_t u = b * cfg->Hkv; u < (b + 1) * cfg->Hkv; ++u)
+      t += cta_of_chunk((u + 1) * cpu - 1, c_tot, sp.n_cta) - cta_of_chunk(u * cpu, c_tot, sp.n_cta) + 1;
+    max_tickets = std::max(max_tickets, t);
+  }
+  const int64_t span = (ceil_div(c_tot, (int64_t)sp.n_cta) - 1) / cpu + 2;
+  MKV_REQUIRE(max_tickets <= 255 && span <= kvquant_step_max_units_per_cta(), MKV_ERR_UNSUPPORTED,
+              "kvquant_step: %lld CTA-unit pairs read one batch entry's length (at most 255) or a CTA spans %lld "
+              "units (at most %d); use mkv_quantize_kv + mkv_decode_attention",
+              (long long)max_tickets, (long long)span, kvquant_step_max_units_per_cta());
+  MKV_REQUIRE(cache->T_cap < (1 << 24), MKV_ERR_UNSUPPORTED,
+              "kvquant_step needs T_cap < 2^24 (T_cap %lld); use mkv_quantize_kv + mkv_decode_attention",
+              (long long)cache->T_cap);
+  MKV_CUDA(launch_decode_kvquant(*cfg, q, *cache, *qparams, out, decode_ws(*cfg, cache->T_cap, ws), sp,
+                                 as_stream(stream), k_new, v_new));
   return MKV_OK;
 }
 

@@ -103,9 +103,13 @@ cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const 
                                       const int32_t* page_idx, void* out, const DecodeWs& ws,
                                       const Split& sp, cudaStream_t st, const void* k_new = nullptr,
                                       const void* v_new = nullptr);
+// k_new / v_new (KVQUANT fused step): the step's token, quantized and appended by the same launch.
 cudaError_t launch_decode_kvquant(const mkv_config& c, const void* q, const mkv_cache& cache,
                                   const mkv_quant_params& qp, void* out,
-                                  const DecodeWs& ws, const Split& sp, cudaStream_t st);
+                                  const DecodeWs& ws, const Split& sp, cudaStream_t st,
+                                  const void* k_new = nullptr, const void* v_new = nullptr);
+// Units one CTA of the fused KVQuant step may touch (its length tables).
+int kvquant_step_max_units_per_cta();
 cudaError_t launch_append(const mkv_config& c, const void* k_new, const void* v_new,
                           const mkv_cache& cache, cudaStream_t st);
 cudaError_t launch_rope_table(int D, float theta, int64_t T_max, float* table, cudaStream_t st);
@@ -144,6 +148,7 @@ cudaError_t take_status_append(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_rocket(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_decode(uint32_t* flags, cudaStream_t st);
 cudaError_t take_status_prefill(uint32_t* flags, cudaStream_t st);
+cudaError_t take_status_kvq_step(uint32_t* flags, cudaStream_t st);
 cudaError_t launch_wait_selftest(int ms, cudaStream_t st);
 
 }  // namespace mkv

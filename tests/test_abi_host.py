@@ -164,3 +164,30 @@ def test_decode_step_checks(L):
     cache.T_cap = 1 << 24
     st = L.mkv_decode_step(ctypes.byref(fc), 64, 80, 96, ctypes.byref(cache), 128, 4096, big, None)
     assert st == mkv.MKV_ERR_UNSUPPORTED
+
+
+def test_kvquant_step_checks(L):
+    """mkv_kvquant_step is for KVQUANT, needs its inputs and a workspace, and counts the CTAs that read
+    T_len[b] in its top 8 bits (T_cap < 2^24); every rejection happens on the host."""
+    kq = mkv.config(mkv.MKV_KVQUANT, 1, 32, 8, 128, bits=4)
+    qp = mkv.mkv_quant_params()
+    for name in ("t_lo", "t_hi", "k_lo", "k_scale", "k_dq", "v_tbl", "rope"):
+        setattr(qp, name, 1 << 20)
+    qp.k_cb, qp.v_cb, qp.rope_len = 1 << 20, 1 << 20, 1 << 16
+    cache = mkv.mkv_cache()
+    cache.T_cap, cache.T_len = 8192, 8
+    cache.k_codes, cache.v_codes, cache.v_params, cache.v_out = 1 << 12, 1 << 13, 1 << 14, 1 << 15
+    cache.k_out_off, cache.k_out, cache.k_out_cap = 1 << 16, 1 << 17, 4096
+    big = ctypes.c_size_t(1 << 40)
+    args = lambda cfg, kn: (ctypes.byref(cfg), ctypes.byref(qp), 64, kn, 96, ctypes.byref(cache), 128, 4096, big, None)
+    fc = mkv.config(mkv.MKV_FP16, 1, 32, 8, 128)
+    assert L.mkv_kvquant_step(*args(fc, 80)) == mkv.MKV_ERR_INVALID_ARG
+    assert "KVQUANT" in mkv.mkv_last_error()
+    assert L.mkv_kvquant_step(*args(kq, None)) == mkv.MKV_ERR_INVALID_ARG
+    st = L.mkv_kvquant_step(ctypes.byref(kq), ctypes.byref(qp), 64, 80, 96, ctypes.byref(cache), 128, 4096,
+                            ctypes.c_size_t(16), None)
+    assert st == mkv.MKV_ERR_WORKSPACE
+    cache.T_cap, qp.rope_len = 1 << 24, 1 << 25
+    st = L.mkv_kvquant_step(*args(kq, 80))
+    assert st == mkv.MKV_ERR_UNSUPPORTED and "2^24" in mkv.mkv_last_error()
+
