@@ -104,6 +104,9 @@ typedef struct {
  *
  *  FP16 / ROCKET: k, v fp16 [B][Hkv][T_cap][D], rows 0..T_len-1 valid.
  *  H2O:   k, v fp16 [B][Hkv][T_cap][D] with T_cap >= heavy + recent + 1;
+ *         only slots 0..heavy+recent are ever used (the prefill fills slots
+ *         from 0 and each step writes the lowest free slot or the one its
+ *         eviction freed), and the decode and the update read only those;
  *         pos int32 [B][Hkv][T_cap] (position held by each slot, -1 = empty);
  *         acc fp32 [B][Hkv][T_cap] accumulated attention score;
  *         slot int32 [B][Hkv] the slot the next append writes.
@@ -260,7 +263,7 @@ mkv_status mkv_append_kv(const mkv_config* cfg, const void* k_new, const void* v
  *   FP16, KVQUANT: slots 0..T_len[b]-1 (KVQUANT dequantizes keys, restores
  *                  outliers, rotates keys by their position, dequantizes
  *                  values -- all fused; Section 2.1 KVQuant paragraph);
- *   H2O:           every slot with pos >= 0;
+ *   H2O:           every slot among 0..heavy+recent with pos >= 0;
  *   ROCKET:        the pages listed in page_idx [B][Hkv][topk_pages] (int32,
  *                  -1 = unused) plus the tail page that holds the newest
  *                  token (Section 2.1, RocketKV paragraph, second stage).

@@ -14,6 +14,8 @@
 // mkv_decode_step appends the step's token in the same launch (FP16, H2O).
 #include <math.h>
 
+#include <algorithm>
+
 #include <mutex>
 
 #include "mkv_common.cuh"
@@ -37,6 +39,7 @@ struct Fp16Args {
   const int32_t* pos;     // H2O [B][Hkv][T_cap]
   const int32_t* page_idx;// ROCKET [B][Hkv][kp]
   int64_t T_cap;
+  int64_t n_slots;         // H2O: slots a unit can hold, min(T_cap, H + R + 1)
   int Hq, Hkv, G;
   int chunks_per_split;
   int kp;
@@ -132,7 +135,7 @@ __global__ void __launch_bounds__(kThreads, 2) decode_fp16_kernel(const Fp16Args
     n_len = step ? (int)min((int64_t)t_old + (ok_b ? 1 : 0), a.T_cap) : (int)min((int64_t)a.T_len[b], a.T_cap);
     v_total = n_len;
   } else if (MODE == 1) {
-    v_total = a.T_cap;
+    v_total = a.n_slots;                 // slots past H + R are never used (H2O slot policy)
   } else {
     n_len = (int)min((int64_t)a.T_len[b], a.T_cap);
     ns = n_len > 0 ? (n_len - 1) / kPage : 0;
@@ -417,6 +420,9 @@ cudaError_t launch_decode_fp16_family(const mkv_config& c, const void* q, const 
   a.pos = cache.pos;
   a.page_idx = page_idx;
   a.T_cap = cache.T_cap;
+  // H2O: the prefill keeps at most H + R tokens in slots 0.., and each step's token goes to the
+  // lowest free slot or to the slot its eviction freed, so no slot past H + R is ever used
+  a.n_slots = std::min<int64_t>(cache.T_cap, (int64_t)c.h2o_heavy + c.h2o_recent + 1);
   a.Hq = c.Hq;
   a.Hkv = c.Hkv;
   a.G = c.Hq / c.Hkv;

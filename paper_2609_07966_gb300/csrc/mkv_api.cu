@@ -25,7 +25,9 @@ void set_error(const char* fmt, ...) {
 
 Split decode_split(const mkv_config& c, int64_t T_cap) {
   Split s{};
-  s.v_tokens = c.method == MKV_ROCKET ? (int64_t)(c.topk_pages + 1) * kPage : T_cap;
+  s.v_tokens = c.method == MKV_ROCKET ? (int64_t)(c.topk_pages + 1) * kPage
+              : c.method == MKV_H2O  ? std::min<int64_t>(T_cap, (int64_t)c.h2o_heavy + c.h2o_recent + 1)
+                                     : T_cap;
   const int64_t chunks = std::max<int64_t>(1, ceil_div(s.v_tokens, kChunk));
   const int64_t units = (int64_t)c.B * c.Hkv;
   // The fp16-family decode kernels keep two CTAs resident per SM, the KVQuant

@@ -46,7 +46,8 @@ __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits
   int best_slot = -1, first_free = INT32_MAX;
   // kU slots per thread per pass, their loads issued together so their latencies overlap
   constexpr int kU = 4;
-  for (int64_t s0 = threadIdx.x; s0 < T_cap; s0 += (int64_t)kU * blockDim.x) {
+  const int64_t n_slots = min(T_cap, (int64_t)H + R + 1);   // no slot past H + R is ever used
+  for (int64_t s0 = threadIdx.x; s0 < n_slots; s0 += (int64_t)kU * blockDim.x) {
     int32_t p[kU];
     float a_old[kU], add[kU];
     // every load of the pass first (a slot's acc and logits are read even when it is empty, so
@@ -54,7 +55,7 @@ __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
       const int64_t s = s0 + (int64_t)u * blockDim.x;
-      const bool in = s < T_cap;
+      const bool in = s < n_slots;
       p[u] = in ? pos[bh * T_cap + s] : -1;
       a_old[u] = in ? acc[bh * T_cap + s] : 0.f;
       add[u] = 0.f;
@@ -75,7 +76,7 @@ __device__ __forceinline__ void h2o_update_unit(const float* __restrict__ logits
     for (int u = 0; u < kU; ++u) {
       const int64_t s = s0 + (int64_t)u * blockDim.x;
       if (p[u] < 0) {                 // an empty slot (past the end: not a slot)
-        if (s < T_cap) first_free = min(first_free, (int)s);
+        if (s < n_slots) first_free = min(first_free, (int)s);
         continue;
       }
       ++held;
