@@ -37,13 +37,17 @@
 // registers (movmatrix).  Tile columns hold pair i at columns (2i, 2i+1) =
 // channels (i, i + D/2); the output is un-permuted at the end.
 //
-// Fused step (mkv_kvquant_step): the same launch first appends the step's token
-// to every unit.  Each CTA reads the lengths of the batch entries it touches
-// with a ticket in the top 8 bits of T_len[b] (the last of them stores the new
-// length) and takes every cache as holding the token.  The CTA whose range
-// holds a unit's new chunk row has its attention warps quantize the token while
-// the producers stage the first chunk; the producers wait for that (one named
-// barrier) before they copy the chunk that holds the token.
+// Fused step (mkv_kvquant_step, the kStep instantiation): the same launch first
+// appends the step's token to every unit.  Each CTA reads the lengths of the
+// batch entries it touches with a ticket in the top 8 bits of T_len[b] (the
+// last of them stores the new length) and takes every cache as holding the
+// token.  The CTA whose range holds a unit's new chunk row has its attention
+// warps quantize the token (the quantize kernel's routine, so the bits match)
+// before they attend to anything, while the producers stage the first chunks.
+// Every copy made after the producers' first wait for a released tile buffer,
+// or in a later segment, therefore reads the new rows; only a new token in one
+// of the first segment's first NS + 2 chunks makes the producers wait for the
+// quantizer (one named barrier) before they copy anything.
 #include <math.h>
 
 #include "mkv_common.cuh"
