@@ -453,10 +453,11 @@ def time_decode_launches(runner, reps):
     return a.elapsed_time(b) / (reps * runner.w.L)
 
 
-def time_e2e(runner, steps, warmup):
+def time_e2e(runner, steps, warmup, graph=True):
     """Through the public API with host buffers: per step, one H2D copy of every layer's q and
     new k/v from pinned memory (packed in one buffer), the step's API calls, and one D2H copy of
-    every layer's output."""
+    every layer's output.  graph: the step (copies included) captured once in a CUDA graph and
+    replayed, as a serving loop runs it; otherwise eager launches."""
     torch = runner.torch
     w = runner.w
     ins = [t for l in range(w.L) for t in (runner.q[l], runner.kn[l], runner.vn[l])]
@@ -479,12 +480,24 @@ def time_e2e(runner, steps, warmup):
         runner.join_side()
         h_out.copy_(d_out, non_blocking=True)
 
+    run = one
+    if graph:
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            one()                             # the launch paths warmed outside capture
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            one()
+        run = g.replay
     for _ in range(warmup):
-        one()
+        run()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(steps):
-        one()
+        run()
     torch.cuda.synchronize()
     dt = (time.perf_counter() - t0) / steps
     h2d = h_in.numel() * h_in.element_size()
@@ -837,7 +850,7 @@ def main():
 
     alg_bytes, T_now, ovh_bytes = runner.decode_bytes()
     dec_ms = time_decode_launches(runner, 10)
-    e2e_s, h2d, d2h = time_e2e(runner, max(1, min(args.steps, 5)), 1)
+    e2e_s, h2d, d2h = time_e2e(runner, max(1, min(args.steps, 5)), 1, graph=not args.no_graph)
     peak, peak_kind = peaks()
     achieved = alg_bytes / (dec_ms * 1e-3) / 1e9
     value = whole_job_tokens_per_s(w.B, world, ms)
@@ -848,7 +861,7 @@ def main():
             "data": "synthetic (seeded, device-generated)", "config": config,
             "gpu_launches": runner.launches_per_step() * args.steps,
             "e2e": {"value": w.B * world / e2e_s, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h},
+                    "d2h_bytes_per_step": d2h, "cuda_graph": not args.no_graph},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": captured_traffic(args.workload),
                          "kernel": "mkv_decode_attention (one fused split-KV decode kernel), one layer",
