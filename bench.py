@@ -103,6 +103,40 @@ class ClockSampler:
 
 # --------------------------------------------------------------------------- GPU arm
 
+# Algorithmic bytes of one decode launch of one layer (the compressed-KV bytes the method must read),
+# per (batch, kv-head) unit: the roofline's numerator.
+
+def alg_bytes_fp16(units: int, T: int, D: int) -> int:
+    """K and V rows of the T tokens, fp16."""
+    return units * T * D * 2 * 2
+
+
+def alg_bytes_kvquant(units: int, T: int, D: int, bits: int, n_v: int, n_key_outliers: int) -> int:
+    """Per token: key and value codes (D*bits/8 bytes each), the value range (lo, scale: 8 B), n_v
+    value outliers of 4 B and the key-outlier CSR offset (4 B); plus 4 B per key-outlier entry."""
+    return units * T * (2 * (D * bits // 8) + 8 + 4 * n_v + 4) + 4 * n_key_outliers
+
+
+def alg_bytes_h2o(units: int, held: int, D: int) -> int:
+    """K and V rows of the held slots, fp16."""
+    return units * held * D * 2 * 2
+
+
+def overhead_bytes_h2o(units: int, slots: int, G: int) -> int:
+    """What the H2O decode moves besides the model: each slot's position (4 B, the mask) and the G
+    fp32 logits it writes for the score update."""
+    return units * slots * (4 + 4 * G)
+
+
+def alg_bytes_rocket(units: int, n: int, D: int, k_p: int, r_d: int, page: int = 16) -> int:
+    """The full pages before the newest token's page are candidates; per candidate page the chosen
+    r_d dims' min and max (fp16); K and V rows of the k_p chosen pages and of the tail page (the
+    newest token's, 1..page tokens)."""
+    ns = (n - 1) // page if n > 0 else 0
+    tail = n - page * ns
+    return units * ((min(k_p, ns) * page + tail) * D * 2 * 2 + ns * r_d * 2 * 2)
+
+
 class Runner:
     """All layers of one workload resident on the device, plus the step."""
 
@@ -389,24 +423,17 @@ class Runner:
         units = w.B * w.Hkv
         T = int(cache.t["T_len"][0])
         if self.method == "fp16":
-            return units * T * w.D * 2 * 2, T, 0
+            return alg_bytes_fp16(units, T, w.D), T, 0
         if self.method == "kvquant":
             nv = self.mkv.n_value_outliers(w.D, w.outlier_frac)
-            per_tok = 2 * (w.D * w.bits // 8) + 8 + 4 * nv + 4
             n_kout = int(cache.t["k_out_off"][:, :, T].sum())
-            return units * T * per_tok + 4 * n_kout, T, 0
+            return alg_bytes_kvquant(units, T, w.D, w.bits, nv, n_kout), T, 0
         if self.method == "h2o":
             held = int(cache.t["pos"][0, 0].ge(0).sum())
-            # K and V rows of the held slots; the slot's position (mask) and the G logits written for
-            # the score update are overhead
-            return units * held * w.D * 2 * 2, held, units * self.T_cap * (4 + 4 * w.G)
-        n = T
-        ns = (n - 1) // 16
-        tail = n - 16 * ns
-        # the attended pages' K and V rows, and the chosen dims' min/max of every candidate page
-        alg = units * ((min(w.topk_pages, ns) * 16 + tail) * w.D * 2 * 2 + ns * w.topq_dims * 2 * 2)
-        # the bounds of the other dims, which the fused step reads before the dims are chosen
-        return alg, n, units * ns * (w.D - w.topq_dims) * 2 * 2
+            slots = min(self.T_cap, w.h2o_heavy + w.h2o_recent + 1)
+            return alg_bytes_h2o(units, held, w.D), held, overhead_bytes_h2o(units, slots, w.G)
+        # the fused step reads only the chosen dims' page bounds: no overhead beyond the model
+        return alg_bytes_rocket(units, T, w.D, w.topk_pages, w.topq_dims), T, 0
 
 
 def time_steps(runner, steps, warmup):

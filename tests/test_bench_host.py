@@ -46,3 +46,50 @@ def test_prefill_scoring_flops_counts_causal_pairs():
         pos0 = T - rows
         pairs = sum(1 for i in range(rows) for j in range(T) if j <= pos0 + i)
         assert bench.prefill_scoring_flops(B, Hq, D, T, rows) == 2 * 2 * D * pairs * B * Hq
+
+
+def test_byte_models_match_per_element_counts():
+    """The roofline's algorithmic bytes (one decode launch of one layer) against a count that walks
+    the cache token by token, page by page and dim by dim: FP16 and H2O K/V rows, KVQuant codes,
+    value ranges, value outliers, CSR offsets and key-outlier entries, RocketKV candidate-page bounds
+    of the chosen dims plus the K/V rows of the chosen and the tail pages (incl. a cache shorter
+    than one page and one with fewer full pages than k_p)."""
+    import bench
+
+    def per_unit_fp16(T, D):
+        return sum(2 * D * 2 for _ in range(T))            # K row + V row per token
+
+    def per_unit_kvq(T, D, bits, n_v):
+        b = 0
+        for _ in range(T):
+            b += D * bits // 8                               # key codes
+            b += D * bits // 8                               # value codes
+            b += 4 + 4                                       # value lo, scale (fp32)
+            b += n_v * 4                                     # value outliers (channel << 16 | fp16)
+            b += 4                                           # the token's CSR offset
+        return b
+
+    def per_unit_rocket(n, D, k_p, r_d, page=16):
+        newest_page = (n - 1) // page
+        candidates = list(range(newest_page))               # full pages before the newest token's page
+        b = 0
+        for _ in candidates:
+            for _ in range(r_d):
+                b += 2 + 2                                   # min and max (fp16) of a chosen dim
+        chosen = candidates[:k_p]                            # how many, not which
+        for _ in chosen:
+            for _ in range(page):
+                b += 2 * D * 2
+        for _ in range(n - page * newest_page):              # the tail page's tokens
+            b += 2 * D * 2
+        return b
+
+    for units, T, D in [(64, 8193, 128), (1, 1, 64), (3, 77, 64)]:
+        assert bench.alg_bytes_fp16(units, T, D) == units * per_unit_fp16(T, D)
+        assert bench.alg_bytes_h2o(units, T, D) == units * per_unit_fp16(T, D)
+    for units, T, D, bits, n_v, n_out in [(64, 8198, 128, 4, 2, 81920), (2, 33, 64, 3, 1, 0), (5, 700, 128, 2, 13, 999)]:
+        assert bench.alg_bytes_kvquant(units, T, D, bits, n_v, n_out) == units * per_unit_kvq(T, D, bits, n_v) + 4 * n_out
+    for units, n, D, k_p, r_d in [(32, 4097, 128, 64, 32), (4, 1, 128, 64, 32), (4, 16, 64, 4, 16),
+                                   (4, 17, 64, 4, 16), (2, 100, 64, 64, 16), (2, 4100, 128, 128, 32)]:
+        assert bench.alg_bytes_rocket(units, n, D, k_p, r_d) == units * per_unit_rocket(n, D, k_p, r_d), (n, k_p)
+    assert bench.overhead_bytes_h2o(128, 3278, 4) == 128 * sum(4 + 4 * 4 for _ in range(3278))
