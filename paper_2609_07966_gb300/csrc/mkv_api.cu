@@ -423,22 +423,15 @@ mkv_status mkv_kvquant_step(const mkv_config* cfg, const mkv_quant_params* qpara
   MKV_REQUIRE(ws != nullptr && ws_bytes >= need.bytes, MKV_ERR_WORKSPACE,
               "workspace %zu bytes < %zu needed", ws_bytes, need.bytes);
   const Split sp = decode_split(*cfg, cache->T_cap);
-  // Each (CTA, unit) pair of batch entry b takes a ticket in the top 8 bits of T_len[b] (at most 255
-  // of them); a CTA keeps its units' lengths in 32-entry tables (it spans at most 28 of the <= 4096
-  // units).
+  // Each CTA that touches batch entry b takes one ticket in the top 8 bits of T_len[b] (at most
+  // n_cta <= 152 of them, within the 8 bits); a CTA keeps its units' lengths in 32-entry tables (it
+  // spans at most 28 of the <= 4096 units).
   const int64_t units = (int64_t)cfg->B * cfg->Hkv, cpu = sp.chunks_per_unit, c_tot = cpu * units;
-  int64_t max_tickets = 0;
-  for (int64_t b = 0; b < cfg->B; ++b) {
-    int64_t t = 0;
-    for (int64_t u = b * cfg->Hkv; u < (b + 1) * cfg->Hkv; ++u)
-      t += cta_of_chunk((u + 1) * cpu - 1, c_tot, sp.n_cta) - cta_of_chunk(u * cpu, c_tot, sp.n_cta) + 1;
-    max_tickets = std::max(max_tickets, t);
-  }
   const int64_t span = (ceil_div(c_tot, (int64_t)sp.n_cta) - 1) / cpu + 2;
-  MKV_REQUIRE(max_tickets <= 255 && span <= kvquant_step_max_units_per_cta(), MKV_ERR_UNSUPPORTED,
-              "kvquant_step: %lld CTA-unit pairs read one batch entry's length (at most 255) or a CTA spans %lld "
-              "units (at most %d); use mkv_quantize_kv + mkv_decode_attention",
-              (long long)max_tickets, (long long)span, kvquant_step_max_units_per_cta());
+  MKV_REQUIRE(sp.n_cta <= 255 && span <= kvquant_step_max_units_per_cta(), MKV_ERR_UNSUPPORTED,
+              "kvquant_step: %d CTAs read one batch entry's length (at most 255) or a CTA spans %lld units "
+              "(at most %d); use mkv_quantize_kv + mkv_decode_attention",
+              sp.n_cta, (long long)span, kvquant_step_max_units_per_cta());
   MKV_REQUIRE(cache->T_cap < (1 << 24), MKV_ERR_UNSUPPORTED,
               "kvquant_step needs T_cap < 2^24 (T_cap %lld); use mkv_quantize_kv + mkv_decode_attention",
               (long long)cache->T_cap);
