@@ -191,3 +191,25 @@ def test_kvquant_step_checks(L):
     st = L.mkv_kvquant_step(*args(kq, 80))
     assert st == mkv.MKV_ERR_UNSUPPORTED and "2^24" in mkv.mkv_last_error()
 
+
+
+def test_kvquant_step_accepts_the_tested_shapes(L):
+    """The host checks of mkv_kvquant_step let the shapes the GPU tests and the bench use through to
+    the launch (on a machine without a GPU the launch itself then fails with MKV_ERR_CUDA): many
+    one-chunk units per CTA, the 8 x 8K bench shape, a short cache and 128K at B = 1."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("would launch on the GPU")
+    for B, Hkv, T_cap in [(40, 4, 64), (8, 8, 8320), (3, 2, 256), (1, 8, 131072 + 200)]:
+        kq = mkv.config(mkv.MKV_KVQUANT, B, 4 * Hkv, Hkv, 128, bits=4)
+        qp = mkv.mkv_quant_params()
+        for name in ("t_lo", "t_hi", "k_lo", "k_scale", "k_dq", "v_tbl", "rope"):
+            setattr(qp, name, 1 << 20)
+        qp.k_cb, qp.v_cb, qp.rope_len = 1 << 20, 1 << 20, T_cap + 64
+        cache = mkv.mkv_cache()
+        cache.T_cap, cache.T_len = T_cap, 8
+        cache.k_codes, cache.v_codes, cache.v_params, cache.v_out = 1 << 12, 1 << 13, 1 << 14, 1 << 15
+        cache.k_out_off, cache.k_out, cache.k_out_cap = 1 << 16, 1 << 17, 4096
+        st = L.mkv_kvquant_step(ctypes.byref(kq), ctypes.byref(qp), 64, 80, 96, ctypes.byref(cache), 128, 4096,
+                                ctypes.c_size_t(1 << 40), None)
+        assert st == mkv.MKV_ERR_CUDA, (B, Hkv, T_cap, st, mkv.mkv_last_error())
