@@ -93,3 +93,26 @@ def test_byte_models_match_per_element_counts():
                                    (4, 17, 64, 4, 16), (2, 100, 64, 64, 16), (2, 4100, 128, 128, 32)]:
         assert bench.alg_bytes_rocket(units, n, D, k_p, r_d) == units * per_unit_rocket(n, D, k_p, r_d), (n, k_p)
     assert bench.overhead_bytes_h2o(128, 3278, 4) == 128 * sum(4 + 4 * 4 for _ in range(3278))
+
+
+def test_reference_arm_prints_the_contract_line():
+    """`bench.py --impl reference` (the fp64 oracle on the host cores, a bounded sample of the headline
+    workload) prints one JSON line with the contract's keys, its cpu_baseline and a zero-copy e2e."""
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--steps", "1", "--warmup", "0",
+                          "--cpu-budget", "1"], cwd=root, capture_output=True, text=True, timeout=600)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
+                "scaling", "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
+        assert key in line, key
+    assert line["impl"] == "reference" and line["value"] > 0 and line["higher_is_better"] is True
+    assert line["config"]["workload"] == "kvquant_nuq4_b8_t8192"
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == line["value"] and cb["sample"]
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"], "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
